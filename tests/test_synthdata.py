@@ -1,0 +1,62 @@
+"""The seeded input generator: known-answer Philox block, shapes and
+invariants of the drawn CSR, reproducibility across thread counts."""
+import numpy as np
+import pytest
+
+import synthdata
+
+
+def test_philox_known_answer():
+    # Philox4x32-10 with zero counter and key (Salmon et al., SC'11 test vector)
+    out = synthdata.philox4x32_10([0, 0, 0, 0], [0, 0])
+    assert [hex(int(x)) for x in out] == ["0x6627e8d5", "0xe169c58d", "0xbc57ac4c", "0x9b00dbd8"]
+
+
+@pytest.mark.parametrize("name,kw", [
+    ("tiny", {}),
+    ("zipf-1m", dict(n_rows=20000)),
+    ("ctr", dict(n_rows=20000, n_cols=200000)),
+    ("low-conflict", dict(n_rows=20000, n_cols=1_000_000)),
+    ("deep-chain", dict(n_rows=2000)),
+])
+def test_workload_shape(name, kw):
+    p = synthdata.generate(name, **kw)
+    spec = dict(synthdata.WORKLOADS[name], **kw)
+    k = spec["k"]
+    assert p.n_rows == spec["n_rows"] and p.nnz == p.n_rows * k
+    assert np.array_equal(p.row_ptr, np.arange(p.n_rows + 1) * k)
+    rows = p.col.reshape(p.n_rows, k)
+    assert np.all(np.diff(rows, axis=1) > 0)            # distinct and ascending in every row
+    assert p.col.min() >= 0 and p.col.max() < p.n_cols
+    if spec["vals"] == "ones":
+        assert p.val is None
+    elif spec["vals"] == "uniform":
+        assert p.val.min() >= -1 and p.val.max() < 1
+    if spec["labels"] in ("sign", "bernoulli"):
+        assert set(np.unique(p.y).tolist()) <= {-1.0, 1.0}
+    assert p.y.dtype == np.float32 and np.all(np.isfinite(p.y))
+
+
+def test_deterministic_across_threads():
+    a = synthdata.generate("zipf-1m", n_rows=5000, nthreads=1)
+    b = synthdata.generate("zipf-1m", n_rows=5000, nthreads=7)
+    assert np.array_equal(a.col, b.col) and np.array_equal(a.val, b.val) and np.array_equal(a.y, b.y)
+    c = synthdata.generate("zipf-1m", n_rows=5000, seed=99)
+    assert not np.array_equal(a.col, c.col)
+
+
+def test_zipf_head_frequency():
+    # P(top id in a row) for k draws-without-repeats is close to 1-(1-p1)^k for small p1
+    p = synthdata.generate("zipf-1m", n_rows=20000)
+    s, F, k = 1.0, p.n_cols, 20
+    p1 = 1.0 / np.sum(np.arange(1, F + 1, dtype=np.float64) ** -s)
+    top = np.bincount(p.col, minlength=F).argmax()
+    frac = np.mean([(p.col[p.row_ptr[t]:p.row_ptr[t + 1]] == top).any() for t in range(p.n_rows)])
+    assert abs(frac - (1 - (1 - p1) ** k)) < 0.03
+
+
+def test_ragged_rows():
+    p = synthdata.generate("tiny", n_rows=2000, k_lo=0, k=12)
+    lens = np.diff(p.row_ptr)
+    assert lens.min() == 0 and lens.max() == 12
+    assert abs(lens.mean() - 6) < 0.5
