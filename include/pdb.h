@@ -1,0 +1,211 @@
+/*
+ * pdb.h -- C ABI of libpdb: serially-equivalent sparse SGD on one GPU.
+ *
+ * The method is data-centric synchronization (Parameter Database): each
+ * training example's sparse SGD update is a transaction whose read and write
+ * set is the example's nonzero features.  Examples that share no feature run
+ * concurrently; examples that share one run in data order, so the trained
+ * weights equal those of sequential SGD over the data in its given order.
+ *
+ * Paper anchors (the paper's own section, definition and algorithm labels):
+ *   Definition 1   parameter database M(Theta, D): D immutable, Theta mutable
+ *   Definition 2   chunks (here: single features)
+ *   Definition 3   an iteration reads its chunks, then writes them
+ *   Algorithm 1,   the sequential computation every result must equal
+ *   Definition 4
+ *   Algorithm 2a   BSP: read barrier, reads, compute, write barrier, writes
+ *   Algorithm 2b   relaxed: per-chunk Read and Write Constraints (Sec. 4.4)
+ *   Theorem 2      RC + WC give the sequential result
+ *   Theorem 3      BSP executions are a subset of RC/WC executions
+ *   Section 5      read protocol: a per-chunk iteration number gates reads
+ *
+ * Conventions for every call:
+ *   - Pointers named as device pointers must be device memory of the current
+ *     CUDA device; the caller owns them and keeps them alive until the work
+ *     queued on `stream` has finished.
+ *   - `stream` is a cudaStream_t passed as void*; NULL is the legacy default
+ *     stream.  Every call only enqueues work on `stream` (asynchronous),
+ *     except where a comment says it synchronizes.
+ *   - Return value: PDB_OK or a negative PDB_E* code for errors found on the
+ *     host (arguments, allocation, launch).  Errors found by the kernels
+ *     (bad CSR contents, expired waits) are recorded in the conflicts
+ *     handle's device status word; read it with pdb_status().  Once a handle
+ *     holds an error, later kernels that use it return at once and the
+ *     handle must be rebuilt.
+ *   - Calls that share a handle must be ordered on one stream (the handles
+ *     hold device-side counters that a concurrent call would clobber).
+ *   - Limits: n_rows, n_cols and nnz below 2^31 (positions and ids are int32).
+ */
+#ifndef PDB_H
+#define PDB_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* ---------------------------------------------------------------- errors */
+#define PDB_OK 0
+#define PDB_EINVAL (-1)   /* null pointer, negative size, row_ptr not nondecreasing from 0 to nnz, size mismatch */
+#define PDB_ERANGE (-2)   /* a feature id outside [0, n_cols) */
+#define PDB_EDUP (-3)     /* a feature id repeated inside one example (read/write sets are sets, Def. 3) */
+#define PDB_ENOMEM (-4)   /* device allocation failed */
+#define PDB_ECUDA (-5)    /* a CUDA runtime call or launch failed */
+#define PDB_ETIMEOUT (-6) /* a bounded device-side wait expired (the kernel stopped, the GPU stays usable) */
+#define PDB_EFAULT (-7)   /* an internal invariant failed on the device */
+#define PDB_ESTATE (-8)   /* wrong handle for this call (e.g. a READY schedule where levels are needed) */
+
+/* ---------------------------------------------------------------- types */
+
+/* The data D of the parameter database M(Theta, D) (Definition 1): n_rows
+ * examples in CSR form over n_cols features.  Example t holds the features
+ * col[row_ptr[t] .. row_ptr[t+1]) with values val[...] (val == NULL means
+ * every value is 1.0, binary features).  Device pointers, caller-owned,
+ * never written by the library.  Example order is the data order that the
+ * result must reproduce.  Rows may be empty; ids in a row must be distinct
+ * (any order). */
+typedef struct {
+    int64_t n_rows, n_cols, nnz;
+    const int64_t *row_ptr; /* [n_rows + 1] */
+    const int32_t *col;     /* [nnz] */
+    const float *val;       /* [nnz] or NULL */
+} pdb_csr;
+
+/* Loss term f_t of example t as a function of its margin m = w . x_t
+ * (Eq. 2's data terms; the regularizer g is not supported).
+ *   LOGISTIC  f = log(1 + exp(-y m)),  y in {-1, +1}
+ *   SQUARED   f = (m - y)^2 / 2
+ *   HINGE     f = max(0, 1 - y m), subgradient 0 at y m = 1 */
+typedef enum { PDB_LOSS_LOGISTIC = 0, PDB_LOSS_SQUARED = 1, PDB_LOSS_HINGE = 2 } pdb_loss;
+
+/* How pdb_sgd_epoch keeps conflicting examples in data order.
+ *   LEVELS  dependency levels: level-synchronous execution, one grid barrier
+ *           per level (each level is one BSP step over disjoint examples,
+ *           Theorem 3)
+ *   READY   per-feature ready counters: an occurrence of feature j with rank
+ *           r reads w_j once the counter of j equals r and sets it to r + 1
+ *           after writing (the read protocol of Section 5 with the
+ *           iteration number counted per feature); no barrier at all */
+typedef enum { PDB_SCHED_LEVELS = 0, PDB_SCHED_READY = 1 } pdb_sched_mode;
+
+/* Launch and wait options; a zeroed struct (or NULL) selects the defaults. */
+typedef struct {
+    int32_t blocks_per_sm;     /* persistent grid = blocks_per_sm x #SM; 0 = occupancy maximum */
+    int32_t reserved0;
+    double wait_timeout_s;     /* limit of every device-side wait; 0 = 2 seconds */
+} pdb_opts;
+
+/* Sizes and timings; timings are CUDA-event milliseconds of the last call of
+ * each kind on the given handles (0 when not run). */
+typedef struct {
+    int64_t n_rows, n_cols, nnz;
+    int64_t n_levels;        /* LEVELS schedule: number of levels L; else -1 */
+    int64_t max_level_width; /* LEVELS schedule: largest level; else -1 */
+    int64_t max_chain;       /* most occurrences of one feature (longest per-feature chain) */
+    double ms_build, ms_schedule, ms_sgd, ms_bsp;
+} pdb_stats;
+
+typedef struct pdb_conflicts pdb_conflicts; /* opaque, library-owned device arrays */
+typedef struct pdb_schedule pdb_schedule;   /* opaque, library-owned device arrays */
+
+/* ---------------------------------------------------------------- calls */
+
+/* Conflict structure of D (Definitions 2-3; read protocol of Section 5).
+ * Validates X on the device (row_ptr, id range, no repeated id in a row),
+ * stable-sorts the (feature, position) pairs by feature and links
+ * consecutive occurrences of each feature into a chain:
+ *   csc_pos[nnz]    positions grouped by feature, data order inside a feature
+ *   feat_ptr[F+1]   feature j occupies csc_pos[feat_ptr[j] .. feat_ptr[j+1])
+ *   prev[p], next[p] previous / next position holding col[p], -1 if none
+ *   rank[p]         number of earlier positions holding col[p]
+ * *out receives a new handle (free with pdb_conflicts_free) even when the
+ * device later reports a CSR error through pdb_status.  Allocates its arrays
+ * stream-ordered on `stream`. */
+int pdb_build_conflicts(const pdb_csr *X, pdb_conflicts **out, void *stream);
+
+/* Borrowed device pointers into the handle (valid until it is freed).  Any
+ * output pointer may be NULL. */
+int pdb_conflicts_arrays(const pdb_conflicts *c, const int32_t **csc_pos, const int64_t **feat_ptr,
+                         const int32_t **prev, const int32_t **next, const int32_t **rank);
+
+/* Schedule for pdb_sgd_epoch.
+ *   LEVELS: level[t] = 1 + max over features j of t with an earlier
+ *     occurrence of level[row of that occurrence], 0 if none (longest
+ *     conflict path), computed by a Kahn-style frontier sweep; order[N] lists
+ *     the examples by level, ascending id inside a level; level_ptr[L+1]
+ *     delimits the levels.
+ *   READY: the per-feature ready counters (zeroed here; the last occurrence
+ *     of each feature in an epoch hands its counter back to 0) and, per
+ *     position, the counter value it waits for.
+ * Allocates stream-ordered on `stream`. */
+int pdb_schedule_build(const pdb_conflicts *c, pdb_sched_mode mode, pdb_schedule **out, void *stream);
+
+/* LEVELS schedule arrays (borrowed device pointers, any may be NULL) and the
+ * level count.  SYNCHRONIZES `stream` to read L from the device.
+ * PDB_ESTATE for a READY schedule. */
+int pdb_schedule_levels(const pdb_schedule *s, const int32_t **level, const int32_t **order,
+                        const int64_t **level_ptr, int64_t *n_levels, void *stream);
+
+/* READY schedule arrays (borrowed device pointers, any may be NULL):
+ * ctr[n_cols] the per-feature ready counters (0 between calls), gate[nnz]
+ * the counter value each position waits for (its rank) with bit 31 set on
+ * the last occurrence of its feature.  PDB_ESTATE for a LEVELS schedule. */
+int pdb_schedule_ready(const pdb_schedule *s, const uint32_t **ctr, const uint32_t **gate);
+
+/* n_epochs passes of SGD over X in data order (Algorithm 1 with one
+ * iteration per example), run concurrently under the schedule's constraint.
+ * w (device, n_cols floats, caller-owned) is read and updated in place; y
+ * (device, n_rows floats) are the labels.  For every example t:
+ *   m = w . x_t         32 partial sums: element i of the row adds into
+ *                       partial i mod 32 with a fused multiply-add, then
+ *                       the partials combine pairwise (xor 16, 8, 4, 2, 1)
+ *   g = dloss/dm (m, y) fp32; logistic uses exp by Cody-Waite reduction and
+ *                       a degree-7 Taylor polynomial
+ *   w_j = w_j - (eta*g) * x_tj  for the features of t
+ * Each fp32 operation is rounded once, so the result is bitwise the same for
+ * every schedule and equals the sequential run (Theorem 2).
+ * X and c must be the same data the schedule was built from. */
+int pdb_sgd_epoch(const pdb_csr *X, const float *y, const pdb_conflicts *c, const pdb_schedule *s, float *w,
+                  pdb_loss loss, float eta, int n_epochs, const pdb_opts *opts, void *stream);
+
+/* BSP comparison (Algorithm 2a with `batch` examples between barriers):
+ * per batch [b*B, min((b+1)*B, N)) every example computes c_i = eta *
+ * dloss/dm at the weights of the batch start (read barrier), then each
+ * feature j takes delta_j = sum over the batch's examples, ascending, of
+ * c_i * x_ij and w_j = w_j - delta_j (write barrier).  batch = 1 equals
+ * sequential SGD (Theorem 1).  Allocates per-call scratch stream-ordered. */
+int pdb_bsp_epoch(const pdb_csr *X, const float *y, const pdb_conflicts *c, float *w, pdb_loss loss, float eta,
+                  int64_t batch, int n_epochs, const pdb_opts *opts, void *stream);
+
+/* SYNCHRONIZES `stream` and returns the device status of handle c: PDB_OK
+ * or the first error a kernel recorded (PDB_EINVAL, PDB_ERANGE, PDB_EDUP,
+ * PDB_ETIMEOUT, PDB_EFAULT); PDB_ECUDA if the synchronization itself fails. */
+int pdb_status(const pdb_conflicts *c, void *stream);
+
+/* Sizes and timings; SYNCHRONIZES (device) to read the event timers and L.
+ * s may be NULL. */
+int pdb_get_stats(const pdb_conflicts *c, const pdb_schedule *s, pdb_stats *out);
+
+/* Release a handle (waits for the device, then frees its arrays). */
+void pdb_conflicts_free(pdb_conflicts *c);
+void pdb_schedule_free(pdb_schedule *s);
+
+/* Text of an error code. */
+const char *pdb_strerror(int code);
+
+/* ---------------------------------------------------------------- utilities */
+
+/* cudaMemcpyAsync with the kind inferred from the pointers (for bindings that
+ * need to read the borrowed arrays). */
+int pdb_memcpy(void *dst, const void *src, size_t bytes, void *stream);
+
+/* out[i] = the library's device exp of x[i] (device arrays of n floats), the
+ * same function the logistic gradient uses. */
+int pdb_eval_expf(const float *x, float *out, int64_t n, void *stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* PDB_H */

@@ -1,0 +1,297 @@
+"""Python binding of libpdb (serially-equivalent sparse SGD on one GPU).
+
+Argument marshalling only: every step of the method runs in the CUDA kernels
+of ``csrc/`` behind the C ABI declared in ``include/pdb.h``.  The functions
+below carry the C names and forward torch tensors' device pointers and the
+current CUDA stream.  There is no CPU fallback: if the compiled library is
+missing or cannot load, every call raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import glob
+import os
+import subprocess
+import threading
+from concurrent.futures import ThreadPoolExecutor
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_ROOT = os.path.dirname(_HERE)
+_CSRC = os.path.join(_HERE, "csrc")
+_INCLUDE = os.path.join(_ROOT, "include")
+_LIBDIR = os.path.join(_HERE, "_lib")
+LIB_PATH = os.path.join(_LIBDIR, "libpdb.so")
+ARCH = "-gencode=arch=compute_103a,code=sm_103a"
+NVCC_FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-fmad=false", "-Xcompiler", "-fPIC", ARCH, f"-I{_INCLUDE}"]
+
+PDB_OK, PDB_EINVAL, PDB_ERANGE, PDB_EDUP, PDB_ENOMEM, PDB_ECUDA, PDB_ETIMEOUT, PDB_EFAULT, PDB_ESTATE = \
+    0, -1, -2, -3, -4, -5, -6, -7, -8
+PDB_LOSS_LOGISTIC, PDB_LOSS_SQUARED, PDB_LOSS_HINGE = 0, 1, 2
+PDB_SCHED_LEVELS, PDB_SCHED_READY = 0, 1
+
+_lock = threading.Lock()
+_lib = None
+
+
+class PdbError(RuntimeError):
+    def __init__(self, code: int, what: str = ""):
+        self.code = code
+        msg = _strerror(code)
+        super().__init__(f"{what}: {msg} ({code})" if what else f"{msg} ({code})")
+
+
+def _sources():
+    return sorted(glob.glob(os.path.join(_CSRC, "*.cu")))
+
+
+def _deps():
+    return _sources() + glob.glob(os.path.join(_CSRC, "*.cuh")) + [os.path.join(_INCLUDE, "pdb.h")]
+
+
+def build(force: bool = False, verbose: bool = False) -> str:
+    """Compile libpdb.so in-tree for sm_103a (nvcc, one object per .cu, in parallel)."""
+    with _lock:
+        os.makedirs(_LIBDIR, exist_ok=True)
+        if (not force and os.path.exists(LIB_PATH)
+                and os.path.getmtime(LIB_PATH) >= max(os.path.getmtime(p) for p in _deps())):
+            return LIB_PATH
+        objs = []
+
+        def compile_one(src):
+            obj = os.path.join(_LIBDIR, os.path.basename(src)[:-3] + f".{os.getpid()}.o")
+            cmd = ["nvcc", *NVCC_FLAGS, "-c", src, "-o", obj]
+            if verbose:
+                cmd += ["-Xptxas", "-v"]
+            r = subprocess.run(cmd, capture_output=True, text=True)
+            if r.returncode != 0:
+                raise RuntimeError(f"nvcc failed for {src}:\n{r.stderr}")
+            if verbose:
+                print(r.stderr)
+            return obj
+
+        with ThreadPoolExecutor(max_workers=len(_sources())) as ex:
+            objs = list(ex.map(compile_one, _sources()))
+        tmp = f"{LIB_PATH}.{os.getpid()}.tmp"
+        r = subprocess.run(["nvcc", "-shared", ARCH, "-o", tmp, *objs], capture_output=True, text=True)
+        for o in objs:
+            os.remove(o)
+        if r.returncode != 0:
+            raise RuntimeError(f"link of libpdb.so failed:\n{r.stderr}")
+        os.replace(tmp, LIB_PATH)
+        return LIB_PATH
+
+
+class pdb_csr(ctypes.Structure):
+    _fields_ = [("n_rows", ctypes.c_int64), ("n_cols", ctypes.c_int64), ("nnz", ctypes.c_int64),
+                ("row_ptr", ctypes.c_void_p), ("col", ctypes.c_void_p), ("val", ctypes.c_void_p)]
+
+
+class pdb_opts(ctypes.Structure):
+    _fields_ = [("blocks_per_sm", ctypes.c_int32), ("reserved0", ctypes.c_int32),
+                ("wait_timeout_s", ctypes.c_double)]
+
+
+class pdb_stats(ctypes.Structure):
+    _fields_ = [("n_rows", ctypes.c_int64), ("n_cols", ctypes.c_int64), ("nnz", ctypes.c_int64),
+                ("n_levels", ctypes.c_int64), ("max_level_width", ctypes.c_int64), ("max_chain", ctypes.c_int64),
+                ("ms_build", ctypes.c_double), ("ms_schedule", ctypes.c_double), ("ms_sgd", ctypes.c_double),
+                ("ms_bsp", ctypes.c_double)]
+
+    def as_dict(self):
+        return {k: getattr(self, k) for k, _ in self._fields_}
+
+
+EXPORTS = ["pdb_build_conflicts", "pdb_conflicts_arrays", "pdb_schedule_build", "pdb_schedule_levels",
+           "pdb_schedule_ready",
+           "pdb_sgd_epoch", "pdb_bsp_epoch", "pdb_status", "pdb_get_stats", "pdb_conflicts_free",
+           "pdb_schedule_free", "pdb_strerror", "pdb_memcpy", "pdb_eval_expf"]
+
+
+def load(path: str | None = None):
+    """Load libpdb.so (building it first if it is absent or stale); raises if that fails."""
+    global _lib
+    if _lib is None:
+        lib = ctypes.CDLL(path or build())
+        P, I64, I32 = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int
+        PP = ctypes.POINTER(ctypes.c_void_p)
+        lib.pdb_build_conflicts.argtypes = [ctypes.POINTER(pdb_csr), PP, P]
+        lib.pdb_conflicts_arrays.argtypes = [P, PP, PP, PP, PP, PP]
+        lib.pdb_schedule_build.argtypes = [P, I32, PP, P]
+        lib.pdb_schedule_levels.argtypes = [P, PP, PP, PP, ctypes.POINTER(I64), P]
+        lib.pdb_schedule_ready.argtypes = [P, PP, PP]
+        lib.pdb_sgd_epoch.argtypes = [ctypes.POINTER(pdb_csr), P, P, P, P, I32, ctypes.c_float, I32,
+                                      ctypes.POINTER(pdb_opts), P]
+        lib.pdb_bsp_epoch.argtypes = [ctypes.POINTER(pdb_csr), P, P, P, I32, ctypes.c_float, I64, I32,
+                                      ctypes.POINTER(pdb_opts), P]
+        lib.pdb_status.argtypes = [P, P]
+        lib.pdb_get_stats.argtypes = [P, P, ctypes.POINTER(pdb_stats)]
+        lib.pdb_conflicts_free.argtypes = [P]
+        lib.pdb_conflicts_free.restype = None
+        lib.pdb_schedule_free.argtypes = [P]
+        lib.pdb_schedule_free.restype = None
+        lib.pdb_strerror.argtypes = [I32]
+        lib.pdb_strerror.restype = ctypes.c_char_p
+        lib.pdb_memcpy.argtypes = [P, P, ctypes.c_size_t, P]
+        lib.pdb_eval_expf.argtypes = [P, P, I64, P]
+        _lib = lib
+    return _lib
+
+
+def _strerror(code: int) -> str:
+    try:
+        return load().pdb_strerror(int(code)).decode()
+    except Exception:  # the library itself failed to load
+        return f"error {code}"
+
+
+def _check(rc: int, what: str):
+    if rc != PDB_OK:
+        raise PdbError(rc, what)
+
+
+def _stream(stream):
+    if stream is None:
+        import torch
+        return ctypes.c_void_p(torch.cuda.current_stream().cuda_stream)
+    if isinstance(stream, int):
+        return ctypes.c_void_p(stream)
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+class Csr:
+    """CSR examples on the device: int64 row_ptr, int32 col, float32 val (or None)."""
+
+    def __init__(self, row_ptr, col, val, n_cols: int):
+        self.row_ptr, self.col, self.val, self.n_cols = row_ptr, col, val, int(n_cols)
+        self.struct = pdb_csr(row_ptr.numel() - 1, self.n_cols, col.numel(), _ptr(row_ptr), _ptr(col), _ptr(val))
+
+    @classmethod
+    def from_problem(cls, problem, device="cuda"):
+        import torch
+        row_ptr = torch.from_numpy(problem.row_ptr).to(device)
+        col = torch.from_numpy(problem.col).to(device)
+        val = None if problem.val is None else torch.from_numpy(problem.val).to(device)
+        return cls(row_ptr, col, val, problem.n_cols)
+
+
+class Conflicts:
+    """Owns a pdb_conflicts handle."""
+
+    def __init__(self, handle, n_rows, n_cols, nnz):
+        self.handle = handle
+        self.n_rows, self.n_cols, self.nnz = n_rows, n_cols, nnz
+
+    def __del__(self):
+        if getattr(self, "handle", None) and _lib is not None:
+            _lib.pdb_conflicts_free(self.handle)
+            self.handle = None
+
+
+class Schedule:
+    """Owns a pdb_schedule handle (keeps its conflicts alive)."""
+
+    def __init__(self, handle, conflicts, mode):
+        self.handle, self.conflicts, self.mode = handle, conflicts, mode
+
+    def __del__(self):
+        if getattr(self, "handle", None) and _lib is not None:
+            _lib.pdb_schedule_free(self.handle)
+            self.handle = None
+
+
+def pdb_build_conflicts(X: Csr, stream=None) -> Conflicts:
+    h = ctypes.c_void_p()
+    _check(load().pdb_build_conflicts(ctypes.byref(X.struct), ctypes.byref(h), _stream(stream)),
+           "pdb_build_conflicts")
+    return Conflicts(h, X.struct.n_rows, X.struct.n_cols, X.struct.nnz)
+
+
+def pdb_conflicts_arrays(c: Conflicts) -> dict:
+    """Borrowed device pointers (ints) of csc_pos, feat_ptr, prev, next, rank."""
+    ptrs = [ctypes.c_void_p() for _ in range(5)]
+    _check(load().pdb_conflicts_arrays(c.handle, *[ctypes.byref(p) for p in ptrs]), "pdb_conflicts_arrays")
+    return dict(zip(["csc_pos", "feat_ptr", "prev", "next", "rank"], [p.value for p in ptrs]))
+
+
+def pdb_schedule_build(c: Conflicts, mode: int, stream=None) -> Schedule:
+    h = ctypes.c_void_p()
+    _check(load().pdb_schedule_build(c.handle, int(mode), ctypes.byref(h), _stream(stream)), "pdb_schedule_build")
+    return Schedule(h, c, mode)
+
+
+def pdb_schedule_levels(s: Schedule, stream=None) -> dict:
+    ptrs = [ctypes.c_void_p() for _ in range(3)]
+    L = ctypes.c_int64()
+    _check(load().pdb_schedule_levels(s.handle, *[ctypes.byref(p) for p in ptrs], ctypes.byref(L), _stream(stream)),
+           "pdb_schedule_levels")
+    return dict(level=ptrs[0].value, order=ptrs[1].value, level_ptr=ptrs[2].value, n_levels=L.value)
+
+
+def pdb_schedule_ready(s: Schedule) -> dict:
+    """Borrowed device pointers (ints) of the READY schedule's ctr and gate arrays."""
+    ptrs = [ctypes.c_void_p() for _ in range(2)]
+    _check(load().pdb_schedule_ready(s.handle, *[ctypes.byref(p) for p in ptrs]), "pdb_schedule_ready")
+    return dict(ctr=ptrs[0].value, gate=ptrs[1].value)
+
+
+def _opts(opts):
+    if opts is None:
+        return None
+    if isinstance(opts, pdb_opts):
+        return ctypes.byref(opts)
+    return ctypes.byref(pdb_opts(**opts))
+
+
+def pdb_sgd_epoch(X: Csr, y, c: Conflicts, s: Schedule, w, loss: int, eta: float, n_epochs: int, opts=None,
+                  stream=None):
+    _check(load().pdb_sgd_epoch(ctypes.byref(X.struct), _ptr(y), c.handle, s.handle, _ptr(w), int(loss), float(eta),
+                                int(n_epochs), _opts(opts), _stream(stream)), "pdb_sgd_epoch")
+
+
+def pdb_bsp_epoch(X: Csr, y, c: Conflicts, w, loss: int, eta: float, batch: int, n_epochs: int, opts=None,
+                  stream=None):
+    _check(load().pdb_bsp_epoch(ctypes.byref(X.struct), _ptr(y), c.handle, _ptr(w), int(loss), float(eta),
+                                int(batch), int(n_epochs), _opts(opts), _stream(stream)), "pdb_bsp_epoch")
+
+
+def pdb_status(c: Conflicts, stream=None) -> int:
+    return int(load().pdb_status(c.handle, _stream(stream)))
+
+
+def pdb_get_stats(c: Conflicts, s: Schedule | None = None) -> dict:
+    st = pdb_stats()
+    _check(load().pdb_get_stats(c.handle, None if s is None else s.handle, ctypes.byref(st)), "pdb_get_stats")
+    return st.as_dict()
+
+
+def pdb_memcpy(dst_ptr: int, src_ptr: int, nbytes: int, stream=None):
+    _check(load().pdb_memcpy(ctypes.c_void_p(dst_ptr), ctypes.c_void_p(src_ptr), int(nbytes), _stream(stream)),
+           "pdb_memcpy")
+
+
+def pdb_eval_expf(x, out, stream=None):
+    _check(load().pdb_eval_expf(_ptr(x), _ptr(out), x.numel(), _stream(stream)), "pdb_eval_expf")
+
+
+def pdb_strerror(code: int) -> str:
+    return _strerror(code)
+
+
+def device_array(ptr: int, n: int, dtype, stream=None):
+    """Copy n elements of a borrowed device array into a new torch tensor."""
+    import torch
+    out = torch.empty(n, dtype=dtype, device="cuda")
+    if n:
+        pdb_memcpy(out.data_ptr(), ptr, n * out.element_size(), stream)
+    return out
+
+
+def check_status(c: Conflicts, stream=None):
+    """Synchronize and raise PdbError if a kernel recorded an error in c."""
+    rc = pdb_status(c, stream)
+    if rc != PDB_OK:
+        raise PdbError(rc, "device status")

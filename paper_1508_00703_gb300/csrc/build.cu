@@ -1,0 +1,501 @@
+// Conflict structure and schedules: pdb_build_conflicts, pdb_schedule_build
+// and the handle utilities of the C ABI.
+//
+// The read protocol of Section 5 keeps one iteration number per chunk and
+// lets a read of iteration alpha+1 proceed once the chunk's number is alpha.
+// With chunk = feature and iteration = example, that number becomes the
+// per-feature occurrence rank, and the constraint links each occurrence to
+// the previous occurrence of its feature: the chains built here.
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cstdlib>
+#include <cstring>
+#include <new>
+
+#include "common.cuh"
+
+using namespace pdb;
+
+namespace {
+
+// row_ptr[0] = 0, row_ptr[N] = nnz, nondecreasing (Definition 1: D is a list of examples)
+__global__ void k_validate_rows(const int64_t *__restrict__ row_ptr, int64_t n_rows, int64_t nnz, int *status)
+{
+    for (int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; t <= n_rows;
+         t += (int64_t)gridDim.x * blockDim.x) {
+        int64_t a = row_ptr[t];
+        bool bad = (t == 0 && a != 0) || (t == n_rows && a != nnz) || (t < n_rows && row_ptr[t + 1] < a) ||
+                   a < 0 || a > nnz;
+        if (bad) set_status(status, PDB_EINVAL);
+    }
+}
+
+// ids in [0, n_cols)
+__global__ void k_validate_cols(const int32_t *__restrict__ col, int64_t nnz, int64_t n_cols, int *status)
+{
+    bool bad = false;
+    for (int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; p < nnz; p += (int64_t)gridDim.x * blockDim.x) {
+        int32_t j = col[p];
+        bad |= (j < 0) || ((int64_t)j >= n_cols);
+    }
+    if (__any_sync(FULL, bad) && bad) set_status(status, PDB_ERANGE);
+}
+
+// row_of[p] = example holding position p (one warp per example)
+__global__ void k_row_of(const int64_t *__restrict__ row_ptr, int64_t n_rows, int32_t *__restrict__ row_of,
+                         const int *status)
+{
+    if (read_status(status)) return;
+    const int lane = threadIdx.x & 31;
+    const int64_t gw = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    for (int64_t t = gw; t < n_rows; t += nw) {
+        int64_t b = row_ptr[t], e = row_ptr[t + 1];
+        for (int64_t p = b + lane; p < e; p += 32) row_of[p] = (int32_t)t;
+    }
+}
+
+// Chains from the feature-sorted positions: slot s of feature j's run links
+// to its neighbours in the run; rank = offset inside the run.
+__global__ void k_link(const uint32_t *__restrict__ skey, const int32_t *__restrict__ spos, int64_t nnz,
+                       const int64_t *__restrict__ feat_ptr, int32_t *__restrict__ prev, int32_t *__restrict__ next,
+                       int32_t *__restrict__ rank, int *max_chain, const int *status)
+{
+    if (read_status(status)) return;
+    int longest = 0;
+    for (int64_t s = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; s < nnz; s += (int64_t)gridDim.x * blockDim.x) {
+        uint32_t j = skey[s];
+        int32_t p = spos[s];
+        bool first = s == 0 || skey[s - 1] != j;
+        bool last = s == nnz - 1 || skey[s + 1] != j;
+        int32_t r = (int32_t)(s - feat_ptr[j]);
+        prev[p] = first ? -1 : spos[s - 1];
+        next[p] = last ? -1 : spos[s + 1];
+        rank[p] = r;
+        if (last) longest = max(longest, r + 1);
+    }
+    for (int off = 16; off >= 1; off >>= 1) longest = max(longest, __shfl_xor_sync(FULL, longest, off));
+    if ((threadIdx.x & 31) == 0 && longest > 0) atomicMax(max_chain, longest);
+}
+
+// per example: number of features with an earlier occurrence (in-degree of
+// the conflict DAG) and the repeated-id check (the previous occurrence of a
+// feature lying inside the same row means the id repeats in that row)
+__global__ void k_row_links(const int64_t *__restrict__ row_ptr, int64_t n_rows, const int32_t *__restrict__ prev,
+                            int32_t *__restrict__ npred, int *status)
+{
+    if (read_status(status)) return;
+    const int lane = threadIdx.x & 31;
+    const int64_t gw = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    for (int64_t t = gw; t < n_rows; t += nw) {
+        int64_t b = row_ptr[t], e = row_ptr[t + 1];
+        int cnt = 0;
+        bool dup = false;
+        for (int64_t p = b + lane; p < e; p += 32) {
+            int32_t q = prev[p];
+            cnt += q >= 0;
+            dup |= q >= b;
+        }
+        for (int off = 16; off >= 1; off >>= 1) cnt += __shfl_xor_sync(FULL, cnt, off);
+        if (__any_sync(FULL, dup) && lane == 0) set_status(status, PDB_EDUP);
+        if (lane == 0) npred[t] = cnt;
+    }
+}
+
+// append the flagged lanes' items to a global queue (one atomic per warp)
+__device__ __forceinline__ int warp_append(bool flag, int *tail)
+{
+    unsigned m = __ballot_sync(FULL, flag);
+    if (m == 0) return -1;
+    const int lane = threadIdx.x & 31;
+    const int leader = __ffs(m) - 1;
+    int base = 0;
+    if (lane == leader) base = atomicAdd(tail, __popc(m));
+    base = __shfl_sync(FULL, base, leader);
+    return flag ? base + __popc(m & lanemask_lt()) : -1;
+}
+
+// Kahn-style frontier sweep over the conflict DAG (edge: occurrence p ->
+// next occurrence of the same feature).  Frontier l holds the examples all
+// of whose predecessors are in frontiers < l; an example joins frontier l+1
+// when its last incoming edge is consumed, which gives exactly the
+// longest-path level.  One cooperative persistent launch; the frontiers are
+// consecutive ranges of one queue and a grid barrier separates them.
+__global__ __launch_bounds__(THREADS) void k_levels_kahn(int32_t n_rows, const int64_t *__restrict__ row_ptr,
+                                                         const int32_t *__restrict__ next,
+                                                         const int32_t *__restrict__ row_of,
+                                                         const int32_t *__restrict__ npred, int32_t *indeg,
+                                                         int32_t *queue, int32_t *level, LevelCtl *ctl, int *status,
+                                                         uint64_t timeout)
+{
+    if (read_status(status)) return;
+    const int lane = threadIdx.x & 31;
+    const int gw = (int)(((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5);
+    const int nw = (int)(((int64_t)gridDim.x * blockDim.x) >> 5);
+    for (int t0 = gw * 32; t0 < n_rows; t0 += nw * 32) {
+        int t = t0 + lane;
+        bool zero = false;
+        if (t < n_rows) {
+            int d = npred[t];
+            indeg[t] = d;
+            zero = d == 0;
+            if (zero) level[t] = 0;
+        }
+        int slot = warp_append(zero, &ctl->tail);
+        if (zero) queue[slot] = t;
+    }
+    if (!grid_sync(&ctl->bar, status, timeout)) return;
+    int head = 0, end = ld_acquire_i(&ctl->tail), lvl = 0, widest = 0;
+    while (head < end) {
+        widest = max(widest, end - head);
+        for (int i = head + gw; i < end; i += nw) {
+            int t = __ldcg(queue + i);
+            int64_t b = row_ptr[t], e = row_ptr[t + 1];
+            for (int64_t p0 = b; p0 < e; p0 += 32) {
+                int64_t p = p0 + lane;
+                bool fire = false;
+                int u = -1;
+                if (p < e) {
+                    int q = next[p];
+                    if (q >= 0) {
+                        u = row_of[q];
+                        fire = atomicSub(indeg + u, 1) == 1;
+                    }
+                }
+                int slot = warp_append(fire, &ctl->tail);
+                if (fire) {
+                    queue[slot] = u;
+                    level[u] = lvl + 1;
+                }
+            }
+        }
+        if (!grid_sync(&ctl->bar, status, timeout)) return;
+        head = end;
+        end = ld_acquire_i(&ctl->tail);
+        ++lvl;
+    }
+    if (blockIdx.x == 0 && threadIdx.x == 0) {
+        ctl->n_levels = lvl;
+        ctl->max_width = widest;
+        if (end != n_rows) set_status(status, PDB_EFAULT);
+    }
+}
+
+// gate[p] = rank[p] with bit 31 set on the last occurrence of its feature:
+// the ready-counter value the occurrence waits for, and whether its release
+// hands the counter back to 0 for the next epoch
+__global__ void k_make_gate(const int32_t *__restrict__ rank, const int32_t *__restrict__ next, int64_t nnz,
+                            uint32_t *__restrict__ gate, const int *status)
+{
+    if (read_status(status)) return;
+    for (int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; p < nnz; p += (int64_t)gridDim.x * blockDim.x)
+        gate[p] = (uint32_t)rank[p] | (next[p] < 0 ? 0x80000000u : 0u);
+}
+
+__global__ void k_iota_u32_level(const int32_t *__restrict__ level, uint32_t *__restrict__ key, int32_t n)
+{
+    for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < n; i += gridDim.x * blockDim.x) key[i] = (uint32_t)level[i];
+}
+
+int grid_1d(int64_t n, int threads = 256)
+{
+    int64_t b = (n + threads - 1) / threads;
+    return (int)std::max<int64_t>(1, std::min<int64_t>(b, 152 * 32));
+}
+
+int check_csr(const pdb_csr *X)
+{
+    if (!X || X->n_rows < 0 || X->n_cols < 0 || X->nnz < 0) return PDB_EINVAL;
+    if (X->n_rows >= (1ll << 31) - 1 || X->n_cols >= (1ll << 31) - 1 || X->nnz >= (1ll << 31) - 1) return PDB_EINVAL;
+    if (!X->row_ptr) return PDB_EINVAL;
+    if (X->nnz > 0 && (!X->col || X->n_cols == 0)) return PDB_EINVAL;
+    return PDB_OK;
+}
+
+}  // namespace
+
+// ------------------------------------------------------------------ C ABI
+extern "C" {
+
+const char *pdb_strerror(int code)
+{
+    switch (code) {
+    case PDB_OK: return "ok";
+    case PDB_EINVAL: return "invalid argument or malformed row_ptr";
+    case PDB_ERANGE: return "feature id outside [0, n_cols)";
+    case PDB_EDUP: return "feature id repeated inside one example";
+    case PDB_ENOMEM: return "device allocation failed";
+    case PDB_ECUDA: return "CUDA runtime error";
+    case PDB_ETIMEOUT: return "device-side wait expired";
+    case PDB_EFAULT: return "internal invariant failed on the device";
+    case PDB_ESTATE: return "handle in the wrong mode for this call";
+    default: return "unknown error";
+    }
+}
+
+void pdb_conflicts_free(pdb_conflicts *c)
+{
+    if (!c) return;
+    cudaDeviceSynchronize();
+    void *ptrs[] = {c->row_ptr, c->csc_pos, c->prev,     c->next,     c->rank,
+                    c->row_of,  c->npred,   c->feat_ptr, c->status, c->max_chain};
+    for (void *p : ptrs)
+        if (p) cudaFree(p);
+    cudaEvent_t evs[] = {c->ev0, c->ev1, c->ev_sgd0, c->ev_sgd1, c->ev_bsp0, c->ev_bsp1};
+    for (cudaEvent_t e : evs)
+        if (e) cudaEventDestroy(e);
+    delete c;
+}
+
+int pdb_build_conflicts(const pdb_csr *X, pdb_conflicts **out, void *stream)
+{
+    if (!out) return PDB_EINVAL;
+    *out = nullptr;
+    int rc = check_csr(X);
+    if (rc != PDB_OK) return rc;
+    cudaStream_t s = (cudaStream_t)stream;
+    pdb_conflicts *c = new (std::nothrow) pdb_conflicts();
+    if (!c) return PDB_ENOMEM;
+    cudaGetDevice(&c->device);
+    c->n_rows = X->n_rows;
+    c->n_cols = X->n_cols;
+    c->nnz = X->nnz;
+    const int64_t N = X->n_rows, F = X->n_cols, nnz = X->nnz;
+    for (cudaEvent_t *e : {&c->ev0, &c->ev1, &c->ev_sgd0, &c->ev_sgd1, &c->ev_bsp0, &c->ev_bsp1})
+        if (cudaEventCreate(e) != cudaSuccess) { pdb_conflicts_free(c); return PDB_ECUDA; }
+    cudaEventRecord(c->ev0, s);
+    rc = PDB_OK;
+    rc = rc ? rc : alloc((void **)&c->status, sizeof(int) * 2, s);
+    rc = rc ? rc : alloc((void **)&c->max_chain, sizeof(int), s);
+    rc = rc ? rc : alloc((void **)&c->row_ptr, sizeof(int64_t) * (N + 1), s);
+    rc = rc ? rc : alloc((void **)&c->csc_pos, sizeof(int32_t) * nnz, s);
+    rc = rc ? rc : alloc((void **)&c->prev, sizeof(int32_t) * nnz, s);
+    rc = rc ? rc : alloc((void **)&c->next, sizeof(int32_t) * nnz, s);
+    rc = rc ? rc : alloc((void **)&c->rank, sizeof(int32_t) * nnz, s);
+    rc = rc ? rc : alloc((void **)&c->row_of, sizeof(int32_t) * nnz, s);
+    rc = rc ? rc : alloc((void **)&c->npred, sizeof(int32_t) * N, s);
+    rc = rc ? rc : alloc((void **)&c->feat_ptr, sizeof(int64_t) * (F + 1), s);
+    uint32_t *skey = nullptr, *tkey = nullptr;
+    int32_t *tval = nullptr;
+    rc = rc ? rc : alloc((void **)&skey, sizeof(uint32_t) * nnz, s);
+    rc = rc ? rc : alloc((void **)&tkey, sizeof(uint32_t) * nnz, s);
+    rc = rc ? rc : alloc((void **)&tval, sizeof(int32_t) * nnz, s);
+    if (rc != PDB_OK) {
+        release(skey, s);
+        release(tkey, s);
+        release(tval, s);
+        cudaStreamSynchronize(s);
+        pdb_conflicts_free(c);
+        return rc;
+    }
+    cudaMemsetAsync(c->status, 0, sizeof(int) * 2, s);
+    cudaMemsetAsync(c->max_chain, 0, sizeof(int), s);
+    cudaMemcpyAsync(c->row_ptr, X->row_ptr, sizeof(int64_t) * (N + 1), cudaMemcpyDeviceToDevice, s);
+    k_validate_rows<<<grid_1d(N + 1), 256, 0, s>>>(X->row_ptr, N, nnz, c->status);
+    if (nnz > 0) k_validate_cols<<<grid_1d(nnz), 256, 0, s>>>(X->col, nnz, F, c->status);
+    if (N > 0) k_row_of<<<grid_1d(N * 32), 256, 0, s>>>(X->row_ptr, N, c->row_of, c->status);
+    // (feature, position) pairs sorted by feature, stable: positions stay in data order
+    rc = radix_sort((const uint32_t *)X->col, nullptr, skey, c->csc_pos, tkey, tval, nnz, bits_for(F > 0 ? F - 1 : 0),
+                    c->status, s);
+    if (rc == PDB_OK) rc = segment_bounds(skey, nnz, F, nullptr, c->feat_ptr, c->status, s);
+    if (rc == PDB_OK && nnz > 0)
+        k_link<<<grid_1d(nnz), 256, 0, s>>>(skey, c->csc_pos, nnz, c->feat_ptr, c->prev, c->next, c->rank,
+                                            c->max_chain, c->status);
+    if (rc == PDB_OK && N > 0)
+        k_row_links<<<grid_1d(N * 32), 256, 0, s>>>(X->row_ptr, N, c->prev, c->npred, c->status);
+    release(skey, s);
+    release(tkey, s);
+    release(tval, s);
+    cudaEventRecord(c->ev1, s);
+    c->timed_build = true;
+    if (rc == PDB_OK && cudaPeekAtLastError() != cudaSuccess) rc = PDB_ECUDA;
+    if (rc != PDB_OK) {
+        cudaStreamSynchronize(s);
+        pdb_conflicts_free(c);
+        return rc;
+    }
+    *out = c;
+    return PDB_OK;
+}
+
+int pdb_conflicts_arrays(const pdb_conflicts *c, const int32_t **csc_pos, const int64_t **feat_ptr,
+                         const int32_t **prev, const int32_t **next, const int32_t **rank)
+{
+    if (!c) return PDB_EINVAL;
+    if (csc_pos) *csc_pos = c->csc_pos;
+    if (feat_ptr) *feat_ptr = c->feat_ptr;
+    if (prev) *prev = c->prev;
+    if (next) *next = c->next;
+    if (rank) *rank = c->rank;
+    return PDB_OK;
+}
+
+int pdb_status(const pdb_conflicts *c, void *stream)
+{
+    if (!c) return PDB_EINVAL;
+    if (cudaStreamSynchronize((cudaStream_t)stream) != cudaSuccess) return PDB_ECUDA;
+    int st = 0;
+    if (cudaMemcpy(&st, c->status, sizeof(int), cudaMemcpyDeviceToHost) != cudaSuccess) return PDB_ECUDA;
+    return st;
+}
+
+void pdb_schedule_free(pdb_schedule *s)
+{
+    if (!s) return;
+    cudaDeviceSynchronize();
+    void *ptrs[] = {s->level, s->order, s->indeg, s->queue, s->level_ptr, s->ctl, s->ctr, s->gate, s->bar, s->ticket};
+    for (void *p : ptrs)
+        if (p) cudaFree(p);
+    if (s->ev0) cudaEventDestroy(s->ev0);
+    if (s->ev1) cudaEventDestroy(s->ev1);
+    delete s;
+}
+
+int pdb_schedule_build(const pdb_conflicts *c, pdb_sched_mode mode, pdb_schedule **out, void *stream)
+{
+    if (!c || !out || (mode != PDB_SCHED_LEVELS && mode != PDB_SCHED_READY)) return PDB_EINVAL;
+    *out = nullptr;
+    cudaStream_t s = (cudaStream_t)stream;
+    pdb_schedule *h = new (std::nothrow) pdb_schedule();
+    if (!h) return PDB_ENOMEM;
+    h->c = c;
+    h->mode = mode;
+    if (cudaEventCreate(&h->ev0) != cudaSuccess || cudaEventCreate(&h->ev1) != cudaSuccess) {
+        pdb_schedule_free(h);
+        return PDB_ECUDA;
+    }
+    const int64_t N = c->n_rows, F = c->n_cols;
+    cudaEventRecord(h->ev0, s);
+    int rc = PDB_OK;
+    rc = rc ? rc : alloc((void **)&h->bar, sizeof(GridBarrier), s);
+    rc = rc ? rc : alloc((void **)&h->ticket, sizeof(unsigned long long), s);
+    if (rc == PDB_OK) {
+        cudaMemsetAsync(h->bar, 0, sizeof(GridBarrier), s);
+        cudaMemsetAsync(h->ticket, 0, sizeof(unsigned long long), s);
+    }
+    if (mode == PDB_SCHED_READY) {
+        rc = rc ? rc : alloc((void **)&h->ctr, sizeof(unsigned) * F, s);
+        rc = rc ? rc : alloc((void **)&h->gate, sizeof(uint32_t) * c->nnz, s);
+        if (rc == PDB_OK) {
+            cudaMemsetAsync(h->ctr, 0, sizeof(unsigned) * F, s);
+            if (c->nnz > 0)
+                k_make_gate<<<grid_1d(c->nnz), 256, 0, s>>>(c->rank, c->next, c->nnz, h->gate, c->status);
+        }
+    } else {
+        rc = rc ? rc : alloc((void **)&h->level, sizeof(int32_t) * N, s);
+        rc = rc ? rc : alloc((void **)&h->order, sizeof(int32_t) * N, s);
+        rc = rc ? rc : alloc((void **)&h->indeg, sizeof(int32_t) * N, s);
+        rc = rc ? rc : alloc((void **)&h->queue, sizeof(int32_t) * N, s);
+        rc = rc ? rc : alloc((void **)&h->level_ptr, sizeof(int64_t) * (N + 1), s);
+        rc = rc ? rc : alloc((void **)&h->ctl, sizeof(LevelCtl), s);
+        uint32_t *key = nullptr, *skey = nullptr, *tkey = nullptr;
+        int32_t *tval = nullptr;
+        rc = rc ? rc : alloc((void **)&key, sizeof(uint32_t) * N, s);
+        rc = rc ? rc : alloc((void **)&skey, sizeof(uint32_t) * N, s);
+        rc = rc ? rc : alloc((void **)&tkey, sizeof(uint32_t) * N, s);
+        rc = rc ? rc : alloc((void **)&tval, sizeof(int32_t) * N, s);
+        if (rc == PDB_OK) {
+            cudaMemsetAsync(h->ctl, 0, sizeof(LevelCtl), s);
+            if (N > 0) {
+                const void *kern = (const void *)k_levels_kahn;
+                int grid = persistent_grid(kern, nullptr);
+                int32_t n32 = (int32_t)N;
+                uint64_t tmo = timeout_ns(nullptr);
+                void *args[] = {&n32, (void *)&c->row_ptr, (void *)&c->next, (void *)&c->row_of,
+                                (void *)&c->npred, &h->indeg, &h->queue, &h->level, &h->ctl,
+                                (void *)&c->status, &tmo};
+                if (cudaLaunchCooperativeKernel(kern, grid, THREADS, args, 0, s) != cudaSuccess) rc = PDB_ECUDA;
+                if (rc == PDB_OK) {
+                    k_iota_u32_level<<<grid_1d(N), 256, 0, s>>>(h->level, key, n32);
+                    rc = radix_sort(key, nullptr, skey, h->order, tkey, tval, N, bits_for(N), c->status, s);
+                }
+                if (rc == PDB_OK) rc = segment_bounds(skey, N, N, &h->ctl->n_levels, h->level_ptr, c->status, s);
+            } else {
+                cudaMemsetAsync(h->level_ptr, 0, sizeof(int64_t), s);
+            }
+        }
+        release(key, s);
+        release(skey, s);
+        release(tkey, s);
+        release(tval, s);
+    }
+    cudaEventRecord(h->ev1, s);
+    h->timed = true;
+    if (rc == PDB_OK && cudaPeekAtLastError() != cudaSuccess) rc = PDB_ECUDA;
+    if (rc != PDB_OK) {
+        cudaGetLastError();
+        cudaStreamSynchronize(s);
+        pdb_schedule_free(h);
+        return rc;
+    }
+    *out = h;
+    return PDB_OK;
+}
+
+int pdb_schedule_levels(const pdb_schedule *h, const int32_t **level, const int32_t **order,
+                        const int64_t **level_ptr, int64_t *n_levels, void *stream)
+{
+    if (!h) return PDB_EINVAL;
+    if (h->mode != PDB_SCHED_LEVELS) return PDB_ESTATE;
+    if (level) *level = h->level;
+    if (order) *order = h->order;
+    if (level_ptr) *level_ptr = h->level_ptr;
+    if (n_levels) {
+        if (cudaStreamSynchronize((cudaStream_t)stream) != cudaSuccess) return PDB_ECUDA;
+        LevelCtl ctl;
+        if (cudaMemcpy(&ctl, h->ctl, sizeof ctl, cudaMemcpyDeviceToHost) != cudaSuccess) return PDB_ECUDA;
+        *n_levels = h->c->n_rows > 0 ? ctl.n_levels : 0;
+    }
+    return PDB_OK;
+}
+
+int pdb_schedule_ready(const pdb_schedule *h, const uint32_t **ctr, const uint32_t **gate)
+{
+    if (!h) return PDB_EINVAL;
+    if (h->mode != PDB_SCHED_READY) return PDB_ESTATE;
+    if (ctr) *ctr = h->ctr;
+    if (gate) *gate = h->gate;
+    return PDB_OK;
+}
+
+int pdb_get_stats(const pdb_conflicts *c, const pdb_schedule *h, pdb_stats *out)
+{
+    if (!c || !out) return PDB_EINVAL;
+    std::memset(out, 0, sizeof *out);
+    if (cudaDeviceSynchronize() != cudaSuccess) return PDB_ECUDA;
+    out->n_rows = c->n_rows;
+    out->n_cols = c->n_cols;
+    out->nnz = c->nnz;
+    out->n_levels = -1;
+    out->max_level_width = -1;
+    int mc = 0;
+    cudaMemcpy(&mc, c->max_chain, sizeof(int), cudaMemcpyDeviceToHost);
+    out->max_chain = mc;
+    float ms = 0;
+    if (c->timed_build && cudaEventElapsedTime(&ms, c->ev0, c->ev1) == cudaSuccess) out->ms_build = ms;
+    if (c->timed_sgd && cudaEventElapsedTime(&ms, c->ev_sgd0, c->ev_sgd1) == cudaSuccess) out->ms_sgd = ms;
+    if (c->timed_bsp && cudaEventElapsedTime(&ms, c->ev_bsp0, c->ev_bsp1) == cudaSuccess) out->ms_bsp = ms;
+    if (h) {
+        if (h->timed && cudaEventElapsedTime(&ms, h->ev0, h->ev1) == cudaSuccess) out->ms_schedule = ms;
+        if (h->mode == PDB_SCHED_LEVELS) {
+            LevelCtl ctl;
+            if (cudaMemcpy(&ctl, h->ctl, sizeof ctl, cudaMemcpyDeviceToHost) != cudaSuccess) return PDB_ECUDA;
+            out->n_levels = c->n_rows > 0 ? ctl.n_levels : 0;
+            out->max_level_width = ctl.max_width;
+        }
+    }
+    cudaGetLastError();
+    return PDB_OK;
+}
+
+int pdb_memcpy(void *dst, const void *src, size_t bytes, void *stream)
+{
+    if (bytes == 0) return PDB_OK;
+    if (!dst || !src) return PDB_EINVAL;
+    return cudaMemcpyAsync(dst, src, bytes, cudaMemcpyDefault, (cudaStream_t)stream) == cudaSuccess ? PDB_OK
+                                                                                                 : PDB_ECUDA;
+}
+
+}  // extern "C"

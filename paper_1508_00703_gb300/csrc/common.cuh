@@ -1,0 +1,208 @@
+// Internal helpers shared by the libpdb translation units: status words,
+// acquire/release memory operations, bounded waits, the grid barrier of the
+// persistent kernels, the fp32 numerics of one SGD transaction, and the
+// handle layouts.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "pdb.h"
+
+namespace pdb {
+
+constexpr unsigned FULL = 0xffffffffu;
+constexpr int THREADS = 256;             // block size of every persistent kernel
+constexpr int WARPS = THREADS / 32;
+
+// ------------------------------------------------------------------ host
+struct Launch {
+    int sms = 0;
+    int device = 0;
+};
+Launch launch_info();
+int occupancy_blocks(const void *kernel, int threads, size_t smem);
+int persistent_grid(const void *kernel, const pdb_opts *opts);
+uint64_t timeout_ns(const pdb_opts *opts);
+int alloc(void **p, size_t bytes, cudaStream_t s);   // stream-ordered, 256-byte aligned
+void release(void *p, cudaStream_t s);
+int bits_for(int64_t max_key);                        // bits to hold values 0..max_key (>= 1)
+
+// Stable LSD radix sort of (key, value) pairs, 8-bit digits.  vals_in ==
+// nullptr means value = index.  Sorted pairs land in keys_out/vals_out;
+// keys_tmp/vals_tmp are scratch of n elements each.  Kernels return early
+// when *status != 0.
+int radix_sort(const uint32_t *keys_in, const int32_t *vals_in, uint32_t *keys_out, int32_t *vals_out,
+               uint32_t *keys_tmp, int32_t *vals_tmp, int64_t n, int key_bits, const int *status,
+               cudaStream_t s);
+
+// ptr[k] = first index i of the sorted keys with keys[i] >= k, k = 0..n_bins
+// (n_bins read from *n_bins_dev when that is non-null).
+int segment_bounds(const uint32_t *sorted_keys, int64_t n, int64_t n_bins, const int *n_bins_dev, int64_t *ptr,
+                   const int *status, cudaStream_t s);
+
+// ------------------------------------------------------------------ device
+__host__ __device__ __forceinline__ int64_t min64(int64_t a, int64_t b) { return a < b ? a : b; }
+__device__ __forceinline__ void set_status(int *st, int code) { atomicCAS(st, 0, code); }
+__device__ __forceinline__ int read_status(const int *st) { return *(volatile const int *)st; }
+
+__device__ __forceinline__ unsigned ld_acquire(const unsigned *p)
+{
+    unsigned v;
+    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+__device__ __forceinline__ void st_release(unsigned *p, unsigned v)
+{
+    asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+__device__ __forceinline__ int ld_acquire_i(const int *p)
+{
+    int v;
+    asm volatile("ld.acquire.gpu.global.s32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+__device__ __forceinline__ uint64_t globaltimer()
+{
+    uint64_t t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+__device__ __forceinline__ unsigned lanemask_lt()
+{
+    unsigned m;
+    asm("mov.u32 %0, %%lanemask_lt;" : "=r"(m));
+    return m;
+}
+
+// Grid barrier for cooperative (co-resident) launches.  Generation counter:
+// read the generation, arrive, the last arriver resets the count and bumps
+// the generation; the others wait for the bump.  Every wait is bounded by
+// `deadline` (globaltimer ns) and gives up early when the status word is
+// set, so a failed block cannot hang the rest.  Returns false on give-up.
+struct GridBarrier {
+    unsigned count;
+    unsigned gen;
+};
+
+__device__ __forceinline__ bool grid_sync(GridBarrier *bar, int *status, uint64_t timeout)
+{
+    __shared__ int s_ok;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        int ok = 1;
+        unsigned gen = ld_acquire(&bar->gen);
+        __threadfence();
+        unsigned arrived = atomicAdd(&bar->count, 1u);
+        if (arrived == gridDim.x - 1) {
+            atomicExch(&bar->count, 0u);
+            __threadfence();
+            st_release(&bar->gen, gen + 1);
+        } else {
+            uint64_t t0 = globaltimer();
+            unsigned spins = 0;
+            while (ld_acquire(&bar->gen) == gen) {
+                if ((++spins & 63u) == 0) {
+                    if (read_status(status) != 0) { ok = 0; break; }
+                    if (globaltimer() - t0 > timeout) { set_status(status, PDB_ETIMEOUT); ok = 0; break; }
+                }
+                __nanosleep(32);
+            }
+        }
+        __threadfence();
+        s_ok = ok && read_status(status) == 0;
+    }
+    __syncthreads();
+    return s_ok != 0;
+}
+
+// ------------------------------------------------------------------ numerics
+// e^x: Cody-Waite argument reduction x = k ln2 + r with k = rint(x log2e)
+// (W. J. Cody and W. Waite, Software Manual for the Elementary Functions,
+// 1980); ln2 is split into a head with 16 significant bits, so k*head is
+// exact for |k| <= 256 and x - k*head is exact (Sterbenz), and a tail.  e^r
+// is the degree-7 Taylor polynomial sum r^n/n! in Horner form with fused
+// multiply-adds (|r| <= 0.35: truncation below 1e-8 relative).  2^k is
+// applied as two exact power-of-two factors so the one rounding happens in
+// the final product, also for subnormal results.  Inputs are clamped to
+// [-104, 89], where the result has already underflowed to 0 / overflowed.
+__device__ __forceinline__ float dev_expf(float x)
+{
+    if (x != x) return x;
+    x = x > 89.0f ? 89.0f : x;
+    x = x < -104.0f ? -104.0f : x;
+    const float log2e = 1.44269502162933349609375f;      // nearest float to log2(e)
+    const float ln2_head = 0.693145751953125f;           // 45426 * 2^-16
+    const float ln2_tail = 1.428606765330187045e-06f;     // ln2 - head, rounded to float
+    float kf = rintf(__fmul_rn(x, log2e));
+    float r = __fsub_rn(x, __fmul_rn(kf, ln2_head));
+    r = __fsub_rn(r, __fmul_rn(kf, ln2_tail));
+    float p = 1.0f / 5040.0f;
+    p = __fmaf_rn(p, r, 1.0f / 720.0f);
+    p = __fmaf_rn(p, r, 1.0f / 120.0f);
+    p = __fmaf_rn(p, r, 1.0f / 24.0f);
+    p = __fmaf_rn(p, r, 1.0f / 6.0f);
+    p = __fmaf_rn(p, r, 0.5f);
+    p = __fmaf_rn(p, r, 1.0f);
+    p = __fmaf_rn(p, r, 1.0f);
+    int k = (int)kf;
+    int h = k / 2;
+    int k2 = k - h;
+    float s1 = __int_as_float((h + 127) << 23);
+    float s2 = __int_as_float((k2 + 127) << 23);
+    return __fmul_rn(__fmul_rn(p, s1), s2);
+}
+
+// derivative of the example's loss with respect to its margin m
+__device__ __forceinline__ float dev_grad(int loss, float m, float y)
+{
+    if (loss == PDB_LOSS_LOGISTIC) return __fdiv_rn(-y, __fadd_rn(1.0f, dev_expf(__fmul_rn(y, m))));
+    if (loss == PDB_LOSS_SQUARED) return __fsub_rn(m, y);
+    return __fmul_rn(y, m) < 1.0f ? -y : 0.0f;
+}
+
+// combine the 32 lane partial sums pairwise: xor 16, 8, 4, 2, 1 (every lane
+// ends with the same value because fp32 addition commutes)
+__device__ __forceinline__ float warp_combine(float a)
+{
+#pragma unroll
+    for (int off = 16; off >= 1; off >>= 1) a = __fadd_rn(a, __shfl_xor_sync(FULL, a, off));
+    return a;
+}
+
+}  // namespace pdb
+
+// ------------------------------------------------------------------ handles
+struct pdb_conflicts {
+    int device;
+    int64_t n_rows, n_cols, nnz;
+    int64_t *row_ptr;     // library copy of the caller's row_ptr
+    int32_t *csc_pos, *prev, *next, *rank, *row_of, *npred;
+    int64_t *feat_ptr;
+    int *status;          // device word: first error recorded by a kernel
+    int *max_chain;       // device
+    cudaEvent_t ev0, ev1, ev_sgd0, ev_sgd1, ev_bsp0, ev_bsp1;
+    bool timed_build, timed_sgd, timed_bsp;
+};
+
+struct LevelCtl {
+    int tail;                 // frontier queue length
+    int n_levels;             // L
+    int max_width;
+    int pad;
+    pdb::GridBarrier bar;
+};
+
+struct pdb_schedule {
+    const pdb_conflicts *c;
+    pdb_sched_mode mode;
+    int32_t *level, *order, *indeg, *queue;
+    int64_t *level_ptr;
+    LevelCtl *ctl;            // device
+    unsigned *ctr;            // READY: per-feature ready counters
+    uint32_t *gate;           // READY: per position, rank | last-occurrence bit
+    pdb::GridBarrier *bar;    // barrier for the level-synchronous engine
+    unsigned long long *ticket;
+    cudaEvent_t ev0, ev1;
+    bool timed;
+};

@@ -1,0 +1,427 @@
+// Update engines: pdb_sgd_epoch (level-synchronous or ready-counter
+// dataflow) and pdb_bsp_epoch (the BSP mini-batch comparison).
+//
+// One warp runs one example (one transaction, Definition 3): the lanes load
+// the example's ids and values with coalesced loads, gather w through L2,
+// form the margin with per-lane fused multiply-adds and a xor-shuffle
+// combine, compute the scalar eta*g, and scatter w_j -= eta*g*x_j.  No
+// atomics touch w: the schedule guarantees that no other example holds any
+// of these features at the same time.
+#include <cuda_runtime.h>
+
+#include <algorithm>
+
+#include "common.cuh"
+
+using namespace pdb;
+
+namespace {
+
+constexpr int R = 8;   // elements per lane held in registers (rows up to 256 ids)
+
+__device__ __forceinline__ unsigned ld_relaxed(const unsigned *p)
+{
+    unsigned v;
+    asm volatile("ld.relaxed.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+__device__ __forceinline__ void st_relaxed(unsigned *p, unsigned v)
+{
+    asm volatile("st.relaxed.gpu.global.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+
+// ---------------------------------------------------------------- one example, no waits
+// Used by the level-synchronous engine: the level schedule already keeps
+// every example of a level disjoint from the others (Theorem 3).
+__device__ __forceinline__ void sgd_example(int t, const int64_t *__restrict__ row_ptr, const int32_t *__restrict__ col,
+                                            const float *__restrict__ val, const float *__restrict__ y, float *w,
+                                            int loss, float eta)
+{
+    const int lane = threadIdx.x & 31;
+    const int64_t b = row_ptr[t];
+    const int k = (int)(row_ptr[t + 1] - b);
+    const float yt = y[t];
+    float acc = 0.0f;
+    if (k <= 32 * R) {
+        int j[R];
+        float x[R], wv[R];
+#pragma unroll
+        for (int r = 0; r < R; ++r) {
+            int i = r * 32 + lane;
+            j[r] = i < k ? col[b + i] : 0;
+            x[r] = i < k ? (val ? val[b + i] : 1.0f) : 0.0f;
+        }
+#pragma unroll
+        for (int r = 0; r < R; ++r)
+            if (r * 32 + lane < k) wv[r] = __ldcg(w + j[r]);
+#pragma unroll
+        for (int r = 0; r < R; ++r)
+            if (r * 32 + lane < k) acc = __fmaf_rn(wv[r], x[r], acc);
+        const float m = warp_combine(acc);
+        const float c = __fmul_rn(eta, dev_grad(loss, m, yt));
+#pragma unroll
+        for (int r = 0; r < R; ++r)
+            if (r * 32 + lane < k) __stcg(w + j[r], __fsub_rn(wv[r], __fmul_rn(c, x[r])));
+    } else {
+        for (int i = lane; i < k; i += 32) acc = __fmaf_rn(__ldcg(w + col[b + i]), val ? val[b + i] : 1.0f, acc);
+        const float m = warp_combine(acc);
+        const float c = __fmul_rn(eta, dev_grad(loss, m, yt));
+        for (int i = lane; i < k; i += 32) {
+            int jj = col[b + i];
+            float xx = val ? val[b + i] : 1.0f;
+            __stcg(w + jj, __fsub_rn(__ldcg(w + jj), __fmul_rn(c, xx)));
+        }
+    }
+}
+
+// ---------------------------------------------------------------- level-synchronous engine
+// Persistent cooperative kernel: level l's examples are spread over all
+// warps, a grid barrier closes the level (the read barrier of the next BSP
+// step and the write barrier of this one, Algorithm 2a per level).
+__global__ __launch_bounds__(THREADS) void k_sgd_levels(const int64_t *__restrict__ row_ptr,
+                                                        const int32_t *__restrict__ col, const float *__restrict__ val,
+                                                        const float *__restrict__ y, const int32_t *__restrict__ order,
+                                                        const int64_t *__restrict__ level_ptr, const LevelCtl *ctl,
+                                                        float *w, int loss, float eta, int epochs, GridBarrier *bar,
+                                                        int *status, uint64_t timeout)
+{
+    if (read_status(status)) return;
+    const int L = ctl->n_levels;
+    const int gw = (int)(((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5);
+    const int nw = (int)(((int64_t)gridDim.x * blockDim.x) >> 5);
+    for (int ep = 0; ep < epochs; ++ep)
+        for (int l = 0; l < L; ++l) {
+            const int64_t b = level_ptr[l], e = level_ptr[l + 1];
+            for (int64_t i = b + gw; i < e; i += nw) sgd_example(order[i], row_ptr, col, val, y, w, loss, eta);
+            if (!grid_sync(bar, status, timeout)) return;
+        }
+}
+
+// ---------------------------------------------------------------- ready-counter dataflow engine
+// The read protocol of Section 5 per feature: ctr[j] counts the writes of
+// feature j so far in this epoch.  The occurrence of j with rank r may read
+// w_j once ctr[j] == r (Read Constraint: the previous writer is done), and
+// publishes r + 1 after its write (Write Constraint: its own read, the only
+// read of that version, precedes the write).  The last occurrence of j in
+// the epoch (gate bit 31) resets ctr[j] to 0 for the next epoch.
+// Examples are taken in data order from a ticket counter, so the oldest
+// unfinished example never waits on a younger one and the kernel cannot
+// deadlock regardless of how many warps are resident.
+// Acquire/release: relaxed polls of all the lane's counters, then one
+// fence; w stores, one fence, then relaxed counter stores.
+__device__ __forceinline__ bool wait_ready(const unsigned *ctr, const int *j, const unsigned *want, int lane, int k,
+                                           int *status, uint64_t timeout)
+{
+    bool ready;
+    uint64_t t0 = 0;
+    unsigned spins = 0;
+    for (;;) {
+        ready = true;
+#pragma unroll
+        for (int r = 0; r < R; ++r)
+            if (r * 32 + lane < k) ready &= ld_relaxed(ctr + j[r]) == want[r];
+        if (ready) break;
+        if (spins == 0) t0 = globaltimer();
+        if ((++spins & 127u) == 0) {
+            if (read_status(status)) return false;
+            if (globaltimer() - t0 > timeout) {
+                set_status(status, PDB_ETIMEOUT);
+                return false;
+            }
+        }
+    }
+    __threadfence();
+    return true;
+}
+
+__global__ __launch_bounds__(THREADS) void k_sgd_ready(int32_t n_rows, const int64_t *__restrict__ row_ptr,
+                                                       const int32_t *__restrict__ col, const float *__restrict__ val,
+                                                       const float *__restrict__ y, const uint32_t *__restrict__ gate,
+                                                       unsigned *ctr, float *w, int loss, float eta,
+                                                       unsigned long long *ticket, int *status, uint64_t timeout)
+{
+    if (read_status(status)) return;
+    const int lane = threadIdx.x & 31;
+    for (;;) {
+        unsigned long long tk = 0;
+        if (lane == 0) tk = atomicAdd(ticket, 1ull);
+        tk = __shfl_sync(FULL, tk, 0);
+        if (tk >= (unsigned long long)n_rows) return;
+        const int t = (int)tk;
+        const int64_t b = row_ptr[t];
+        const int k = (int)(row_ptr[t + 1] - b);
+        const float yt = y[t];
+        if (k <= 32 * R) {
+            int j[R];
+            float x[R], wv[R];
+            unsigned want[R], next[R];
+#pragma unroll
+            for (int r = 0; r < R; ++r) {
+                int i = r * 32 + lane;
+                j[r] = i < k ? col[b + i] : 0;
+                x[r] = i < k ? (val ? val[b + i] : 1.0f) : 0.0f;
+                uint32_t g = i < k ? gate[b + i] : 0u;
+                want[r] = g & 0x7fffffffu;
+                next[r] = (g >> 31) ? 0u : want[r] + 1u;
+            }
+            bool ok = wait_ready(ctr, j, want, lane, k, status, timeout);
+            if (!__all_sync(FULL, ok)) return;
+            float acc = 0.0f;
+#pragma unroll
+            for (int r = 0; r < R; ++r)
+                if (r * 32 + lane < k) wv[r] = __ldcg(w + j[r]);
+#pragma unroll
+            for (int r = 0; r < R; ++r)
+                if (r * 32 + lane < k) acc = __fmaf_rn(wv[r], x[r], acc);
+            const float m = warp_combine(acc);
+            const float c = __fmul_rn(eta, dev_grad(loss, m, yt));
+#pragma unroll
+            for (int r = 0; r < R; ++r)
+                if (r * 32 + lane < k) __stcg(w + j[r], __fsub_rn(wv[r], __fmul_rn(c, x[r])));
+            __threadfence();
+#pragma unroll
+            for (int r = 0; r < R; ++r)
+                if (r * 32 + lane < k) st_relaxed(ctr + j[r], next[r]);
+        } else {
+            // long example: wait and gather element by element, then a second pass
+            float acc = 0.0f;
+            bool ok = true;
+            for (int i = lane; i < k && ok; i += 32) {
+                int jj = col[b + i];
+                unsigned want = gate[b + i] & 0x7fffffffu;
+                int j1[R] = {jj};
+                unsigned w1[R] = {want};
+                ok = wait_ready(ctr, j1, w1, 0, 1, status, timeout);
+                if (ok) acc = __fmaf_rn(__ldcg(w + jj), val ? val[b + i] : 1.0f, acc);
+            }
+            if (!__all_sync(FULL, ok)) return;
+            const float m = warp_combine(acc);
+            const float c = __fmul_rn(eta, dev_grad(loss, m, yt));
+            for (int i = lane; i < k; i += 32) {
+                int jj = col[b + i];
+                float xx = val ? val[b + i] : 1.0f;
+                __stcg(w + jj, __fsub_rn(__ldcg(w + jj), __fmul_rn(c, xx)));
+            }
+            __threadfence();
+            for (int i = lane; i < k; i += 32) {
+                uint32_t g = gate[b + i];
+                st_relaxed(ctr + col[b + i], (g >> 31) ? 0u : (g & 0x7fffffffu) + 1u);
+            }
+        }
+    }
+}
+
+// ---------------------------------------------------------------- BSP
+// margin of example t at the current w (all lanes return the same value)
+__device__ __forceinline__ float margin(int t, const int64_t *__restrict__ row_ptr, const int32_t *__restrict__ col,
+                                        const float *__restrict__ val, const float *w)
+{
+    const int lane = threadIdx.x & 31;
+    const int64_t b = row_ptr[t];
+    const int k = (int)(row_ptr[t + 1] - b);
+    float acc = 0.0f;
+    for (int i = lane; i < k; i += 32) acc = __fmaf_rn(__ldcg(w + col[b + i]), val ? val[b + i] : 1.0f, acc);
+    return warp_combine(acc);
+}
+
+// Algorithm 2a with B examples per step: reads (margins at the snapshot),
+// barrier, writes (ordered per-feature sums), barrier.  The batch's pairs
+// are pre-sorted by (batch, feature, example), so each feature's terms of a
+// batch are one contiguous run summed in ascending example order.
+__global__ __launch_bounds__(THREADS) void k_bsp(int32_t n_rows, int64_t batch, int64_t n_batches,
+                                                 const int64_t *__restrict__ row_ptr, const int32_t *__restrict__ col,
+                                                 const float *__restrict__ val, const float *__restrict__ y,
+                                                 const int64_t *__restrict__ bptr, const int32_t *__restrict__ bcol,
+                                                 const int32_t *__restrict__ brow, const float *__restrict__ bval,
+                                                 float *cbuf, float *w, int loss, float eta, int epochs,
+                                                 GridBarrier *bar, int *status, uint64_t timeout)
+{
+    if (read_status(status)) return;
+    const int lane = threadIdx.x & 31;
+    const int64_t gtid = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    const int64_t nthr = (int64_t)gridDim.x * blockDim.x;
+    const int gw = (int)(gtid >> 5), nw = (int)(nthr >> 5);
+    for (int ep = 0; ep < epochs; ++ep)
+        for (int64_t bi = 0; bi < n_batches; ++bi) {
+            const int64_t r0 = bi * batch, r1 = min64(n_rows, r0 + batch);
+            for (int64_t t = r0 + gw; t < r1; t += nw) {
+                float m = margin((int)t, row_ptr, col, val, w);
+                if (lane == 0) cbuf[t - r0] = __fmul_rn(eta, dev_grad(loss, m, y[t]));
+            }
+            if (!grid_sync(bar, status, timeout)) return;
+            const int64_t s0 = bptr[bi], s1 = bptr[bi + 1];
+            for (int64_t s = s0 + gtid; s < s1; s += nthr) {
+                const int32_t j = bcol[s];
+                if (s > s0 && bcol[s - 1] == j) continue;
+                float delta = 0.0f;
+                for (int64_t q = s; q < s1 && bcol[q] == j; ++q)
+                    delta = __fadd_rn(delta, __fmul_rn(__ldcg(cbuf + (brow[q] - r0)), bval[q]));
+                __stcg(w + j, __fsub_rn(__ldcg(w + j), delta));
+            }
+            if (!grid_sync(bar, status, timeout)) return;
+        }
+}
+
+__global__ void k_bsp_keys(const int32_t *__restrict__ csc_pos, const int32_t *__restrict__ row_of, int64_t nnz,
+                           int64_t batch, uint32_t *__restrict__ key, const int *status)
+{
+    if (read_status(status)) return;
+    for (int64_t s = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; s < nnz; s += (int64_t)gridDim.x * blockDim.x)
+        key[s] = (uint32_t)(row_of[csc_pos[s]] / batch);
+}
+
+__global__ void k_bsp_gather(const int32_t *__restrict__ bpos, const int32_t *__restrict__ col,
+                             const float *__restrict__ val, const int32_t *__restrict__ row_of, int64_t nnz,
+                             int32_t *__restrict__ bcol, int32_t *__restrict__ brow, float *__restrict__ bval,
+                             const int *status)
+{
+    if (read_status(status)) return;
+    for (int64_t s = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; s < nnz; s += (int64_t)gridDim.x * blockDim.x) {
+        int32_t p = bpos[s];
+        bcol[s] = col[p];
+        brow[s] = row_of[p];
+        bval[s] = val ? val[p] : 1.0f;
+    }
+}
+
+__global__ void k_eval_expf(const float *__restrict__ x, float *__restrict__ out, int64_t n)
+{
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x)
+        out[i] = dev_expf(x[i]);
+}
+
+int grid_1d(int64_t n)
+{
+    int64_t b = (n + 255) / 256;
+    return (int)std::max<int64_t>(1, std::min<int64_t>(b, 152 * 32));
+}
+
+int check_run(const pdb_csr *X, const float *y, const pdb_conflicts *c, const float *w, int loss, int epochs)
+{
+    if (!X || !c || epochs < 0) return PDB_EINVAL;
+    if (loss != PDB_LOSS_LOGISTIC && loss != PDB_LOSS_SQUARED && loss != PDB_LOSS_HINGE) return PDB_EINVAL;
+    if (X->n_rows != c->n_rows || X->n_cols != c->n_cols || X->nnz != c->nnz) return PDB_EINVAL;
+    if (!X->row_ptr || (X->nnz > 0 && !X->col)) return PDB_EINVAL;
+    if ((X->n_rows > 0 && !y) || (X->n_cols > 0 && !w)) return PDB_EINVAL;
+    return PDB_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+int pdb_sgd_epoch(const pdb_csr *X, const float *y, const pdb_conflicts *c, const pdb_schedule *h, float *w,
+                  pdb_loss loss, float eta, int n_epochs, const pdb_opts *opts, void *stream)
+{
+    int rc = check_run(X, y, c, w, loss, n_epochs);
+    if (rc != PDB_OK) return rc;
+    if (!h || h->c != c) return PDB_EINVAL;
+    cudaStream_t s = (cudaStream_t)stream;
+    pdb_conflicts *cm = const_cast<pdb_conflicts *>(c);
+    cudaEventRecord(cm->ev_sgd0, s);
+    const uint64_t tmo = timeout_ns(opts);
+    int32_t n32 = (int32_t)X->n_rows;
+    int lossi = (int)loss;
+    if (X->n_rows > 0 && n_epochs > 0) {
+        if (h->mode == PDB_SCHED_LEVELS) {
+            const void *kern = (const void *)k_sgd_levels;
+            int grid = persistent_grid(kern, opts);
+            const int64_t *rp = X->row_ptr;
+            const int32_t *cl = X->col;
+            const float *vl = X->val;
+            void *args[] = {(void *)&rp,        (void *)&cl, (void *)&vl,       (void *)&y,
+                            (void *)&h->order,  (void *)&h->level_ptr, (void *)&h->ctl, (void *)&w,
+                            (void *)&lossi,     (void *)&eta, (void *)&n_epochs, (void *)&h->bar,
+                            (void *)&cm->status, (void *)&tmo};
+            if (cudaLaunchCooperativeKernel(kern, grid, THREADS, args, 0, s) != cudaSuccess) rc = PDB_ECUDA;
+        } else {
+            int grid = persistent_grid((const void *)k_sgd_ready, opts);
+            for (int ep = 0; ep < n_epochs; ++ep) {
+                cudaMemsetAsync(h->ticket, 0, sizeof(unsigned long long), s);
+                k_sgd_ready<<<grid, THREADS, 0, s>>>(n32, X->row_ptr, X->col, X->val, y, h->gate, h->ctr, w, lossi,
+                                                     eta, h->ticket, cm->status, tmo);
+            }
+        }
+    }
+    cudaEventRecord(cm->ev_sgd1, s);
+    cm->timed_sgd = true;
+    if (rc == PDB_OK && cudaPeekAtLastError() != cudaSuccess) rc = PDB_ECUDA;
+    if (rc != PDB_OK) cudaGetLastError();
+    return rc;
+}
+
+int pdb_bsp_epoch(const pdb_csr *X, const float *y, const pdb_conflicts *c, float *w, pdb_loss loss, float eta,
+                  int64_t batch, int n_epochs, const pdb_opts *opts, void *stream)
+{
+    int rc = check_run(X, y, c, w, loss, n_epochs);
+    if (rc != PDB_OK) return rc;
+    if (batch < 1) return PDB_EINVAL;
+    cudaStream_t s = (cudaStream_t)stream;
+    pdb_conflicts *cm = const_cast<pdb_conflicts *>(c);
+    const int64_t N = X->n_rows, nnz = X->nnz;
+    if (batch > N && N > 0) batch = N;
+    cudaEventRecord(cm->ev_bsp0, s);
+    if (N > 0 && n_epochs > 0) {
+        const int64_t n_batches = (N + batch - 1) / batch;
+        uint32_t *key = nullptr, *skey = nullptr, *tkey = nullptr;
+        int32_t *bpos = nullptr, *tval = nullptr, *bcol = nullptr, *brow = nullptr;
+        float *bval = nullptr, *cbuf = nullptr;
+        int64_t *bptr = nullptr;
+        GridBarrier *bar = nullptr;
+        rc = alloc((void **)&key, sizeof(uint32_t) * nnz, s);
+        rc = rc ? rc : alloc((void **)&skey, sizeof(uint32_t) * nnz, s);
+        rc = rc ? rc : alloc((void **)&tkey, sizeof(uint32_t) * nnz, s);
+        rc = rc ? rc : alloc((void **)&bpos, sizeof(int32_t) * nnz, s);
+        rc = rc ? rc : alloc((void **)&tval, sizeof(int32_t) * nnz, s);
+        rc = rc ? rc : alloc((void **)&bcol, sizeof(int32_t) * nnz, s);
+        rc = rc ? rc : alloc((void **)&brow, sizeof(int32_t) * nnz, s);
+        rc = rc ? rc : alloc((void **)&bval, sizeof(float) * nnz, s);
+        rc = rc ? rc : alloc((void **)&cbuf, sizeof(float) * batch, s);
+        rc = rc ? rc : alloc((void **)&bptr, sizeof(int64_t) * (n_batches + 1), s);
+        rc = rc ? rc : alloc((void **)&bar, sizeof(GridBarrier), s);
+        if (rc == PDB_OK) {
+            cudaMemsetAsync(bar, 0, sizeof(GridBarrier), s);
+            if (nnz > 0) {
+                k_bsp_keys<<<grid_1d(nnz), 256, 0, s>>>(c->csc_pos, c->row_of, nnz, batch, key, cm->status);
+                // stable by batch: inside a batch the feature-major CSC order survives
+                rc = radix_sort(key, c->csc_pos, skey, bpos, tkey, tval, nnz, bits_for(n_batches - 1), cm->status, s);
+                if (rc == PDB_OK)
+                    k_bsp_gather<<<grid_1d(nnz), 256, 0, s>>>(bpos, X->col, X->val, c->row_of, nnz, bcol, brow, bval,
+                                                              cm->status);
+            }
+            if (rc == PDB_OK) rc = segment_bounds(skey, nnz, n_batches, nullptr, bptr, cm->status, s);
+            if (rc == PDB_OK) {
+                const void *kern = (const void *)k_bsp;
+                int grid = persistent_grid(kern, opts);
+                int32_t n32 = (int32_t)N;
+                int lossi = (int)loss;
+                uint64_t tmo = timeout_ns(opts);
+                const int64_t *rp = X->row_ptr;
+                const int32_t *cl = X->col;
+                const float *vl = X->val;
+                void *args[] = {&n32,  &batch, (void *)&n_batches, (void *)&rp, (void *)&cl, (void *)&vl,
+                                (void *)&y, &bptr, &bcol, &brow, &bval, &cbuf, &w, &lossi, &eta, &n_epochs, &bar,
+                                (void *)&cm->status, &tmo};
+                if (cudaLaunchCooperativeKernel(kern, grid, THREADS, args, 0, s) != cudaSuccess) rc = PDB_ECUDA;
+            }
+        }
+        for (void *p : {(void *)key, (void *)skey, (void *)tkey, (void *)bpos, (void *)tval, (void *)bcol, (void *)brow,
+                        (void *)bval, (void *)cbuf, (void *)bptr, (void *)bar})
+            release(p, s);
+    }
+    cudaEventRecord(cm->ev_bsp1, s);
+    cm->timed_bsp = true;
+    if (rc == PDB_OK && cudaPeekAtLastError() != cudaSuccess) rc = PDB_ECUDA;
+    if (rc != PDB_OK) cudaGetLastError();
+    return rc;
+}
+
+int pdb_eval_expf(const float *x, float *out, int64_t n, void *stream)
+{
+    if (n < 0 || (n > 0 && (!x || !out))) return PDB_EINVAL;
+    if (n == 0) return PDB_OK;
+    k_eval_expf<<<grid_1d(n), 256, 0, (cudaStream_t)stream>>>(x, out, n);
+    return cudaPeekAtLastError() == cudaSuccess ? PDB_OK : PDB_ECUDA;
+}
+
+}  // extern "C"

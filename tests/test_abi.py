@@ -1,0 +1,66 @@
+"""The C ABI library builds for sm_103a, loads without a GPU, and exports
+every function include/pdb.h declares (no compute calls here)."""
+import ctypes
+import os
+import re
+import subprocess
+
+import pytest
+
+import paper_1508_00703_gb300 as pdb
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def _declared():
+    names = set()
+    for fn in os.listdir(os.path.join(ROOT, "include")):
+        if fn.endswith(".h"):
+            text = open(os.path.join(ROOT, "include", fn)).read()
+            text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+            names |= set(re.findall(r"\b(pdb_\w+)\s*\(", text))
+    return names
+
+
+def test_library_exports_every_declared_symbol():
+    path = pdb.build()
+    out = subprocess.run(["nm", "-D", "--defined-only", path], capture_output=True, text=True, check=True).stdout
+    exported = {line.split()[-1] for line in out.splitlines() if " T " in line}
+    declared = _declared()
+    assert declared, "no declarations found"
+    assert declared <= exported, declared - exported
+    assert set(pdb.EXPORTS) == declared
+
+
+def test_library_loads_and_resolves():
+    lib = ctypes.CDLL(pdb.build())
+    for name in _declared():
+        assert getattr(lib, name) is not None
+
+
+def test_strerror_without_gpu():
+    lib = pdb.load()
+    assert lib.pdb_strerror(pdb.PDB_EDUP).decode().startswith("feature id repeated")
+    assert lib.pdb_strerror(0).decode() == "ok"
+
+
+def test_host_argument_errors_need_no_gpu():
+    # argument checks happen on the host before any CUDA call
+    lib = pdb.load()
+    h = ctypes.c_void_p()
+    assert lib.pdb_build_conflicts(None, ctypes.byref(h), None) == pdb.PDB_EINVAL
+    bad = pdb.pdb_csr(-1, 4, 0, None, None, None)
+    assert lib.pdb_build_conflicts(ctypes.byref(bad), ctypes.byref(h), None) == pdb.PDB_EINVAL
+    big = pdb.pdb_csr(1, 4, 1 << 31, ctypes.c_void_p(8), ctypes.c_void_p(8), None)
+    assert lib.pdb_build_conflicts(ctypes.byref(big), ctypes.byref(h), None) == pdb.PDB_EINVAL
+    assert lib.pdb_schedule_build(None, 0, ctypes.byref(h), None) == pdb.PDB_EINVAL
+
+
+def test_nvcc_targets_sm_103a_only():
+    assert pdb.ARCH == "-gencode=arch=compute_103a,code=sm_103a"
+    assert "-fmad=false" in pdb.NVCC_FLAGS and "--use_fast_math" not in pdb.NVCC_FLAGS
+
+
+def test_graft_entry_build():
+    import __graft_entry__
+    __graft_entry__.build()

@@ -1,0 +1,179 @@
+"""Parity of the CUDA path (through the C ABI) with the CPU oracle.
+
+Bar: the conflict chains, levels and level order are integer results and
+must match bit for bit; fp32 weights must be within max relative error 1e-5
+(max |w_gpu - w_oracle| / max |w_oracle|).  Because both sides follow the
+same fp32 operation order, the weights are also checked for bitwise
+equality."""
+import numpy as np
+import pytest
+
+from tests import _cases as C
+
+torch = pytest.importorskip("torch")
+pdb = pytest.importorskip("paper_1508_00703_gb300")
+
+pytestmark = pytest.mark.gpu
+
+TOL = 1e-5
+ALL = list(C.SMALL) + C.EDGES
+
+
+def _gpu(name):
+    p = C.problem(name)
+    X = pdb.Csr.from_problem(p)
+    y = torch.from_numpy(p.y).cuda()
+    return p, X, y
+
+
+def _arr(ptr, n, dtype):
+    return pdb.device_array(ptr, n, dtype).cpu().numpy()
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _cuda():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    pdb.load()
+
+
+def test_expf_matches_oracle_bitwise_and_fp64():
+    import oracle
+    x = np.concatenate([np.linspace(-110, 95, 3_000_001, dtype=np.float64).astype(np.float32),
+                        np.random.default_rng(0).normal(0, 3, 1_000_000).astype(np.float32),
+                        np.array([0.0, -0.0, np.inf, -np.inf, np.nan], np.float32)])
+    xt = torch.from_numpy(x).cuda()
+    out = torch.empty_like(xt)
+    pdb.pdb_eval_expf(xt, out)
+    got = out.cpu().numpy()
+    ref = oracle.expf(x)
+    assert np.array_equal(got.view(np.uint32), ref.view(np.uint32))
+    m = (x > -87) & (x < 88.5)
+    e64 = np.exp(x[m].astype(np.float64))
+    ulp = np.spacing(e64.astype(np.float32)).astype(np.float64)
+    assert np.max(np.abs(got[m] - e64) / ulp) <= 2.0
+
+
+@pytest.mark.parametrize("name", ALL)
+def test_chains_bit_exact(name):
+    p, X, y = _gpu(name)
+    c = pdb.pdb_build_conflicts(X)
+    pdb.check_status(c)
+    arrs = pdb.pdb_conflicts_arrays(c)
+    ref = C.oracle_chains(name)
+    for key in ("csc_pos", "prev", "next", "rank"):
+        assert np.array_equal(_arr(arrs[key], p.nnz, torch.int32), ref[key]), key
+    assert np.array_equal(_arr(arrs["feat_ptr"], p.n_cols + 1, torch.int64), ref["feat_ptr"])
+    st = pdb.pdb_get_stats(c)
+    counts = np.diff(ref["feat_ptr"])
+    assert st["max_chain"] == (counts.max() if counts.size else 0)
+
+
+@pytest.mark.parametrize("name", ALL)
+def test_levels_bit_exact(name):
+    p, X, y = _gpu(name)
+    c = pdb.pdb_build_conflicts(X)
+    s = pdb.pdb_schedule_build(c, pdb.PDB_SCHED_LEVELS)
+    info = pdb.pdb_schedule_levels(s)
+    pdb.check_status(c)
+    lv, L, order, level_ptr = C.oracle_levels(name)
+    assert info["n_levels"] == L
+    assert np.array_equal(_arr(info["level"], p.n_rows, torch.int32), lv)
+    assert np.array_equal(_arr(info["order"], p.n_rows, torch.int32), order)
+    assert np.array_equal(_arr(info["level_ptr"], L + 1, torch.int64), level_ptr)
+    st = pdb.pdb_get_stats(c, s)
+    assert st["n_levels"] == L
+    if L:
+        assert st["max_level_width"] == np.max(np.diff(level_ptr))
+
+
+def _sgd(name, mode, opts=None):
+    p, X, y = _gpu(name)
+    c = pdb.pdb_build_conflicts(X)
+    s = pdb.pdb_schedule_build(c, mode)
+    w = torch.zeros(p.n_cols, dtype=torch.float32, device="cuda")
+    pdb.pdb_sgd_epoch(X, y, c, s, w, p.loss, p.eta, p.epochs, opts=opts)
+    pdb.check_status(c)
+    return w.cpu().numpy()
+
+
+@pytest.mark.parametrize("mode", ["levels", "ready"])
+@pytest.mark.parametrize("name", ALL)
+def test_sgd_weights(name, mode):
+    m = pdb.PDB_SCHED_LEVELS if mode == "levels" else pdb.PDB_SCHED_READY
+    got = _sgd(name, m)
+    ref = C.oracle_sgd(name)
+    assert C.rel_err(got, ref) <= TOL
+    assert np.array_equal(got, ref)       # same fp32 operation order on both sides
+
+
+def test_sgd_small_grid_and_repeat_calls():
+    # a one-block-per-SM grid, and a second call continuing from the first
+    name = "zipf-shape"
+    p, X, y = _gpu(name)
+    c = pdb.pdb_build_conflicts(X)
+    for mode in (pdb.PDB_SCHED_LEVELS, pdb.PDB_SCHED_READY):
+        s = pdb.pdb_schedule_build(c, mode)
+        w = torch.zeros(p.n_cols, dtype=torch.float32, device="cuda")
+        pdb.pdb_sgd_epoch(X, y, c, s, w, p.loss, p.eta, 1, opts=dict(blocks_per_sm=1))
+        pdb.pdb_sgd_epoch(X, y, c, s, w, p.loss, p.eta, 1)
+        pdb.check_status(c)
+        import oracle
+        assert np.array_equal(w.cpu().numpy(), oracle.sgd(p, epochs=2))
+
+
+@pytest.mark.parametrize("batch", [1, 7, 64, 4096, 10**9])
+@pytest.mark.parametrize("name", ["tiny", "deepchain-shape", "ragged-empty-rows", "ctr-shape-binary"])
+def test_bsp_weights(name, batch):
+    import oracle
+    p, X, y = _gpu(name)
+    c = pdb.pdb_build_conflicts(X)
+    w = torch.zeros(p.n_cols, dtype=torch.float32, device="cuda")
+    epochs = min(p.epochs, 2)
+    pdb.pdb_bsp_epoch(X, y, c, w, p.loss, p.eta, batch, epochs)
+    pdb.check_status(c)
+    ref = oracle.bsp(p, batch, epochs=epochs)
+    got = w.cpu().numpy()
+    assert C.rel_err(got, ref) <= TOL
+    assert np.array_equal(got, ref)
+
+
+@pytest.mark.parametrize("row_ptr,col,code", [
+    ([0, 2, 1, 3], [0, 1, 2], -1),
+    ([0, 2, 3], [0, 4, 1], -2),
+    ([0, 2, 3], [0, -1, 1], -2),
+    ([0, 3, 4], [2, 0, 2, 1], -3),
+])
+def test_device_validation(row_ptr, col, code):
+    import synthdata
+    p = synthdata.from_arrays(row_ptr, col, None, np.ones(len(row_ptr) - 1), n_cols=4)
+    X = pdb.Csr.from_problem(p)
+    c = pdb.pdb_build_conflicts(X)
+    assert pdb.pdb_status(c) == code
+    # a poisoned handle stays poisoned and later kernels do nothing
+    s = pdb.pdb_schedule_build(c, pdb.PDB_SCHED_READY)
+    y = torch.ones(p.n_rows, device="cuda")
+    w = torch.zeros(4, device="cuda")
+    pdb.pdb_sgd_epoch(X, y, c, s, w, 0, 0.1, 1)
+    assert pdb.pdb_status(c) == code
+    assert torch.count_nonzero(w).item() == 0
+
+
+def test_wait_timeout_is_reported_not_hung():
+    # A ready counter that nothing will ever release: every bounded wait
+    # gives up after the short limit, the kernel returns, the status says so,
+    # and the context stays usable.
+    name = "tiny"
+    p, X, y = _gpu(name)
+    c = pdb.pdb_build_conflicts(X)
+    s = pdb.pdb_schedule_build(c, pdb.PDB_SCHED_READY)
+    pdb.check_status(c)
+    ctr_ptr = pdb.pdb_schedule_ready(s)["ctr"]
+    j = int(p.col[p.row_ptr[5]])                          # a feature that example 5 reads
+    poison = torch.tensor([12345], dtype=torch.int32, device="cuda")
+    pdb.pdb_memcpy(ctr_ptr + 4 * j, poison.data_ptr(), 4)
+    w = torch.zeros(p.n_cols, dtype=torch.float32, device="cuda")
+    pdb.pdb_sgd_epoch(X, y, c, s, w, p.loss, p.eta, 1, opts=dict(wait_timeout_s=0.2))
+    assert pdb.pdb_status(c) == pdb.PDB_ETIMEOUT
+    t = torch.arange(10, device="cuda").sum().item()     # the device still works
+    assert t == 45
