@@ -1,0 +1,392 @@
+#!/usr/bin/env python3
+"""Benchmark of serially-equivalent sparse SGD on GB300.
+
+One step = the whole hot path over one synthetic problem held in HBM:
+pdb_build_conflicts (validate, feature sort, chains) + pdb_schedule_build +
+pdb_sgd_epoch over all of the workload's epochs.  The metric is
+nnz-updates per second (epochs x nnz / step time).  Default workload: the
+low-conflict, HBM-bound problem (4e6 examples x 1e8 features, 100 uniform
+ids per example, squared loss, eta = 1e-3, 2 epochs).
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+Under torchrun each rank runs an independent replica on its own GPU (the
+method's conflict structure does not shard without a per-hop exchange), and
+the aggregate is the sum of all ranks' updates over the slowest rank's time.
+``--impl reference`` times the CPU oracle (sequential SGD, one core) on a
+bounded sample of the same workload.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "serially-equivalent sparse SGD nnz-updates/sec at 1 GB300; % of HBM roofline"
+UNIT = "nnz-updates/s"
+ALG_BYTES_PER_NNZ = 16      # col 4 + val 4 + w read 4 + w write 4
+ALG_BYTES_PER_ROW = 12      # row_ptr 8 + y 4
+L2_BYTES = 129 * 2 ** 20
+
+
+def parse_args(argv=None):
+    ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default="low-conflict")
+    ap.add_argument("--mode", choices=["ready", "levels"], default="ready")
+    ap.add_argument("--rows", type=int, default=None, help="override the workload's example count")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=10.0, help="target length of the CPU oracle sample")
+    return ap.parse_args(argv)
+
+
+# ---------------------------------------------------------------- distributed helpers
+def dist_env():
+    return int(os.environ.get("RANK", 0)), int(os.environ.get("WORLD_SIZE", 1)), int(os.environ.get("LOCAL_RANK", 0))
+
+
+def reduce_max(value: float, world: int) -> float:
+    if world == 1:
+        return value
+    import torch
+    import torch.distributed as dist
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([value], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def reduce_sum(value: float, world: int) -> float:
+    if world == 1:
+        return value
+    import torch
+    import torch.distributed as dist
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([value], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.SUM)
+    return float(t.item())
+
+
+def barrier(world: int):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+# ---------------------------------------------------------------- measurement helpers
+def measured_peak_hbm():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            return float(json.load(f)["hbm_gbs"]), "measured"
+    except Exception:
+        return 6800.0, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi samples of SM clock and throttle reasons during the timed region."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.file = None
+
+    def __enter__(self):
+        try:
+            self.file = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                         stdout=self.file, stderr=subprocess.DEVNULL)
+            time.sleep(0.3)
+        except Exception:
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            time.sleep(0.15)
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self):
+        if self.proc is None or self.file is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        rows = []
+        with open(self.file.name) as f:
+            for line in f:
+                parts = [x.strip() for x in line.split(",")]
+                if len(parts) >= 9:
+                    rows.append(parts)
+        os.unlink(self.file.name)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[5 + i].lower().startswith("active")})
+
+        def num(x):
+            try:
+                return float(x)
+            except ValueError:
+                return None
+        sm = [num(r[1]) for r in rows if num(r[1])]
+        mx = [num(r[2]) for r in rows if num(r[2])]
+        pw = [num(r[3]) for r in rows if num(r[3])]
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "power_w_max": max(pw) if pw else None, "samples": len(rows), "reasons": reasons}
+
+
+def cpu_baseline(problem, target_s: float):
+    """The oracle (sequential SGD, one thread) on the first R examples, R sized to ~target_s."""
+    import numpy as np
+    import oracle
+    n = problem.n_rows
+    k_mean = problem.nnz / max(n, 1)
+    rows = min(n, 20000)
+    t0 = time.perf_counter()
+    oracle.sgd(problem, epochs=1, rows=rows)
+    dt = time.perf_counter() - t0
+    rows = int(min(n, max(rows, rows * target_s / max(dt, 1e-6))))
+    t0 = time.perf_counter()
+    oracle.sgd(problem, epochs=1, rows=rows)
+    dt = time.perf_counter() - t0
+    nnz = int(problem.row_ptr[rows])
+    del np
+    return {"value": nnz / dt, "unit": UNIT, "cores": 1, "kind": "oracle",
+            "sample": f"first {rows} of {n} examples ({nnz} nnz, k~{k_mean:.0f}), 1 epoch, sequential "
+                      f"Algorithm-1 SGD in plain C, {dt:.1f} s"}
+
+
+def workload_config(name, problem, mode):
+    import synthdata
+    spec = synthdata.WORKLOADS[name]
+    desc = (f"{name}: {problem.n_rows} examples x {problem.n_cols} features, {spec['k']} nnz/row "
+            f"{spec['ids']}{' s=' + str(spec['zipf_s']) if spec['ids'] == 'zipf' else ''} ids, "
+            f"{spec['vals']} values, {spec['loss']} loss, eta={spec['eta']}, {spec['epochs']} epochs")
+    in_bytes = problem.nnz * (4 + (0 if problem.val is None else 4)) + 8 * (problem.n_rows + 1)
+    return {"workload": desc, "schedule": mode, "epochs": problem.epochs,
+            "nnz": problem.nnz, "n_rows": problem.n_rows, "n_cols": problem.n_cols,
+            "l2": ("inputs larger than L2: CSR %.2f GB and w %.2f GB vs %d MB L2" %
+                   (in_bytes / 1e9, 4 * problem.n_cols / 1e9, L2_BYTES // 2 ** 20)
+                   if in_bytes > L2_BYTES else "inputs fit in L2")}
+
+
+# ---------------------------------------------------------------- our implementation
+def run_ours(args, rank, world, local_rank):
+    import numpy as np
+    import torch
+
+    import synthdata
+    import paper_1508_00703_gb300 as pdb
+
+    torch.cuda.set_device(local_rank)
+    overrides = {} if args.rows is None else {"n_rows": args.rows}
+    p = synthdata.generate(args.workload, seed=synthdata.DATA_SEED + rank, **overrides)
+    E = p.epochs
+    mode = pdb.PDB_SCHED_READY if args.mode == "ready" else pdb.PDB_SCHED_LEVELS
+    X = pdb.Csr.from_problem(p)
+    y = torch.from_numpy(p.y).cuda()
+    w = torch.zeros(p.n_cols, dtype=torch.float32, device="cuda")
+    stream = torch.cuda.current_stream()
+
+    def step():
+        w.zero_()
+        c = pdb.pdb_build_conflicts(X, stream)
+        s = pdb.pdb_schedule_build(c, mode, stream)
+        pdb.pdb_sgd_epoch(X, y, c, s, w, p.loss, p.eta, E, stream=stream)
+        return c, s
+
+    for _ in range(args.warmup):
+        c, s = step()
+        pdb.check_status(c, stream)
+        del c, s
+
+    phases = []
+    barrier(world)
+    torch.cuda.synchronize()
+    launches0 = pdb.pdb_launch_count()
+    with ClockSampler(local_rank) as clk:
+        ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        ev0.record(stream)
+        for _ in range(args.steps):
+            c, s = step()
+            phases.append(pdb.pdb_get_stats(c, s))   # synchronizes; frees the step's handles below
+            del c, s
+        ev1.record(stream)
+        torch.cuda.synchronize()
+    barrier(world)
+    launches = pdb.pdb_launch_count() - launches0
+    ms_step = ev0.elapsed_time(ev1) / args.steps
+    ms_step = reduce_max(ms_step, world)
+    units = E * p.nnz
+    total_units = reduce_sum(units, world)
+    value = total_units / (ms_step / 1e3)
+
+    # the step's result is checked after timing: parity with the oracle is the tests' job
+    c, s = step()
+    pdb.check_status(c, stream)
+    del c, s
+
+    ms_sgd = statistics.median(ph["ms_sgd"] for ph in phases)
+    ms_build = statistics.median(ph["ms_build"] for ph in phases)
+    ms_sched = statistics.median(ph["ms_schedule"] for ph in phases)
+    peak, peak_kind = measured_peak_hbm()
+    sgd_bytes_per_launch = ALG_BYTES_PER_NNZ * p.nnz + ALG_BYTES_PER_ROW * p.n_rows
+    sgd_launch_ms = ms_sgd / E
+    sgd_gbs = sgd_bytes_per_launch / (sgd_launch_ms / 1e3) / 1e9
+    roofline = {"kernel": "k_sgd_ready" if mode == pdb.PDB_SCHED_READY else "k_sgd_levels",
+                "bound": "hbm", "achieved": round(sgd_gbs, 1), "peak": peak, "unit": "GB/s",
+                "frac": round(sgd_gbs / peak, 4), "traffic": None, "peak_source": peak_kind,
+                "algorithmic_bytes_per_launch": sgd_bytes_per_launch, "launch_ms": round(sgd_launch_ms, 4),
+                "frac_of_8TBs": round(sgd_gbs / 8000.0, 4)}
+    result = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f32", "data": "synthetic (seeded generator, no dataset)",
+        "config": dict(workload_config(args.workload, p, args.mode),
+                       parallelism=f"replicas{world}" if world > 1 else "single GPU"),
+        "roofline": roofline,
+        "phases_ms": {"build_conflicts": ms_build, "schedule": ms_sched, "sgd_all_epochs": ms_sgd},
+        "sgd_only": {"value": units / (ms_sgd / 1e3), "unit": UNIT},
+        "gpu_launches": int(launches),
+        "clocks": clk.summary(),
+    }
+
+    if not args.no_e2e:
+        result["e2e"] = run_e2e(args, p, mode, pdb, torch, world)
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        result["cpu_baseline"] = cpu_baseline(p, args.cpu_seconds)
+    del np
+    return result
+
+
+def run_e2e(args, p, mode, pdb, torch, world):
+    """Same metric through the public API from pinned host buffers: H2D of the
+    inputs and D2H of the trained weights inside the timed region."""
+    stream = torch.cuda.current_stream()
+    h_row = torch.from_numpy(p.row_ptr).pin_memory()
+    h_col = torch.from_numpy(p.col).pin_memory()
+    h_val = None if p.val is None else torch.from_numpy(p.val).pin_memory()
+    h_y = torch.from_numpy(p.y).pin_memory()
+    h_w0 = torch.zeros(p.n_cols, dtype=torch.float32).pin_memory()
+    h_w = torch.empty(p.n_cols, dtype=torch.float32).pin_memory()
+    d_row = torch.empty_like(h_row, device="cuda")
+    d_col = torch.empty_like(h_col, device="cuda")
+    d_val = None if h_val is None else torch.empty_like(h_val, device="cuda")
+    d_y = torch.empty_like(h_y, device="cuda")
+    d_w = torch.empty_like(h_w0, device="cuda")
+    X = pdb.Csr(d_row, d_col, d_val, p.n_cols)
+    h2d = sum(t.numel() * t.element_size() for t in (h_row, h_col, h_val, h_y, h_w0) if t is not None)
+    d2h = h_w.numel() * h_w.element_size()
+
+    def step():
+        d_row.copy_(h_row, non_blocking=True)
+        d_col.copy_(h_col, non_blocking=True)
+        if d_val is not None:
+            d_val.copy_(h_val, non_blocking=True)
+        d_y.copy_(h_y, non_blocking=True)
+        d_w.copy_(h_w0, non_blocking=True)
+        c = pdb.pdb_build_conflicts(X, stream)
+        s = pdb.pdb_schedule_build(c, mode, stream)
+        pdb.pdb_sgd_epoch(X, d_y, c, s, d_w, p.loss, p.eta, p.epochs, stream=stream)
+        h_w.copy_(d_w, non_blocking=True)
+        rc = pdb.pdb_status(c, stream)          # synchronizes: the weights are on the host
+        if rc != 0:
+            raise pdb.PdbError(rc, "e2e step")
+        del c, s
+
+    steps = max(2, min(args.steps, 5))
+    step()
+    barrier(world)
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    for _ in range(steps):
+        step()
+    torch.cuda.synchronize()
+    dt = (time.perf_counter() - t0) / steps
+    dt = reduce_max(dt, world)
+    units = reduce_sum(p.epochs * p.nnz, world)
+    return {"value": units / dt, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+            "ms_per_step": dt * 1e3, "steps": steps}
+
+
+# ---------------------------------------------------------------- reference arm: the CPU oracle
+def run_reference(args, rank, world):
+    import synthdata
+    import oracle
+
+    overrides = {} if args.rows is None else {"n_rows": args.rows}
+    p = synthdata.generate(args.workload, **overrides)
+    n = p.n_rows
+    per_step_s = max(1.0, min(10.0, 150.0 / max(1, args.steps + args.warmup)))
+    rows = min(n, 20000)
+    t0 = time.perf_counter()
+    oracle.sgd(p, epochs=1, rows=rows)
+    dt = time.perf_counter() - t0
+    rows = int(min(n, max(rows, rows * per_step_s / max(dt, 1e-6))))
+    for _ in range(args.warmup):
+        oracle.sgd(p, epochs=1, rows=rows)
+    times = []
+    for _ in range(args.steps):
+        t0 = time.perf_counter()
+        oracle.sgd(p, epochs=1, rows=rows)
+        times.append(time.perf_counter() - t0)
+    nnz = int(p.row_ptr[rows])
+    ms = 1e3 * sum(times) / len(times)
+    value = nnz / (ms / 1e3)
+    sample = (f"first {rows} of {n} examples ({nnz} nnz), 1 epoch per step, sequential Algorithm-1 SGD "
+              f"in plain C on 1 host core")
+    cfg = workload_config(args.workload, p, "sequential")
+    return {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic (seeded generator, no dataset)",
+            "config": cfg,
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+
+
+def main(argv=None):
+    args = parse_args(argv)
+    rank, world, local_rank = dist_env()
+    if args.impl == "reference":
+        if rank != 0:
+            return 0
+        print(json.dumps(run_reference(args, rank, world)), flush=True)
+        return 0
+    if world > 1:
+        import torch
+        import torch.distributed as dist
+        backend = "nccl" if torch.cuda.is_available() else "gloo"
+        if backend == "nccl":
+            torch.cuda.set_device(local_rank)
+        dist.init_process_group(backend=backend)
+    result = run_ours(args, rank, world, local_rank)
+    if rank == 0:
+        print(json.dumps(result), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

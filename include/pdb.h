@@ -201,6 +201,10 @@ const char *pdb_strerror(int code);
  * need to read the borrowed arrays). */
 int pdb_memcpy(void *dst, const void *src, size_t bytes, void *stream);
 
+/* Number of CUDA kernels this library has launched in this process so far
+ * (every launch site counts once per launch). */
+int64_t pdb_launch_count(void);
+
 /* out[i] = the library's device exp of x[i] (device arrays of n floats), the
  * same function the logistic gradient uses. */
 int pdb_eval_expf(const float *x, float *out, int64_t n, void *stream);

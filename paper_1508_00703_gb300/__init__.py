@@ -104,7 +104,7 @@ class pdb_stats(ctypes.Structure):
 EXPORTS = ["pdb_build_conflicts", "pdb_conflicts_arrays", "pdb_schedule_build", "pdb_schedule_levels",
            "pdb_schedule_ready",
            "pdb_sgd_epoch", "pdb_bsp_epoch", "pdb_status", "pdb_get_stats", "pdb_conflicts_free",
-           "pdb_schedule_free", "pdb_strerror", "pdb_memcpy", "pdb_eval_expf"]
+           "pdb_schedule_free", "pdb_strerror", "pdb_memcpy", "pdb_eval_expf", "pdb_launch_count"]
 
 
 def load(path: str | None = None):
@@ -133,6 +133,8 @@ def load(path: str | None = None):
         lib.pdb_strerror.restype = ctypes.c_char_p
         lib.pdb_memcpy.argtypes = [P, P, ctypes.c_size_t, P]
         lib.pdb_eval_expf.argtypes = [P, P, I64, P]
+        lib.pdb_launch_count.argtypes = []
+        lib.pdb_launch_count.restype = I64
         _lib = lib
     return _lib
 
@@ -275,6 +277,10 @@ def pdb_memcpy(dst_ptr: int, src_ptr: int, nbytes: int, stream=None):
 
 def pdb_eval_expf(x, out, stream=None):
     _check(load().pdb_eval_expf(_ptr(x), _ptr(out), x.numel(), _stream(stream)), "pdb_eval_expf")
+
+
+def pdb_launch_count() -> int:
+    return int(load().pdb_launch_count())
 
 
 def pdb_strerror(code: int) -> str:

@@ -146,12 +146,16 @@ __global__ __launch_bounds__(THREADS) void k_levels_kahn(int32_t n_rows, const i
         int slot = warp_append(zero, &ctl->tail);
         if (zero) queue[slot] = t;
     }
-    if (!grid_sync(&ctl->bar, status, timeout)) return;
-    int head = 0, end = ld_acquire_i(&ctl->tail), lvl = 0, widest = 0;
+    if (!grid_sync(&ctl->bar, status, timeout, &ctl->tail, &ctl->end)) return;
+    int head = 0, end = ld_acquire_i(&ctl->end), lvl = 0, widest = 0;
     while (head < end) {
         widest = max(widest, end - head);
         for (int i = head + gw; i < end; i += nw) {
             int t = __ldcg(queue + i);
+            if (t < 0 || t >= n_rows) {        // cannot happen with a consistent queue
+                set_status(status, PDB_EFAULT);
+                continue;
+            }
             int64_t b = row_ptr[t], e = row_ptr[t + 1];
             for (int64_t p0 = b; p0 < e; p0 += 32) {
                 int64_t p = p0 + lane;
@@ -171,9 +175,9 @@ __global__ __launch_bounds__(THREADS) void k_levels_kahn(int32_t n_rows, const i
                 }
             }
         }
-        if (!grid_sync(&ctl->bar, status, timeout)) return;
+        if (!grid_sync(&ctl->bar, status, timeout, &ctl->tail, &ctl->end)) return;
         head = end;
-        end = ld_acquire_i(&ctl->tail);
+        end = ld_acquire_i(&ctl->end);
         ++lvl;
     }
     if (blockIdx.x == 0 && threadIdx.x == 0) {
@@ -293,18 +297,18 @@ int pdb_build_conflicts(const pdb_csr *X, pdb_conflicts **out, void *stream)
     cudaMemsetAsync(c->status, 0, sizeof(int) * 2, s);
     cudaMemsetAsync(c->max_chain, 0, sizeof(int), s);
     cudaMemcpyAsync(c->row_ptr, X->row_ptr, sizeof(int64_t) * (N + 1), cudaMemcpyDeviceToDevice, s);
-    k_validate_rows<<<grid_1d(N + 1), 256, 0, s>>>(X->row_ptr, N, nnz, c->status);
-    if (nnz > 0) k_validate_cols<<<grid_1d(nnz), 256, 0, s>>>(X->col, nnz, F, c->status);
-    if (N > 0) k_row_of<<<grid_1d(N * 32), 256, 0, s>>>(X->row_ptr, N, c->row_of, c->status);
+    k_validate_rows<<<grid_1d(N + 1), 256, 0, s>>>(X->row_ptr, N, nnz, c->status); note_launch();
+    if (nnz > 0) k_validate_cols<<<grid_1d(nnz), 256, 0, s>>>(X->col, nnz, F, c->status); note_launch();
+    if (N > 0) k_row_of<<<grid_1d(N * 32), 256, 0, s>>>(X->row_ptr, N, c->row_of, c->status); note_launch();
     // (feature, position) pairs sorted by feature, stable: positions stay in data order
     rc = radix_sort((const uint32_t *)X->col, nullptr, skey, c->csc_pos, tkey, tval, nnz, bits_for(F > 0 ? F - 1 : 0),
                     c->status, s);
     if (rc == PDB_OK) rc = segment_bounds(skey, nnz, F, nullptr, c->feat_ptr, c->status, s);
     if (rc == PDB_OK && nnz > 0)
         k_link<<<grid_1d(nnz), 256, 0, s>>>(skey, c->csc_pos, nnz, c->feat_ptr, c->prev, c->next, c->rank,
-                                            c->max_chain, c->status);
+                                            c->max_chain, c->status); note_launch();
     if (rc == PDB_OK && N > 0)
-        k_row_links<<<grid_1d(N * 32), 256, 0, s>>>(X->row_ptr, N, c->prev, c->npred, c->status);
+        k_row_links<<<grid_1d(N * 32), 256, 0, s>>>(X->row_ptr, N, c->prev, c->npred, c->status); note_launch();
     release(skey, s);
     release(tkey, s);
     release(tval, s);
@@ -381,7 +385,7 @@ int pdb_schedule_build(const pdb_conflicts *c, pdb_sched_mode mode, pdb_schedule
         if (rc == PDB_OK) {
             cudaMemsetAsync(h->ctr, 0, sizeof(unsigned) * F, s);
             if (c->nnz > 0)
-                k_make_gate<<<grid_1d(c->nnz), 256, 0, s>>>(c->rank, c->next, c->nnz, h->gate, c->status);
+                k_make_gate<<<grid_1d(c->nnz), 256, 0, s>>>(c->rank, c->next, c->nnz, h->gate, c->status); note_launch();
         }
     } else {
         rc = rc ? rc : alloc((void **)&h->level, sizeof(int32_t) * N, s);
@@ -406,9 +410,9 @@ int pdb_schedule_build(const pdb_conflicts *c, pdb_sched_mode mode, pdb_schedule
                 void *args[] = {&n32, (void *)&c->row_ptr, (void *)&c->next, (void *)&c->row_of,
                                 (void *)&c->npred, &h->indeg, &h->queue, &h->level, &h->ctl,
                                 (void *)&c->status, &tmo};
-                if (cudaLaunchCooperativeKernel(kern, grid, THREADS, args, 0, s) != cudaSuccess) rc = PDB_ECUDA;
+                if (cudaLaunchCooperativeKernel(kern, grid, THREADS, args, 0, s) != cudaSuccess) rc = PDB_ECUDA; note_launch();
                 if (rc == PDB_OK) {
-                    k_iota_u32_level<<<grid_1d(N), 256, 0, s>>>(h->level, key, n32);
+                    k_iota_u32_level<<<grid_1d(N), 256, 0, s>>>(h->level, key, n32); note_launch();
                     rc = radix_sort(key, nullptr, skey, h->order, tkey, tval, N, bits_for(N), c->status, s);
                 }
                 if (rc == PDB_OK) rc = segment_bounds(skey, N, N, &h->ctl->n_levels, h->level_ptr, c->status, s);

@@ -27,6 +27,7 @@ uint64_t timeout_ns(const pdb_opts *opts);
 int alloc(void **p, size_t bytes, cudaStream_t s);   // stream-ordered, 256-byte aligned
 void release(void *p, cudaStream_t s);
 int bits_for(int64_t max_key);                        // bits to hold values 0..max_key (>= 1)
+void note_launch();                                   // count one kernel launch (pdb_launch_count)
 
 // Stable LSD radix sort of (key, value) pairs, 8-bit digits.  vals_in ==
 // nullptr means value = index.  Sorted pairs land in keys_out/vals_out;
@@ -85,7 +86,11 @@ struct GridBarrier {
     unsigned gen;
 };
 
-__device__ __forceinline__ bool grid_sync(GridBarrier *bar, int *status, uint64_t timeout)
+// snap_src/snap_dst (optional): the last arriver copies *snap_src into
+// *snap_dst before it releases the others, so every block reads one value
+// that no block can change until the next barrier.
+__device__ __forceinline__ bool grid_sync(GridBarrier *bar, int *status, uint64_t timeout, int *snap_src = nullptr,
+                                          int *snap_dst = nullptr)
 {
     __shared__ int s_ok;
     __syncthreads();
@@ -95,6 +100,7 @@ __device__ __forceinline__ bool grid_sync(GridBarrier *bar, int *status, uint64_
         __threadfence();
         unsigned arrived = atomicAdd(&bar->count, 1u);
         if (arrived == gridDim.x - 1) {
+            if (snap_src) *(volatile int *)snap_dst = atomicAdd(snap_src, 0);
             atomicExch(&bar->count, 0u);
             __threadfence();
             st_release(&bar->gen, gen + 1);
@@ -189,7 +195,7 @@ struct LevelCtl {
     int tail;                 // frontier queue length
     int n_levels;             // L
     int max_width;
-    int pad;
+    int end;                  // frontier end snapshot taken at each grid barrier
     pdb::GridBarrier bar;
 };
 

@@ -78,7 +78,7 @@ __device__ __forceinline__ void sgd_example(int t, const int64_t *__restrict__ r
 // Persistent cooperative kernel: level l's examples are spread over all
 // warps, a grid barrier closes the level (the read barrier of the next BSP
 // step and the write barrier of this one, Algorithm 2a per level).
-__global__ __launch_bounds__(THREADS) void k_sgd_levels(const int64_t *__restrict__ row_ptr,
+__global__ __launch_bounds__(THREADS) void k_sgd_levels(int32_t n_rows, const int64_t *__restrict__ row_ptr,
                                                         const int32_t *__restrict__ col, const float *__restrict__ val,
                                                         const float *__restrict__ y, const int32_t *__restrict__ order,
                                                         const int64_t *__restrict__ level_ptr, const LevelCtl *ctl,
@@ -92,7 +92,14 @@ __global__ __launch_bounds__(THREADS) void k_sgd_levels(const int64_t *__restric
     for (int ep = 0; ep < epochs; ++ep)
         for (int l = 0; l < L; ++l) {
             const int64_t b = level_ptr[l], e = level_ptr[l + 1];
-            for (int64_t i = b + gw; i < e; i += nw) sgd_example(order[i], row_ptr, col, val, y, w, loss, eta);
+            for (int64_t i = b + gw; i < e; i += nw) {
+                const int t = order[i];
+                if (t < 0 || t >= n_rows) {      // cannot happen with a consistent schedule
+                    set_status(status, PDB_EFAULT);
+                    continue;
+                }
+                sgd_example(t, row_ptr, col, val, y, w, loss, eta);
+            }
             if (!grid_sync(bar, status, timeout)) return;
         }
 }
@@ -254,8 +261,14 @@ __global__ __launch_bounds__(THREADS) void k_bsp(int32_t n_rows, int64_t batch, 
                 const int32_t j = bcol[s];
                 if (s > s0 && bcol[s - 1] == j) continue;
                 float delta = 0.0f;
-                for (int64_t q = s; q < s1 && bcol[q] == j; ++q)
-                    delta = __fadd_rn(delta, __fmul_rn(__ldcg(cbuf + (brow[q] - r0)), bval[q]));
+                for (int64_t q = s; q < s1 && bcol[q] == j; ++q) {
+                    const int64_t i = brow[q] - r0;
+                    if (i < 0 || i >= r1 - r0) {     // cannot happen with a consistent batch sort
+                        set_status(status, PDB_EFAULT);
+                        break;
+                    }
+                    delta = __fadd_rn(delta, __fmul_rn(__ldcg(cbuf + i), bval[q]));
+                }
                 __stcg(w + j, __fsub_rn(__ldcg(w + j), delta));
             }
             if (!grid_sync(bar, status, timeout)) return;
@@ -329,17 +342,17 @@ int pdb_sgd_epoch(const pdb_csr *X, const float *y, const pdb_conflicts *c, cons
             const int64_t *rp = X->row_ptr;
             const int32_t *cl = X->col;
             const float *vl = X->val;
-            void *args[] = {(void *)&rp,        (void *)&cl, (void *)&vl,       (void *)&y,
+            void *args[] = {(void *)&n32, (void *)&rp,        (void *)&cl, (void *)&vl,       (void *)&y,
                             (void *)&h->order,  (void *)&h->level_ptr, (void *)&h->ctl, (void *)&w,
                             (void *)&lossi,     (void *)&eta, (void *)&n_epochs, (void *)&h->bar,
                             (void *)&cm->status, (void *)&tmo};
-            if (cudaLaunchCooperativeKernel(kern, grid, THREADS, args, 0, s) != cudaSuccess) rc = PDB_ECUDA;
+            if (cudaLaunchCooperativeKernel(kern, grid, THREADS, args, 0, s) != cudaSuccess) rc = PDB_ECUDA; note_launch();
         } else {
             int grid = persistent_grid((const void *)k_sgd_ready, opts);
             for (int ep = 0; ep < n_epochs; ++ep) {
                 cudaMemsetAsync(h->ticket, 0, sizeof(unsigned long long), s);
                 k_sgd_ready<<<grid, THREADS, 0, s>>>(n32, X->row_ptr, X->col, X->val, y, h->gate, h->ctr, w, lossi,
-                                                     eta, h->ticket, cm->status, tmo);
+                                                     eta, h->ticket, cm->status, tmo); note_launch();
             }
         }
     }
@@ -382,12 +395,12 @@ int pdb_bsp_epoch(const pdb_csr *X, const float *y, const pdb_conflicts *c, floa
         if (rc == PDB_OK) {
             cudaMemsetAsync(bar, 0, sizeof(GridBarrier), s);
             if (nnz > 0) {
-                k_bsp_keys<<<grid_1d(nnz), 256, 0, s>>>(c->csc_pos, c->row_of, nnz, batch, key, cm->status);
+                k_bsp_keys<<<grid_1d(nnz), 256, 0, s>>>(c->csc_pos, c->row_of, nnz, batch, key, cm->status); note_launch();
                 // stable by batch: inside a batch the feature-major CSC order survives
                 rc = radix_sort(key, c->csc_pos, skey, bpos, tkey, tval, nnz, bits_for(n_batches - 1), cm->status, s);
                 if (rc == PDB_OK)
                     k_bsp_gather<<<grid_1d(nnz), 256, 0, s>>>(bpos, X->col, X->val, c->row_of, nnz, bcol, brow, bval,
-                                                              cm->status);
+                                                              cm->status); note_launch();
             }
             if (rc == PDB_OK) rc = segment_bounds(skey, nnz, n_batches, nullptr, bptr, cm->status, s);
             if (rc == PDB_OK) {
@@ -402,7 +415,7 @@ int pdb_bsp_epoch(const pdb_csr *X, const float *y, const pdb_conflicts *c, floa
                 void *args[] = {&n32,  &batch, (void *)&n_batches, (void *)&rp, (void *)&cl, (void *)&vl,
                                 (void *)&y, &bptr, &bcol, &brow, &bval, &cbuf, &w, &lossi, &eta, &n_epochs, &bar,
                                 (void *)&cm->status, &tmo};
-                if (cudaLaunchCooperativeKernel(kern, grid, THREADS, args, 0, s) != cudaSuccess) rc = PDB_ECUDA;
+                if (cudaLaunchCooperativeKernel(kern, grid, THREADS, args, 0, s) != cudaSuccess) rc = PDB_ECUDA; note_launch();
             }
         }
         for (void *p : {(void *)key, (void *)skey, (void *)tkey, (void *)bpos, (void *)tval, (void *)bcol, (void *)brow,
@@ -420,7 +433,7 @@ int pdb_eval_expf(const float *x, float *out, int64_t n, void *stream)
 {
     if (n < 0 || (n > 0 && (!x || !out))) return PDB_EINVAL;
     if (n == 0) return PDB_OK;
-    k_eval_expf<<<grid_1d(n), 256, 0, (cudaStream_t)stream>>>(x, out, n);
+    k_eval_expf<<<grid_1d(n), 256, 0, (cudaStream_t)stream>>>(x, out, n); note_launch();
     return cudaPeekAtLastError() == cudaSuccess ? PDB_OK : PDB_ECUDA;
 }
 

@@ -11,6 +11,7 @@
 #include <cuda_runtime.h>
 
 #include <algorithm>
+#include <atomic>
 
 #include "common.cuh"
 
@@ -82,6 +83,9 @@ void release(void *p, cudaStream_t s)
 {
     if (p) cudaFreeAsync(p, s);
 }
+
+static std::atomic<long long> g_launches{0};
+void note_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
 
 int bits_for(int64_t max_key)
 {
@@ -289,11 +293,11 @@ int radix_sort(const uint32_t *keys_in, const int32_t *vals_in, uint32_t *keys_o
         uint32_t *ko = to_out ? keys_out : keys_tmp;
         int32_t *vo = to_out ? vals_out : vals_tmp;
         int shift = 8 * p;
-        k_rs_hist<<<(unsigned)n_tiles, RS_THREADS, 0, s>>>(kin, n, shift, hist, status);
-        k_rs_chunk_sum<<<(unsigned)n_chunks, 256, 0, s>>>(hist, n_tiles, csum, status);
-        k_rs_chunk_scan<<<1, 256, 0, s>>>(csum, n_chunks, cbase, status);
-        k_rs_chunk_down<<<(unsigned)n_chunks, 256, 0, s>>>(hist, n_tiles, cbase, status);
-        k_rs_scatter<<<(unsigned)n_tiles, RS_THREADS, 0, s>>>(kin, vin, ko, vo, n, shift, hist, status);
+        k_rs_hist<<<(unsigned)n_tiles, RS_THREADS, 0, s>>>(kin, n, shift, hist, status); note_launch();
+        k_rs_chunk_sum<<<(unsigned)n_chunks, 256, 0, s>>>(hist, n_tiles, csum, status); note_launch();
+        k_rs_chunk_scan<<<1, 256, 0, s>>>(csum, n_chunks, cbase, status); note_launch();
+        k_rs_chunk_down<<<(unsigned)n_chunks, 256, 0, s>>>(hist, n_tiles, cbase, status); note_launch();
+        k_rs_scatter<<<(unsigned)n_tiles, RS_THREADS, 0, s>>>(kin, vin, ko, vo, n, shift, hist, status); note_launch();
         kin = ko;
         vin = vo;
     }
@@ -329,12 +333,14 @@ int segment_bounds(const uint32_t *sorted_keys, int64_t n, int64_t n_bins, const
                    const int *status, cudaStream_t s)
 {
     if (n == 0) {
-        k_fill_i64<<<64, 256, 0, s>>>(ptr, n_bins, n_bins_dev, 0);
+        k_fill_i64<<<64, 256, 0, s>>>(ptr, n_bins, n_bins_dev, 0); note_launch();
     } else {
         int64_t blocks = std::min<int64_t>((n + 255) / 256, 65536);
-        k_segment_bounds<<<(unsigned)blocks, 256, 0, s>>>(sorted_keys, n, n_bins, n_bins_dev, ptr, status);
+        k_segment_bounds<<<(unsigned)blocks, 256, 0, s>>>(sorted_keys, n, n_bins, n_bins_dev, ptr, status); note_launch();
     }
     return cudaPeekAtLastError() == cudaSuccess ? PDB_OK : PDB_ECUDA;
 }
 
 }  // namespace pdb
+
+extern "C" int64_t pdb_launch_count(void) { return (int64_t)pdb::g_launches.load(); }
