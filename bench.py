@@ -47,6 +47,8 @@ def parse_args(argv=None):
     ap.add_argument("--workload", default="low-conflict")
     ap.add_argument("--mode", choices=["ready", "levels"], default="ready")
     ap.add_argument("--rows", type=int, default=None, help="override the workload's example count")
+    ap.add_argument("--ticket-chunk", type=int, default=0, help="READY engine: examples per ticket (0 = default)")
+    ap.add_argument("--blocks-per-sm", type=int, default=0)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=10.0, help="target length of the CPU oracle sample")
@@ -103,10 +105,30 @@ class ClockSampler:
               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
               "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
 
-    def __init__(self, gpu_index: int):
-        self.gpu = gpu_index
+    def __init__(self, local_rank: int):
+        self.gpu = self.smi_id(local_rank)
         self.proc = None
         self.file = None
+
+    @staticmethod
+    def smi_id(local_rank: int) -> str:
+        """nvidia-smi id of the CUDA device this process uses (PCI bus id when torch knows it)."""
+        try:
+            import torch
+            props = torch.cuda.get_device_properties(local_rank)
+            bus = getattr(props, "pci_bus_id", None)
+            dom = getattr(props, "pci_domain_id", None)
+            dev = getattr(props, "pci_device_id", None)
+            if bus is not None and dom is not None and dev is not None:
+                return "%08X:%02X:%02X.0" % (dom, bus, dev)
+        except Exception:
+            pass
+        vis = os.environ.get("CUDA_VISIBLE_DEVICES")
+        if vis:
+            ids = [x.strip() for x in vis.split(",") if x.strip()]
+            if local_rank < len(ids):
+                return ids[local_rank]
+        return str(local_rank)
 
     def __enter__(self):
         try:
@@ -139,7 +161,7 @@ class ClockSampler:
                     rows.append(parts)
         os.unlink(self.file.name)
         if not rows:
-            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"], "gpu": self.gpu}
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
         reasons = sorted({names[i] for r in rows for i in range(4) if r[5 + i].lower().startswith("active")})
 
@@ -152,7 +174,7 @@ class ClockSampler:
         mx = [num(r[2]) for r in rows if num(r[2])]
         pw = [num(r[3]) for r in rows if num(r[3])]
         return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
-                "power_w_max": max(pw) if pw else None, "samples": len(rows), "reasons": reasons}
+                "power_w_max": max(pw) if pw else None, "samples": len(rows), "reasons": reasons, "gpu": self.gpu}
 
 
 def cpu_baseline(problem, target_s: float):
@@ -207,12 +229,13 @@ def run_ours(args, rank, world, local_rank):
     y = torch.from_numpy(p.y).cuda()
     w = torch.zeros(p.n_cols, dtype=torch.float32, device="cuda")
     stream = torch.cuda.current_stream()
+    opts = dict(ticket_chunk=args.ticket_chunk, blocks_per_sm=args.blocks_per_sm)
 
     def step():
         w.zero_()
         c = pdb.pdb_build_conflicts(X, stream)
         s = pdb.pdb_schedule_build(c, mode, stream)
-        pdb.pdb_sgd_epoch(X, y, c, s, w, p.loss, p.eta, E, stream=stream)
+        pdb.pdb_sgd_epoch(X, y, c, s, w, p.loss, p.eta, E, opts=opts, stream=stream)
         return c, s
 
     for _ in range(args.warmup):
@@ -247,11 +270,12 @@ def run_ours(args, rank, world, local_rank):
     del c, s
 
     ms_sgd = statistics.median(ph["ms_sgd"] for ph in phases)
+    ms_kern = statistics.median(ph["ms_sgd_kernels"] for ph in phases)
     ms_build = statistics.median(ph["ms_build"] for ph in phases)
     ms_sched = statistics.median(ph["ms_schedule"] for ph in phases)
     peak, peak_kind = measured_peak_hbm()
     sgd_bytes_per_launch = ALG_BYTES_PER_NNZ * p.nnz + ALG_BYTES_PER_ROW * p.n_rows
-    sgd_launch_ms = ms_sgd / E
+    sgd_launch_ms = ms_kern / E
     sgd_gbs = sgd_bytes_per_launch / (sgd_launch_ms / 1e3) / 1e9
     roofline = {"kernel": "k_sgd_ready" if mode == pdb.PDB_SCHED_READY else "k_sgd_levels",
                 "bound": "hbm", "achieved": round(sgd_gbs, 1), "peak": peak, "unit": "GB/s",
@@ -263,9 +287,11 @@ def run_ours(args, rank, world, local_rank):
         "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f32", "data": "synthetic (seeded generator, no dataset)",
         "config": dict(workload_config(args.workload, p, args.mode),
-                       parallelism=f"replicas{world}" if world > 1 else "single GPU"),
+                       parallelism=f"replicas{world}" if world > 1 else "single GPU",
+                       ticket_chunk=args.ticket_chunk or 2),
         "roofline": roofline,
-        "phases_ms": {"build_conflicts": ms_build, "schedule": ms_sched, "sgd_all_epochs": ms_sgd},
+        "phases_ms": {"build_conflicts": ms_build, "schedule": ms_sched, "sgd_all_epochs": ms_sgd,
+                      "sgd_update_kernels": ms_kern},
         "sgd_only": {"value": units / (ms_sgd / 1e3), "unit": UNIT},
         "gpu_launches": int(launches),
         "clocks": clk.summary(),
@@ -307,7 +333,8 @@ def run_e2e(args, p, mode, pdb, torch, world):
         d_w.copy_(h_w0, non_blocking=True)
         c = pdb.pdb_build_conflicts(X, stream)
         s = pdb.pdb_schedule_build(c, mode, stream)
-        pdb.pdb_sgd_epoch(X, d_y, c, s, d_w, p.loss, p.eta, p.epochs, stream=stream)
+        pdb.pdb_sgd_epoch(X, d_y, c, s, d_w, p.loss, p.eta, p.epochs,
+                          opts=dict(ticket_chunk=args.ticket_chunk, blocks_per_sm=args.blocks_per_sm), stream=stream)
         h_w.copy_(d_w, non_blocking=True)
         rc = pdb.pdb_status(c, stream)          # synchronizes: the weights are on the host
         if rc != 0:

@@ -85,15 +85,16 @@ typedef enum { PDB_LOSS_LOGISTIC = 0, PDB_LOSS_SQUARED = 1, PDB_LOSS_HINGE = 2 }
  *           per level (each level is one BSP step over disjoint examples,
  *           Theorem 3)
  *   READY   per-feature ready counters: an occurrence of feature j with rank
- *           r reads w_j once the counter of j equals r and sets it to r + 1
- *           after writing (the read protocol of Section 5 with the
- *           iteration number counted per feature); no barrier at all */
+ *           r reads w_j once the iteration number of j equals r and
+ *           publishes r + 1 with its write (the read protocol of Section 5
+ *           with the iteration number counted per feature); no barrier at
+ *           all.  The number lives in the same 64-bit word as the weight. */
 typedef enum { PDB_SCHED_LEVELS = 0, PDB_SCHED_READY = 1 } pdb_sched_mode;
 
 /* Launch and wait options; a zeroed struct (or NULL) selects the defaults. */
 typedef struct {
     int32_t blocks_per_sm;     /* persistent grid = blocks_per_sm x #SM; 0 = occupancy maximum */
-    int32_t reserved0;
+    int32_t ticket_chunk;      /* READY: consecutive examples a warp takes per ticket; 0 = 2 */
     double wait_timeout_s;     /* limit of every device-side wait; 0 = 2 seconds */
 } pdb_opts;
 
@@ -105,6 +106,7 @@ typedef struct {
     int64_t max_level_width; /* LEVELS schedule: largest level; else -1 */
     int64_t max_chain;       /* most occurrences of one feature (longest per-feature chain) */
     double ms_build, ms_schedule, ms_sgd, ms_bsp;
+    double ms_sgd_kernels;   /* pdb_sgd_epoch's update kernels alone (no record packing) */
 } pdb_stats;
 
 typedef struct pdb_conflicts pdb_conflicts; /* opaque, library-owned device arrays */
@@ -121,14 +123,19 @@ typedef struct pdb_schedule pdb_schedule;   /* opaque, library-owned device arra
  *   prev[p], next[p] previous / next position holding col[p], -1 if none
  *   rank[p]         number of earlier positions holding col[p]
  * *out receives a new handle (free with pdb_conflicts_free) even when the
- * device later reports a CSR error through pdb_status.  Allocates its arrays
+ * device later reports a CSR error through pdb_status.  The handle keeps
+ * referring to X's arrays (D is immutable, Definition 1): they must stay
+ * valid and unchanged while the handle is in use.  Allocates its arrays
  * stream-ordered on `stream`. */
 int pdb_build_conflicts(const pdb_csr *X, pdb_conflicts **out, void *stream);
 
 /* Borrowed device pointers into the handle (valid until it is freed).  Any
- * output pointer may be NULL. */
+ * output pointer may be NULL.  prev/next/rank are derived from the CSC
+ * order (rank = slot - feat_ptr[j], neighbours in the slot order) and are
+ * materialized by a kernel enqueued on `stream` the first time one of them
+ * is requested; read them after that work has completed. */
 int pdb_conflicts_arrays(const pdb_conflicts *c, const int32_t **csc_pos, const int64_t **feat_ptr,
-                         const int32_t **prev, const int32_t **next, const int32_t **rank);
+                         const int32_t **prev, const int32_t **next, const int32_t **rank, void *stream);
 
 /* Schedule for pdb_sgd_epoch.
  *   LEVELS: level[t] = 1 + max over features j of t with an earlier
@@ -136,9 +143,9 @@ int pdb_conflicts_arrays(const pdb_conflicts *c, const int32_t **csc_pos, const 
  *     conflict path), computed by a Kahn-style frontier sweep; order[N] lists
  *     the examples by level, ascending id inside a level; level_ptr[L+1]
  *     delimits the levels.
- *   READY: the per-feature ready counters (zeroed here; the last occurrence
- *     of each feature in an epoch hands its counter back to 0) and, per
- *     position, the counter value it waits for.
+ *   READY: one 64-bit record per feature, bits(w_j) | version_j << 32,
+ *     filled from w by pdb_sgd_epoch; each position waits for the version
+ *     equal to its occurrence rank (the conflicts' gate array).
  * Allocates stream-ordered on `stream`. */
 int pdb_schedule_build(const pdb_conflicts *c, pdb_sched_mode mode, pdb_schedule **out, void *stream);
 
@@ -149,10 +156,11 @@ int pdb_schedule_levels(const pdb_schedule *s, const int32_t **level, const int3
                         const int64_t **level_ptr, int64_t *n_levels, void *stream);
 
 /* READY schedule arrays (borrowed device pointers, any may be NULL):
- * ctr[n_cols] the per-feature ready counters (0 between calls), gate[nnz]
- * the counter value each position waits for (its rank) with bit 31 set on
- * the last occurrence of its feature.  PDB_ESTATE for a LEVELS schedule. */
-int pdb_schedule_ready(const pdb_schedule *s, const uint32_t **ctr, const uint32_t **gate);
+ * gate[nnz] the version each position waits for (its occurrence rank) with
+ * bit 31 set on the last occurrence of its feature, and records[n_cols]
+ * (weight bits | version << 32, meaningful while pdb_sgd_epoch runs).
+ * PDB_ESTATE for a LEVELS schedule. */
+int pdb_schedule_ready(const pdb_schedule *s, const uint32_t **gate, const uint64_t **records);
 
 /* n_epochs passes of SGD over X in data order (Algorithm 1 with one
  * iteration per example), run concurrently under the schedule's constraint.
@@ -166,7 +174,9 @@ int pdb_schedule_ready(const pdb_schedule *s, const uint32_t **ctr, const uint32
  *   w_j = w_j - (eta*g) * x_tj  for the features of t
  * Each fp32 operation is rounded once, so the result is bitwise the same for
  * every schedule and equals the sequential run (Theorem 2).
- * X and c must be the same data the schedule was built from. */
+ * X and c must be the same data the schedule was built from.  The host
+ * waits for c's build to complete if it has not (the kernel variant depends
+ * on the longest example, which the build records). */
 int pdb_sgd_epoch(const pdb_csr *X, const float *y, const pdb_conflicts *c, const pdb_schedule *s, float *w,
                   pdb_loss loss, float eta, int n_epochs, const pdb_opts *opts, void *stream);
 

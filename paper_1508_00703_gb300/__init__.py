@@ -87,7 +87,7 @@ class pdb_csr(ctypes.Structure):
 
 
 class pdb_opts(ctypes.Structure):
-    _fields_ = [("blocks_per_sm", ctypes.c_int32), ("reserved0", ctypes.c_int32),
+    _fields_ = [("blocks_per_sm", ctypes.c_int32), ("ticket_chunk", ctypes.c_int32),
                 ("wait_timeout_s", ctypes.c_double)]
 
 
@@ -95,7 +95,7 @@ class pdb_stats(ctypes.Structure):
     _fields_ = [("n_rows", ctypes.c_int64), ("n_cols", ctypes.c_int64), ("nnz", ctypes.c_int64),
                 ("n_levels", ctypes.c_int64), ("max_level_width", ctypes.c_int64), ("max_chain", ctypes.c_int64),
                 ("ms_build", ctypes.c_double), ("ms_schedule", ctypes.c_double), ("ms_sgd", ctypes.c_double),
-                ("ms_bsp", ctypes.c_double)]
+                ("ms_bsp", ctypes.c_double), ("ms_sgd_kernels", ctypes.c_double)]
 
     def as_dict(self):
         return {k: getattr(self, k) for k, _ in self._fields_}
@@ -115,7 +115,7 @@ def load(path: str | None = None):
         P, I64, I32 = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int
         PP = ctypes.POINTER(ctypes.c_void_p)
         lib.pdb_build_conflicts.argtypes = [ctypes.POINTER(pdb_csr), PP, P]
-        lib.pdb_conflicts_arrays.argtypes = [P, PP, PP, PP, PP, PP]
+        lib.pdb_conflicts_arrays.argtypes = [P, PP, PP, PP, PP, PP, P]
         lib.pdb_schedule_build.argtypes = [P, I32, PP, P]
         lib.pdb_schedule_levels.argtypes = [P, PP, PP, PP, ctypes.POINTER(I64), P]
         lib.pdb_schedule_ready.argtypes = [P, PP, PP]
@@ -212,10 +212,11 @@ def pdb_build_conflicts(X: Csr, stream=None) -> Conflicts:
     return Conflicts(h, X.struct.n_rows, X.struct.n_cols, X.struct.nnz)
 
 
-def pdb_conflicts_arrays(c: Conflicts) -> dict:
+def pdb_conflicts_arrays(c: Conflicts, stream=None) -> dict:
     """Borrowed device pointers (ints) of csc_pos, feat_ptr, prev, next, rank."""
     ptrs = [ctypes.c_void_p() for _ in range(5)]
-    _check(load().pdb_conflicts_arrays(c.handle, *[ctypes.byref(p) for p in ptrs]), "pdb_conflicts_arrays")
+    _check(load().pdb_conflicts_arrays(c.handle, *[ctypes.byref(p) for p in ptrs], _stream(stream)),
+           "pdb_conflicts_arrays")
     return dict(zip(["csc_pos", "feat_ptr", "prev", "next", "rank"], [p.value for p in ptrs]))
 
 
@@ -234,10 +235,10 @@ def pdb_schedule_levels(s: Schedule, stream=None) -> dict:
 
 
 def pdb_schedule_ready(s: Schedule) -> dict:
-    """Borrowed device pointers (ints) of the READY schedule's ctr and gate arrays."""
+    """Borrowed device pointers (ints) of the READY schedule's gate and records arrays."""
     ptrs = [ctypes.c_void_p() for _ in range(2)]
     _check(load().pdb_schedule_ready(s.handle, *[ctypes.byref(p) for p in ptrs]), "pdb_schedule_ready")
-    return dict(ctr=ptrs[0].value, gate=ptrs[1].value)
+    return dict(gate=ptrs[0].value, records=ptrs[1].value)
 
 
 def _opts(opts):

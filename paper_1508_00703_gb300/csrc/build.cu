@@ -6,6 +6,14 @@
 // With chunk = feature and iteration = example, that number becomes the
 // per-feature occurrence rank, and the constraint links each occurrence to
 // the previous occurrence of its feature: the chains built here.
+//
+// Layout: the (feature, position) pairs are stable-sorted by feature into
+// csc_pos (one slot per nonzero, feature-major, data order inside a
+// feature) delimited by feat_ptr.  The only position-indexed array written
+// by a scatter is gate: the occurrence rank of each position (the read
+// protocol's iteration number) with bit 31 marking the feature's last
+// occurrence.  prev and next of a position follow from gate, feat_ptr and
+// csc_pos by gathers and are materialized only when a caller asks for them.
 #include <cuda_runtime.h>
 
 #include <algorithm>
@@ -19,87 +27,104 @@ using namespace pdb;
 
 namespace {
 
+enum { INFO_STATUS = 0, INFO_MAX_CHAIN = 1, INFO_MAX_ROW = 2, INFO_UNSORTED = 3, INFO_WORDS = 4 };
+
 // row_ptr[0] = 0, row_ptr[N] = nnz, nondecreasing (Definition 1: D is a list of examples)
-__global__ void k_validate_rows(const int64_t *__restrict__ row_ptr, int64_t n_rows, int64_t nnz, int *status)
+__global__ void k_validate_rows(const int64_t *__restrict__ row_ptr, int64_t n_rows, int64_t nnz, int *info)
 {
     for (int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; t <= n_rows;
          t += (int64_t)gridDim.x * blockDim.x) {
         int64_t a = row_ptr[t];
         bool bad = (t == 0 && a != 0) || (t == n_rows && a != nnz) || (t < n_rows && row_ptr[t + 1] < a) ||
                    a < 0 || a > nnz;
-        if (bad) set_status(status, PDB_EINVAL);
+        if (bad) set_status(info, PDB_EINVAL);
     }
 }
 
-// ids in [0, n_cols)
-__global__ void k_validate_cols(const int32_t *__restrict__ col, int64_t nnz, int64_t n_cols, int *status)
+// One warp per example: ids in [0, n_cols) (else ERANGE), row_of, the
+// longest row, and whether the row's ids are strictly increasing (a row
+// that is cannot hold a repeated id; only unsorted rows need the slot check).
+__global__ void k_rows_scan(const int64_t *__restrict__ row_ptr, const int32_t *__restrict__ col, int64_t n_rows,
+                            int64_t n_cols, int32_t *__restrict__ row_of, int *info)
 {
-    bool bad = false;
-    for (int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; p < nnz; p += (int64_t)gridDim.x * blockDim.x) {
-        int32_t j = col[p];
-        bad |= (j < 0) || ((int64_t)j >= n_cols);
-    }
-    if (__any_sync(FULL, bad) && bad) set_status(status, PDB_ERANGE);
-}
-
-// row_of[p] = example holding position p (one warp per example)
-__global__ void k_row_of(const int64_t *__restrict__ row_ptr, int64_t n_rows, int32_t *__restrict__ row_of,
-                         const int *status)
-{
-    if (read_status(status)) return;
+    if (read_status(info)) return;
     const int lane = threadIdx.x & 31;
     const int64_t gw = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
     const int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    bool bad = false, unsorted = false;
+    int longest = 0;
     for (int64_t t = gw; t < n_rows; t += nw) {
-        int64_t b = row_ptr[t], e = row_ptr[t + 1];
-        for (int64_t p = b + lane; p < e; p += 32) row_of[p] = (int32_t)t;
+        const int64_t b = row_ptr[t], e = row_ptr[t + 1];
+        longest = max(longest, (int)(e - b));
+        for (int64_t p = b + lane; p < e; p += 32) {
+            int32_t j = col[p];
+            bad |= j < 0 || (int64_t)j >= n_cols;
+            unsorted |= p > b && col[p - 1] >= j;
+            row_of[p] = (int32_t)t;
+        }
     }
+    if (__any_sync(FULL, bad) && lane == 0) set_status(info, PDB_ERANGE);
+    if (__any_sync(FULL, unsorted) && lane == 0) atomicExch(info + INFO_UNSORTED, 1);
+    if (lane == 0 && longest > 0) atomicMax(info + INFO_MAX_ROW, longest);
 }
 
-// Chains from the feature-sorted positions: slot s of feature j's run links
-// to its neighbours in the run; rank = offset inside the run.
-__global__ void k_link(const uint32_t *__restrict__ skey, const int32_t *__restrict__ spos, int64_t nnz,
-                       const int64_t *__restrict__ feat_ptr, int32_t *__restrict__ prev, int32_t *__restrict__ next,
-                       int32_t *__restrict__ rank, int *max_chain, const int *status)
+// Slot order: gate[csc_pos[s]] = rank | last-occurrence bit (the one
+// scatter of the build), the longest chain, and -- only when some row is
+// unsorted -- the repeated-id check: two neighbouring slots of one feature
+// in the same example.
+__global__ void k_slots(const uint32_t *__restrict__ skey, const int32_t *__restrict__ spos, int64_t nnz,
+                        const int64_t *__restrict__ feat_ptr, const int32_t *__restrict__ row_of,
+                        uint32_t *__restrict__ gate, int *info)
 {
-    if (read_status(status)) return;
+    if (read_status(info)) return;
+    const bool check_dup = *(volatile int *)(info + INFO_UNSORTED) != 0;
     int longest = 0;
+    bool dup = false;
     for (int64_t s = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; s < nnz; s += (int64_t)gridDim.x * blockDim.x) {
-        uint32_t j = skey[s];
-        int32_t p = spos[s];
-        bool first = s == 0 || skey[s - 1] != j;
-        bool last = s == nnz - 1 || skey[s + 1] != j;
-        int32_t r = (int32_t)(s - feat_ptr[j]);
-        prev[p] = first ? -1 : spos[s - 1];
-        next[p] = last ? -1 : spos[s + 1];
-        rank[p] = r;
-        if (last) longest = max(longest, r + 1);
+        const uint32_t j = skey[s];
+        const int32_t p = spos[s];
+        const bool last = s == nnz - 1 || skey[s + 1] != j;
+        const int64_t r = s - feat_ptr[j];
+        gate[p] = (uint32_t)r | (last ? 0x80000000u : 0u);
+        if (last) longest = max(longest, (int)(r + 1));
+        if (check_dup && s > 0 && skey[s - 1] == j) dup |= row_of[spos[s - 1]] == row_of[p];
     }
     for (int off = 16; off >= 1; off >>= 1) longest = max(longest, __shfl_xor_sync(FULL, longest, off));
-    if ((threadIdx.x & 31) == 0 && longest > 0) atomicMax(max_chain, longest);
+    if ((threadIdx.x & 31) == 0 && longest > 0) atomicMax(info + INFO_MAX_CHAIN, longest);
+    if (__any_sync(FULL, dup) && (threadIdx.x & 31) == 0) set_status(info, PDB_EDUP);
 }
 
-// per example: number of features with an earlier occurrence (in-degree of
-// the conflict DAG) and the repeated-id check (the previous occurrence of a
-// feature lying inside the same row means the id repeats in that row)
-__global__ void k_row_links(const int64_t *__restrict__ row_ptr, int64_t n_rows, const int32_t *__restrict__ prev,
-                            int32_t *__restrict__ npred, int *status)
+// Position order: rank, previous and next occurrence of each position's feature.
+__global__ void k_materialize(const int32_t *__restrict__ col, const uint32_t *__restrict__ gate,
+                              const int32_t *__restrict__ csc_pos, const int64_t *__restrict__ feat_ptr, int64_t nnz,
+                              int32_t *__restrict__ prev, int32_t *__restrict__ next, int32_t *__restrict__ rank,
+                              const int *info)
 {
-    if (read_status(status)) return;
+    if (read_status(info)) return;
+    for (int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; p < nnz; p += (int64_t)gridDim.x * blockDim.x) {
+        const uint32_t g = gate[p];
+        const int32_t r = (int32_t)(g & 0x7fffffffu);
+        const int64_t s = feat_ptr[col[p]] + r;
+        rank[p] = r;
+        prev[p] = r > 0 ? csc_pos[s - 1] : -1;
+        next[p] = (g >> 31) ? -1 : csc_pos[s + 1];
+    }
+}
+
+// per example: number of its positions whose feature occurred before (the
+// in-degree of the example in the conflict DAG, counted per edge)
+__global__ void k_npred(const int64_t *__restrict__ row_ptr, int64_t n_rows, const int32_t *__restrict__ prev,
+                        int32_t *__restrict__ npred, const int *info)
+{
+    if (read_status(info)) return;
     const int lane = threadIdx.x & 31;
     const int64_t gw = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
     const int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
     for (int64_t t = gw; t < n_rows; t += nw) {
-        int64_t b = row_ptr[t], e = row_ptr[t + 1];
+        const int64_t b = row_ptr[t], e = row_ptr[t + 1];
         int cnt = 0;
-        bool dup = false;
-        for (int64_t p = b + lane; p < e; p += 32) {
-            int32_t q = prev[p];
-            cnt += q >= 0;
-            dup |= q >= b;
-        }
+        for (int64_t p = b + lane; p < e; p += 32) cnt += prev[p] >= 0;
         for (int off = 16; off >= 1; off >>= 1) cnt += __shfl_xor_sync(FULL, cnt, off);
-        if (__any_sync(FULL, dup) && lane == 0) set_status(status, PDB_EDUP);
         if (lane == 0) npred[t] = cnt;
     }
 }
@@ -122,7 +147,8 @@ __device__ __forceinline__ int warp_append(bool flag, int *tail)
 // of whose predecessors are in frontiers < l; an example joins frontier l+1
 // when its last incoming edge is consumed, which gives exactly the
 // longest-path level.  One cooperative persistent launch; the frontiers are
-// consecutive ranges of one queue and a grid barrier separates them.
+// consecutive ranges of one queue, a grid barrier separates them, and the
+// barrier's last arriver snapshots the queue end for everybody.
 __global__ __launch_bounds__(THREADS) void k_levels_kahn(int32_t n_rows, const int64_t *__restrict__ row_ptr,
                                                          const int32_t *__restrict__ next,
                                                          const int32_t *__restrict__ row_of,
@@ -187,26 +213,11 @@ __global__ __launch_bounds__(THREADS) void k_levels_kahn(int32_t n_rows, const i
     }
 }
 
-// gate[p] = rank[p] with bit 31 set on the last occurrence of its feature:
-// the ready-counter value the occurrence waits for, and whether its release
-// hands the counter back to 0 for the next epoch
-__global__ void k_make_gate(const int32_t *__restrict__ rank, const int32_t *__restrict__ next, int64_t nnz,
-                            uint32_t *__restrict__ gate, const int *status)
+__global__ void k_level_keys(const int32_t *__restrict__ level, uint32_t *__restrict__ key, int32_t n,
+                             const int *status)
 {
     if (read_status(status)) return;
-    for (int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; p < nnz; p += (int64_t)gridDim.x * blockDim.x)
-        gate[p] = (uint32_t)rank[p] | (next[p] < 0 ? 0x80000000u : 0u);
-}
-
-__global__ void k_iota_u32_level(const int32_t *__restrict__ level, uint32_t *__restrict__ key, int32_t n)
-{
     for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < n; i += gridDim.x * blockDim.x) key[i] = (uint32_t)level[i];
-}
-
-int grid_1d(int64_t n, int threads = 256)
-{
-    int64_t b = (n + threads - 1) / threads;
-    return (int)std::max<int64_t>(1, std::min<int64_t>(b, 152 * 32));
 }
 
 int check_csr(const pdb_csr *X)
@@ -216,6 +227,38 @@ int check_csr(const pdb_csr *X)
     if (!X->row_ptr) return PDB_EINVAL;
     if (X->nnz > 0 && (!X->col || X->n_cols == 0)) return PDB_EINVAL;
     return PDB_OK;
+}
+
+void free_ptrs(std::initializer_list<void *> ptrs)
+{
+    for (void *p : ptrs)
+        if (p) cudaFree(p);
+}
+
+// prev/next/rank of every position (idempotent; enqueued on s)
+int materialize_chains(pdb_conflicts *c, cudaStream_t s)
+{
+    if (c->prev) return PDB_OK;
+    const int64_t nnz = c->nnz;
+    int32_t *prev = nullptr, *next = nullptr, *rank = nullptr;
+    int rc = alloc((void **)&prev, sizeof(int32_t) * nnz, s);
+    rc = rc ? rc : alloc((void **)&next, sizeof(int32_t) * nnz, s);
+    rc = rc ? rc : alloc((void **)&rank, sizeof(int32_t) * nnz, s);
+    if (rc != PDB_OK) {
+        release(prev, s);
+        release(next, s);
+        release(rank, s);
+        return rc;
+    }
+    if (nnz > 0) {
+        k_materialize<<<grid_1d(nnz), 256, 0, s>>>(c->col, c->gate, c->csc_pos, c->feat_ptr, nnz, prev, next, rank,
+                                                   c->status);
+        note_launch();
+    }
+    c->prev = prev;
+    c->next = next;
+    c->rank = rank;
+    return cudaPeekAtLastError() == cudaSuccess ? PDB_OK : PDB_ECUDA;
 }
 
 }  // namespace
@@ -243,12 +286,9 @@ void pdb_conflicts_free(pdb_conflicts *c)
 {
     if (!c) return;
     cudaDeviceSynchronize();
-    void *ptrs[] = {c->row_ptr, c->csc_pos, c->prev,     c->next,     c->rank,
-                    c->row_of,  c->npred,   c->feat_ptr, c->status, c->max_chain};
-    for (void *p : ptrs)
-        if (p) cudaFree(p);
-    cudaEvent_t evs[] = {c->ev0, c->ev1, c->ev_sgd0, c->ev_sgd1, c->ev_bsp0, c->ev_bsp1};
-    for (cudaEvent_t e : evs)
+    free_ptrs({c->csc_pos, c->feat_ptr, c->gate, c->row_of, c->prev, c->next, c->rank, c->npred, c->info});
+    if (c->h_info) cudaFreeHost(c->h_info);
+    for (cudaEvent_t e : {c->ev0, c->ev1, c->ev_sgd0, c->ev_sgd1, c->ev_bsp0, c->ev_bsp1, c->ev_k0, c->ev_k1})
         if (e) cudaEventDestroy(e);
     delete c;
 }
@@ -266,56 +306,59 @@ int pdb_build_conflicts(const pdb_csr *X, pdb_conflicts **out, void *stream)
     c->n_rows = X->n_rows;
     c->n_cols = X->n_cols;
     c->nnz = X->nnz;
+    c->row_ptr = X->row_ptr;
+    c->col = X->col;
+    c->val = X->val;
     const int64_t N = X->n_rows, F = X->n_cols, nnz = X->nnz;
-    for (cudaEvent_t *e : {&c->ev0, &c->ev1, &c->ev_sgd0, &c->ev_sgd1, &c->ev_bsp0, &c->ev_bsp1})
-        if (cudaEventCreate(e) != cudaSuccess) { pdb_conflicts_free(c); return PDB_ECUDA; }
+    for (cudaEvent_t *e : {&c->ev0, &c->ev1, &c->ev_sgd0, &c->ev_sgd1, &c->ev_bsp0, &c->ev_bsp1, &c->ev_k0, &c->ev_k1})
+        if (cudaEventCreate(e) != cudaSuccess) {
+            pdb_conflicts_free(c);
+            return PDB_ECUDA;
+        }
+    if (cudaMallocHost((void **)&c->h_info, sizeof(int) * INFO_WORDS) != cudaSuccess) {
+        cudaGetLastError();
+        pdb_conflicts_free(c);
+        return PDB_ENOMEM;
+    }
+    std::memset(c->h_info, 0, sizeof(int) * INFO_WORDS);
     cudaEventRecord(c->ev0, s);
-    rc = PDB_OK;
-    rc = rc ? rc : alloc((void **)&c->status, sizeof(int) * 2, s);
-    rc = rc ? rc : alloc((void **)&c->max_chain, sizeof(int), s);
-    rc = rc ? rc : alloc((void **)&c->row_ptr, sizeof(int64_t) * (N + 1), s);
+    rc = alloc((void **)&c->info, sizeof(int) * INFO_WORDS, s);
     rc = rc ? rc : alloc((void **)&c->csc_pos, sizeof(int32_t) * nnz, s);
-    rc = rc ? rc : alloc((void **)&c->prev, sizeof(int32_t) * nnz, s);
-    rc = rc ? rc : alloc((void **)&c->next, sizeof(int32_t) * nnz, s);
-    rc = rc ? rc : alloc((void **)&c->rank, sizeof(int32_t) * nnz, s);
+    rc = rc ? rc : alloc((void **)&c->gate, sizeof(uint32_t) * nnz, s);
     rc = rc ? rc : alloc((void **)&c->row_of, sizeof(int32_t) * nnz, s);
-    rc = rc ? rc : alloc((void **)&c->npred, sizeof(int32_t) * N, s);
     rc = rc ? rc : alloc((void **)&c->feat_ptr, sizeof(int64_t) * (F + 1), s);
     uint32_t *skey = nullptr, *tkey = nullptr;
     int32_t *tval = nullptr;
     rc = rc ? rc : alloc((void **)&skey, sizeof(uint32_t) * nnz, s);
     rc = rc ? rc : alloc((void **)&tkey, sizeof(uint32_t) * nnz, s);
     rc = rc ? rc : alloc((void **)&tval, sizeof(int32_t) * nnz, s);
-    if (rc != PDB_OK) {
-        release(skey, s);
-        release(tkey, s);
-        release(tval, s);
-        cudaStreamSynchronize(s);
-        pdb_conflicts_free(c);
-        return rc;
+    c->status = c->info;
+    if (rc == PDB_OK) {
+        cudaMemsetAsync(c->info, 0, sizeof(int) * INFO_WORDS, s);
+        k_validate_rows<<<grid_1d(N + 1), 256, 0, s>>>(X->row_ptr, N, nnz, c->info);
+        note_launch();
+        if (N > 0) {
+            k_rows_scan<<<grid_1d(N * 32), 256, 0, s>>>(X->row_ptr, X->col, N, F, c->row_of, c->info);
+            note_launch();
+        }
+        // (feature, position) pairs sorted by feature, stable: positions stay in data order
+        rc = radix_sort((const uint32_t *)X->col, nullptr, skey, c->csc_pos, tkey, tval, nnz,
+                        bits_for(F > 0 ? F - 1 : 0), c->info, s);
     }
-    cudaMemsetAsync(c->status, 0, sizeof(int) * 2, s);
-    cudaMemsetAsync(c->max_chain, 0, sizeof(int), s);
-    cudaMemcpyAsync(c->row_ptr, X->row_ptr, sizeof(int64_t) * (N + 1), cudaMemcpyDeviceToDevice, s);
-    k_validate_rows<<<grid_1d(N + 1), 256, 0, s>>>(X->row_ptr, N, nnz, c->status); note_launch();
-    if (nnz > 0) k_validate_cols<<<grid_1d(nnz), 256, 0, s>>>(X->col, nnz, F, c->status); note_launch();
-    if (N > 0) k_row_of<<<grid_1d(N * 32), 256, 0, s>>>(X->row_ptr, N, c->row_of, c->status); note_launch();
-    // (feature, position) pairs sorted by feature, stable: positions stay in data order
-    rc = radix_sort((const uint32_t *)X->col, nullptr, skey, c->csc_pos, tkey, tval, nnz, bits_for(F > 0 ? F - 1 : 0),
-                    c->status, s);
-    if (rc == PDB_OK) rc = segment_bounds(skey, nnz, F, nullptr, c->feat_ptr, c->status, s);
-    if (rc == PDB_OK && nnz > 0)
-        k_link<<<grid_1d(nnz), 256, 0, s>>>(skey, c->csc_pos, nnz, c->feat_ptr, c->prev, c->next, c->rank,
-                                            c->max_chain, c->status); note_launch();
-    if (rc == PDB_OK && N > 0)
-        k_row_links<<<grid_1d(N * 32), 256, 0, s>>>(X->row_ptr, N, c->prev, c->npred, c->status); note_launch();
+    if (rc == PDB_OK) rc = segment_bounds(skey, nnz, F, nullptr, c->feat_ptr, c->info, s);
+    if (rc == PDB_OK && nnz > 0) {
+        k_slots<<<grid_1d(nnz), 256, 0, s>>>(skey, c->csc_pos, nnz, c->feat_ptr, c->row_of, c->gate, c->info);
+        note_launch();
+    }
     release(skey, s);
     release(tkey, s);
     release(tval, s);
+    if (rc == PDB_OK) cudaMemcpyAsync(c->h_info, c->info, sizeof(int) * INFO_WORDS, cudaMemcpyDeviceToHost, s);
     cudaEventRecord(c->ev1, s);
     c->timed_build = true;
     if (rc == PDB_OK && cudaPeekAtLastError() != cudaSuccess) rc = PDB_ECUDA;
     if (rc != PDB_OK) {
+        cudaGetLastError();
         cudaStreamSynchronize(s);
         pdb_conflicts_free(c);
         return rc;
@@ -325,9 +368,14 @@ int pdb_build_conflicts(const pdb_csr *X, pdb_conflicts **out, void *stream)
 }
 
 int pdb_conflicts_arrays(const pdb_conflicts *c, const int32_t **csc_pos, const int64_t **feat_ptr,
-                         const int32_t **prev, const int32_t **next, const int32_t **rank)
+                         const int32_t **prev, const int32_t **next, const int32_t **rank, void *stream)
 {
     if (!c) return PDB_EINVAL;
+    pdb_conflicts *cm = const_cast<pdb_conflicts *>(c);
+    if (prev || next || rank) {
+        int rc = materialize_chains(cm, (cudaStream_t)stream);
+        if (rc != PDB_OK) return rc;
+    }
     if (csc_pos) *csc_pos = c->csc_pos;
     if (feat_ptr) *feat_ptr = c->feat_ptr;
     if (prev) *prev = c->prev;
@@ -349,9 +397,7 @@ void pdb_schedule_free(pdb_schedule *s)
 {
     if (!s) return;
     cudaDeviceSynchronize();
-    void *ptrs[] = {s->level, s->order, s->indeg, s->queue, s->level_ptr, s->ctl, s->ctr, s->gate, s->bar, s->ticket};
-    for (void *p : ptrs)
-        if (p) cudaFree(p);
+    free_ptrs({s->level, s->order, s->indeg, s->queue, s->level_ptr, s->ctl, s->rec, s->bar, s->ticket});
     if (s->ev0) cudaEventDestroy(s->ev0);
     if (s->ev1) cudaEventDestroy(s->ev1);
     delete s;
@@ -362,6 +408,7 @@ int pdb_schedule_build(const pdb_conflicts *c, pdb_sched_mode mode, pdb_schedule
     if (!c || !out || (mode != PDB_SCHED_LEVELS && mode != PDB_SCHED_READY)) return PDB_EINVAL;
     *out = nullptr;
     cudaStream_t s = (cudaStream_t)stream;
+    pdb_conflicts *cm = const_cast<pdb_conflicts *>(c);
     pdb_schedule *h = new (std::nothrow) pdb_schedule();
     if (!h) return PDB_ENOMEM;
     h->c = c;
@@ -370,24 +417,26 @@ int pdb_schedule_build(const pdb_conflicts *c, pdb_sched_mode mode, pdb_schedule
         pdb_schedule_free(h);
         return PDB_ECUDA;
     }
-    const int64_t N = c->n_rows, F = c->n_cols;
+    const int64_t N = c->n_rows, F = c->n_cols, nnz = c->nnz;
     cudaEventRecord(h->ev0, s);
-    int rc = PDB_OK;
-    rc = rc ? rc : alloc((void **)&h->bar, sizeof(GridBarrier), s);
+    int rc = alloc((void **)&h->bar, sizeof(GridBarrier), s);
     rc = rc ? rc : alloc((void **)&h->ticket, sizeof(unsigned long long), s);
     if (rc == PDB_OK) {
         cudaMemsetAsync(h->bar, 0, sizeof(GridBarrier), s);
         cudaMemsetAsync(h->ticket, 0, sizeof(unsigned long long), s);
     }
     if (mode == PDB_SCHED_READY) {
-        rc = rc ? rc : alloc((void **)&h->ctr, sizeof(unsigned) * F, s);
-        rc = rc ? rc : alloc((void **)&h->gate, sizeof(uint32_t) * c->nnz, s);
-        if (rc == PDB_OK) {
-            cudaMemsetAsync(h->ctr, 0, sizeof(unsigned) * F, s);
-            if (c->nnz > 0)
-                k_make_gate<<<grid_1d(c->nnz), 256, 0, s>>>(c->rank, c->next, c->nnz, h->gate, c->status); note_launch();
-        }
+        // one (weight, version) record per feature; filled from w by pdb_sgd_epoch
+        rc = rc ? rc : alloc((void **)&h->rec, sizeof(unsigned long long) * F, s);
     } else {
+        rc = rc ? rc : materialize_chains(cm, s);
+        if (rc == PDB_OK && !cm->npred) {
+            rc = alloc((void **)&cm->npred, sizeof(int32_t) * N, s);
+            if (rc == PDB_OK && N > 0) {
+                k_npred<<<grid_1d(N * 32), 256, 0, s>>>(c->row_ptr, N, c->prev, cm->npred, c->status);
+                note_launch();
+            }
+        }
         rc = rc ? rc : alloc((void **)&h->level, sizeof(int32_t) * N, s);
         rc = rc ? rc : alloc((void **)&h->order, sizeof(int32_t) * N, s);
         rc = rc ? rc : alloc((void **)&h->indeg, sizeof(int32_t) * N, s);
@@ -407,12 +456,14 @@ int pdb_schedule_build(const pdb_conflicts *c, pdb_sched_mode mode, pdb_schedule
                 int grid = persistent_grid(kern, nullptr);
                 int32_t n32 = (int32_t)N;
                 uint64_t tmo = timeout_ns(nullptr);
-                void *args[] = {&n32, (void *)&c->row_ptr, (void *)&c->next, (void *)&c->row_of,
-                                (void *)&c->npred, &h->indeg, &h->queue, &h->level, &h->ctl,
-                                (void *)&c->status, &tmo};
-                if (cudaLaunchCooperativeKernel(kern, grid, THREADS, args, 0, s) != cudaSuccess) rc = PDB_ECUDA; note_launch();
+                void *args[] = {&n32,       (void *)&c->row_ptr, (void *)&c->next, (void *)&c->row_of,
+                                (void *)&c->npred, &h->indeg, &h->queue, &h->level,
+                                &h->ctl,    (void *)&c->status, &tmo};
+                if (cudaLaunchCooperativeKernel(kern, grid, THREADS, args, 0, s) != cudaSuccess) rc = PDB_ECUDA;
+                note_launch();
                 if (rc == PDB_OK) {
-                    k_iota_u32_level<<<grid_1d(N), 256, 0, s>>>(h->level, key, n32); note_launch();
+                    k_level_keys<<<grid_1d(N), 256, 0, s>>>(h->level, key, n32, c->status);
+                    note_launch();
                     rc = radix_sort(key, nullptr, skey, h->order, tkey, tval, N, bits_for(N), c->status, s);
                 }
                 if (rc == PDB_OK) rc = segment_bounds(skey, N, N, &h->ctl->n_levels, h->level_ptr, c->status, s);
@@ -455,12 +506,12 @@ int pdb_schedule_levels(const pdb_schedule *h, const int32_t **level, const int3
     return PDB_OK;
 }
 
-int pdb_schedule_ready(const pdb_schedule *h, const uint32_t **ctr, const uint32_t **gate)
+int pdb_schedule_ready(const pdb_schedule *h, const uint32_t **gate, const uint64_t **records)
 {
     if (!h) return PDB_EINVAL;
     if (h->mode != PDB_SCHED_READY) return PDB_ESTATE;
-    if (ctr) *ctr = h->ctr;
-    if (gate) *gate = h->gate;
+    if (gate) *gate = h->c->gate;
+    if (records) *records = (const uint64_t *)h->rec;
     return PDB_OK;
 }
 
@@ -474,12 +525,13 @@ int pdb_get_stats(const pdb_conflicts *c, const pdb_schedule *h, pdb_stats *out)
     out->nnz = c->nnz;
     out->n_levels = -1;
     out->max_level_width = -1;
-    int mc = 0;
-    cudaMemcpy(&mc, c->max_chain, sizeof(int), cudaMemcpyDeviceToHost);
-    out->max_chain = mc;
+    int info[INFO_WORDS] = {};
+    if (cudaMemcpy(info, c->info, sizeof info, cudaMemcpyDeviceToHost) != cudaSuccess) return PDB_ECUDA;
+    out->max_chain = info[INFO_MAX_CHAIN];
     float ms = 0;
     if (c->timed_build && cudaEventElapsedTime(&ms, c->ev0, c->ev1) == cudaSuccess) out->ms_build = ms;
     if (c->timed_sgd && cudaEventElapsedTime(&ms, c->ev_sgd0, c->ev_sgd1) == cudaSuccess) out->ms_sgd = ms;
+    if (c->timed_sgd && cudaEventElapsedTime(&ms, c->ev_k0, c->ev_k1) == cudaSuccess) out->ms_sgd_kernels = ms;
     if (c->timed_bsp && cudaEventElapsedTime(&ms, c->ev_bsp0, c->ev_bsp1) == cudaSuccess) out->ms_bsp = ms;
     if (h) {
         if (h->timed && cudaEventElapsedTime(&ms, h->ev0, h->ev1) == cudaSuccess) out->ms_schedule = ms;

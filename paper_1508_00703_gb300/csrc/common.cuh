@@ -27,6 +27,7 @@ uint64_t timeout_ns(const pdb_opts *opts);
 int alloc(void **p, size_t bytes, cudaStream_t s);   // stream-ordered, 256-byte aligned
 void release(void *p, cudaStream_t s);
 int bits_for(int64_t max_key);                        // bits to hold values 0..max_key (>= 1)
+int grid_1d(int64_t n);                               // blocks of 256 threads for a grid-stride loop
 void note_launch();                                   // count one kernel launch (pdb_launch_count)
 
 // Stable LSD radix sort of (key, value) pairs, 8-bit digits.  vals_in ==
@@ -182,13 +183,20 @@ __device__ __forceinline__ float warp_combine(float a)
 struct pdb_conflicts {
     int device;
     int64_t n_rows, n_cols, nnz;
-    int64_t *row_ptr;     // library copy of the caller's row_ptr
-    int32_t *csc_pos, *prev, *next, *rank, *row_of, *npred;
-    int64_t *feat_ptr;
-    int *status;          // device word: first error recorded by a kernel
-    int *max_chain;       // device
-    cudaEvent_t ev0, ev1, ev_sgd0, ev_sgd1, ev_bsp0, ev_bsp1;
+    const int64_t *row_ptr;  // the caller's D (immutable, must outlive the handle)
+    const int32_t *col;
+    const float *val;
+    int32_t *csc_pos;        // positions grouped by feature, data order inside a feature
+    int64_t *feat_ptr;       // [F+1]
+    uint32_t *gate;          // per position: occurrence rank, bit 31 = last occurrence of the feature
+    int32_t *row_of;         // example of each position
+    int32_t *prev, *next, *rank;  // materialized from the above on first request
+    int32_t *npred;          // per example: occurrences with an earlier occurrence (LEVELS)
+    int *info;               // device: [0] status, [1] max chain, [2] longest row, [3] any unsorted row
+    int *h_info;             // pinned host copy of info, filled at the end of the build
+    cudaEvent_t ev0, ev1, ev_sgd0, ev_sgd1, ev_bsp0, ev_bsp1, ev_k0, ev_k1;
     bool timed_build, timed_sgd, timed_bsp;
+    int *status;             // = info (first error recorded by a kernel)
 };
 
 struct LevelCtl {
@@ -205,8 +213,7 @@ struct pdb_schedule {
     int32_t *level, *order, *indeg, *queue;
     int64_t *level_ptr;
     LevelCtl *ctl;            // device
-    unsigned *ctr;            // READY: per-feature ready counters
-    uint32_t *gate;           // READY: per position, rank | last-occurrence bit
+    unsigned long long *rec;  // READY: per feature (weight bits | version << 32)
     pdb::GridBarrier *bar;    // barrier for the level-synchronous engine
     unsigned long long *ticket;
     cudaEvent_t ev0, ev1;

@@ -17,22 +17,15 @@ using namespace pdb;
 
 namespace {
 
-constexpr int R = 8;   // elements per lane held in registers (rows up to 256 ids)
 
-__device__ __forceinline__ unsigned ld_relaxed(const unsigned *p)
-{
-    unsigned v;
-    asm volatile("ld.relaxed.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
-    return v;
-}
-__device__ __forceinline__ void st_relaxed(unsigned *p, unsigned v)
-{
-    asm volatile("st.relaxed.gpu.global.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
-}
 
 // ---------------------------------------------------------------- one example, no waits
 // Used by the level-synchronous engine: the level schedule already keeps
-// every example of a level disjoint from the others (Theorem 3).
+// every example of a level disjoint from the others (Theorem 3).  Element i
+// of the row lives in lane i mod 32, register i / 32; each lane accumulates
+// its elements in increasing i with fused multiply-adds, then the lanes
+// combine pairwise (the fixed order both sides of the parity check use).
+template <int R>
 __device__ __forceinline__ void sgd_example(int t, const int64_t *__restrict__ row_ptr, const int32_t *__restrict__ col,
                                             const float *__restrict__ val, const float *__restrict__ y, float *w,
                                             int loss, float eta)
@@ -78,6 +71,7 @@ __device__ __forceinline__ void sgd_example(int t, const int64_t *__restrict__ r
 // Persistent cooperative kernel: level l's examples are spread over all
 // warps, a grid barrier closes the level (the read barrier of the next BSP
 // step and the write barrier of this one, Algorithm 2a per level).
+template <int R>
 __global__ __launch_bounds__(THREADS) void k_sgd_levels(int32_t n_rows, const int64_t *__restrict__ row_ptr,
                                                         const int32_t *__restrict__ col, const float *__restrict__ val,
                                                         const float *__restrict__ y, const int32_t *__restrict__ order,
@@ -98,38 +92,70 @@ __global__ __launch_bounds__(THREADS) void k_sgd_levels(int32_t n_rows, const in
                     set_status(status, PDB_EFAULT);
                     continue;
                 }
-                sgd_example(t, row_ptr, col, val, y, w, loss, eta);
+                sgd_example<R>(t, row_ptr, col, val, y, w, loss, eta);
             }
             if (!grid_sync(bar, status, timeout)) return;
         }
 }
 
 // ---------------------------------------------------------------- ready-counter dataflow engine
-// The read protocol of Section 5 per feature: ctr[j] counts the writes of
-// feature j so far in this epoch.  The occurrence of j with rank r may read
-// w_j once ctr[j] == r (Read Constraint: the previous writer is done), and
-// publishes r + 1 after its write (Write Constraint: its own read, the only
-// read of that version, precedes the write).  The last occurrence of j in
-// the epoch (gate bit 31) resets ctr[j] to 0 for the next epoch.
-// Examples are taken in data order from a ticket counter, so the oldest
-// unfinished example never waits on a younger one and the kernel cannot
-// deadlock regardless of how many warps are resident.
-// Acquire/release: relaxed polls of all the lane's counters, then one
-// fence; w stores, one fence, then relaxed counter stores.
-__device__ __forceinline__ bool wait_ready(const unsigned *ctr, const int *j, const unsigned *want, int lane, int k,
-                                           int *status, uint64_t timeout)
+// The read protocol of Section 5 per feature.  Feature j's record holds its
+// weight and its iteration number (version) in one aligned 64-bit word:
+// rec[j] = bits(w_j) | version_j << 32.  The occurrence of j with rank r
+// (its gate) may read w_j once version_j == r -- one relaxed 64-bit load
+// both checks the version and returns the weight written with it (Read
+// Constraint: the previous writer is done) -- and publishes the new weight
+// together with version r + 1 in one 64-bit store (Write Constraint: its own
+// read, the only read of that version, came first).  The last occurrence of
+// j in the epoch (gate bit 31) writes version 0 for the next epoch.  Both
+// halves travel in one single-copy-atomic access, so no fence is needed.
+// Examples are taken in data order from a ticket counter, `chunk`
+// consecutive ones at a time and run in order by the warp that took them,
+// so the oldest unfinished example never waits on a younger one and the
+// kernel cannot deadlock whatever the number of resident warps.
+__device__ __forceinline__ unsigned long long ld_rec(const unsigned long long *p)
 {
-    bool ready;
-    uint64_t t0 = 0;
-    unsigned spins = 0;
-    for (;;) {
-        ready = true;
+    unsigned long long v;
+    asm volatile("ld.relaxed.gpu.global.b64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
+    return v;
+}
+__device__ __forceinline__ void st_rec(unsigned long long *p, float w, unsigned version)
+{
+    unsigned long long v = (unsigned long long)__float_as_uint(w) | ((unsigned long long)version << 32);
+    asm volatile("st.relaxed.gpu.global.b64 [%0], %1;" ::"l"(p), "l"(v) : "memory");
+}
+
+// Gathers w for the lane's elements, waiting until each record carries the
+// wanted version.  False when the wait gave up (timeout or a failure
+// elsewhere recorded in status).
+template <int R>
+__device__ __forceinline__ bool gather_ready(const unsigned long long *rec, const int *j, const unsigned *want,
+                                             float *wv, int lane, int k, int *status, uint64_t timeout)
+{
+    unsigned pending = 0;
+#pragma unroll
+    for (int r = 0; r < R; ++r)
+        if (r * 32 + lane < k) {
+            unsigned long long v = ld_rec(rec + j[r]);
+            wv[r] = __uint_as_float((unsigned)v);
+            if ((unsigned)(v >> 32) != want[r]) pending |= 1u << r;
+        }
+    if (pending == 0) return true;
+    const uint64_t t0 = globaltimer();
+    unsigned spins = 0, nap = 32;
+    while (pending) {
+        __nanosleep(nap);                 // back off: a waiting lane should not flood L2 with polls
+        nap = nap < 512 ? 2 * nap : 512;
 #pragma unroll
         for (int r = 0; r < R; ++r)
-            if (r * 32 + lane < k) ready &= ld_relaxed(ctr + j[r]) == want[r];
-        if (ready) break;
-        if (spins == 0) t0 = globaltimer();
-        if ((++spins & 127u) == 0) {
+            if (pending & (1u << r)) {
+                unsigned long long v = ld_rec(rec + j[r]);
+                if ((unsigned)(v >> 32) == want[r]) {
+                    wv[r] = __uint_as_float((unsigned)v);
+                    pending &= ~(1u << r);
+                }
+            }
+        if (pending && (++spins & 15u) == 0) {
             if (read_status(status)) return false;
             if (globaltimer() - t0 > timeout) {
                 set_status(status, PDB_ETIMEOUT);
@@ -137,85 +163,108 @@ __device__ __forceinline__ bool wait_ready(const unsigned *ctr, const int *j, co
             }
         }
     }
-    __threadfence();
     return true;
 }
 
+// one example under the ready protocol; false when a wait gave up
+template <int R>
+__device__ __forceinline__ bool ready_example(int t, const int64_t *__restrict__ row_ptr,
+                                              const int32_t *__restrict__ col, const float *__restrict__ val,
+                                              const float *__restrict__ y, const uint32_t *__restrict__ gate,
+                                              unsigned long long *rec, int loss, float eta, int *status,
+                                              uint64_t timeout)
+{
+    const int lane = threadIdx.x & 31;
+    const int64_t b = row_ptr[t];
+    const int k = (int)(row_ptr[t + 1] - b);
+    const float yt = y[t];
+    if (k <= 32 * R) {
+        int j[R];
+        float x[R], wv[R];
+        unsigned want[R], next[R];
+#pragma unroll
+        for (int r = 0; r < R; ++r) {
+            int i = r * 32 + lane;
+            j[r] = i < k ? col[b + i] : 0;
+            x[r] = i < k ? (val ? val[b + i] : 1.0f) : 0.0f;
+            uint32_t g = i < k ? gate[b + i] : 0u;
+            want[r] = g & 0x7fffffffu;
+            next[r] = (g >> 31) ? 0u : want[r] + 1u;
+            wv[r] = 0.0f;
+        }
+        bool ok = gather_ready<R>(rec, j, want, wv, lane, k, status, timeout);
+        if (!__all_sync(FULL, ok)) return false;
+        float acc = 0.0f;
+#pragma unroll
+        for (int r = 0; r < R; ++r)
+            if (r * 32 + lane < k) acc = __fmaf_rn(wv[r], x[r], acc);
+        const float m = warp_combine(acc);
+        const float c = __fmul_rn(eta, dev_grad(loss, m, yt));
+#pragma unroll
+        for (int r = 0; r < R; ++r)
+            if (r * 32 + lane < k) st_rec(rec + j[r], __fsub_rn(wv[r], __fmul_rn(c, x[r])), next[r]);
+        return true;
+    }
+    // long example: wait and gather element by element, then a second pass
+    // (this example owns its features until it writes them, so re-reading
+    // the records returns the same weights)
+    float acc = 0.0f;
+    bool ok = true;
+    for (int i = lane; i < k && ok; i += 32) {
+        int j1[1] = {col[b + i]};
+        unsigned w1[1] = {gate[b + i] & 0x7fffffffu};
+        float v1[1];
+        ok = gather_ready<1>(rec, j1, w1, v1, 0, 1, status, timeout);
+        if (ok) acc = __fmaf_rn(v1[0], val ? val[b + i] : 1.0f, acc);
+    }
+    if (!__all_sync(FULL, ok)) return false;
+    const float m = warp_combine(acc);
+    const float c = __fmul_rn(eta, dev_grad(loss, m, yt));
+    for (int i = lane; i < k; i += 32) {
+        const int jj = col[b + i];
+        const float xx = val ? val[b + i] : 1.0f;
+        const uint32_t g = gate[b + i];
+        const float wo = __uint_as_float((unsigned)ld_rec(rec + jj));
+        st_rec(rec + jj, __fsub_rn(wo, __fmul_rn(c, xx)), (g >> 31) ? 0u : (g & 0x7fffffffu) + 1u);
+    }
+    return true;
+}
+
+template <int R>
 __global__ __launch_bounds__(THREADS) void k_sgd_ready(int32_t n_rows, const int64_t *__restrict__ row_ptr,
                                                        const int32_t *__restrict__ col, const float *__restrict__ val,
                                                        const float *__restrict__ y, const uint32_t *__restrict__ gate,
-                                                       unsigned *ctr, float *w, int loss, float eta,
-                                                       unsigned long long *ticket, int *status, uint64_t timeout)
+                                                       unsigned long long *rec, int loss, float eta,
+                                                       unsigned long long *ticket, int chunk, int *status,
+                                                       uint64_t timeout)
 {
     if (read_status(status)) return;
     const int lane = threadIdx.x & 31;
     for (;;) {
         unsigned long long tk = 0;
-        if (lane == 0) tk = atomicAdd(ticket, 1ull);
+        if (lane == 0) tk = atomicAdd(ticket, (unsigned long long)chunk);
         tk = __shfl_sync(FULL, tk, 0);
         if (tk >= (unsigned long long)n_rows) return;
-        const int t = (int)tk;
-        const int64_t b = row_ptr[t];
-        const int k = (int)(row_ptr[t + 1] - b);
-        const float yt = y[t];
-        if (k <= 32 * R) {
-            int j[R];
-            float x[R], wv[R];
-            unsigned want[R], next[R];
-#pragma unroll
-            for (int r = 0; r < R; ++r) {
-                int i = r * 32 + lane;
-                j[r] = i < k ? col[b + i] : 0;
-                x[r] = i < k ? (val ? val[b + i] : 1.0f) : 0.0f;
-                uint32_t g = i < k ? gate[b + i] : 0u;
-                want[r] = g & 0x7fffffffu;
-                next[r] = (g >> 31) ? 0u : want[r] + 1u;
-            }
-            bool ok = wait_ready(ctr, j, want, lane, k, status, timeout);
-            if (!__all_sync(FULL, ok)) return;
-            float acc = 0.0f;
-#pragma unroll
-            for (int r = 0; r < R; ++r)
-                if (r * 32 + lane < k) wv[r] = __ldcg(w + j[r]);
-#pragma unroll
-            for (int r = 0; r < R; ++r)
-                if (r * 32 + lane < k) acc = __fmaf_rn(wv[r], x[r], acc);
-            const float m = warp_combine(acc);
-            const float c = __fmul_rn(eta, dev_grad(loss, m, yt));
-#pragma unroll
-            for (int r = 0; r < R; ++r)
-                if (r * 32 + lane < k) __stcg(w + j[r], __fsub_rn(wv[r], __fmul_rn(c, x[r])));
-            __threadfence();
-#pragma unroll
-            for (int r = 0; r < R; ++r)
-                if (r * 32 + lane < k) st_relaxed(ctr + j[r], next[r]);
-        } else {
-            // long example: wait and gather element by element, then a second pass
-            float acc = 0.0f;
-            bool ok = true;
-            for (int i = lane; i < k && ok; i += 32) {
-                int jj = col[b + i];
-                unsigned want = gate[b + i] & 0x7fffffffu;
-                int j1[R] = {jj};
-                unsigned w1[R] = {want};
-                ok = wait_ready(ctr, j1, w1, 0, 1, status, timeout);
-                if (ok) acc = __fmaf_rn(__ldcg(w + jj), val ? val[b + i] : 1.0f, acc);
-            }
-            if (!__all_sync(FULL, ok)) return;
-            const float m = warp_combine(acc);
-            const float c = __fmul_rn(eta, dev_grad(loss, m, yt));
-            for (int i = lane; i < k; i += 32) {
-                int jj = col[b + i];
-                float xx = val ? val[b + i] : 1.0f;
-                __stcg(w + jj, __fsub_rn(__ldcg(w + jj), __fmul_rn(c, xx)));
-            }
-            __threadfence();
-            for (int i = lane; i < k; i += 32) {
-                uint32_t g = gate[b + i];
-                st_relaxed(ctr + col[b + i], (g >> 31) ? 0u : (g & 0x7fffffffu) + 1u);
-            }
-        }
+        const int t1 = (int)min64((int64_t)n_rows, (int64_t)tk + chunk);
+        for (int t = (int)tk; t < t1; ++t)
+            if (!ready_example<R>(t, row_ptr, col, val, y, gate, rec, loss, eta, status, timeout)) return;
     }
+}
+
+// rec[j] = (w_j, version 0) before the first epoch; w_j back after the last
+__global__ void k_pack(const float *__restrict__ w, int64_t n, unsigned long long *__restrict__ rec, const int *status)
+{
+    if (read_status(status)) return;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x)
+        rec[i] = (unsigned long long)__float_as_uint(w[i]);
+}
+
+__global__ void k_unpack(const unsigned long long *__restrict__ rec, int64_t n, float *__restrict__ w,
+                         const int *status)
+{
+    if (read_status(status)) return;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x)
+        w[i] = __uint_as_float((unsigned)rec[i]);
 }
 
 // ---------------------------------------------------------------- BSP
@@ -303,10 +352,18 @@ __global__ void k_eval_expf(const float *__restrict__ x, float *__restrict__ out
         out[i] = dev_expf(x[i]);
 }
 
-int grid_1d(int64_t n)
+// Registers per lane for the example's elements: the smallest of 2, 4, 8
+// that holds the longest row in registers (longer rows take the two-pass
+// path).  The longest row is recorded by the conflict build; this waits for
+// that build to finish if it has not.
+int register_width(const pdb_conflicts *c)
 {
-    int64_t b = (n + 255) / 256;
-    return (int)std::max<int64_t>(1, std::min<int64_t>(b, 152 * 32));
+    if (cudaEventSynchronize(c->ev1) != cudaSuccess) {
+        cudaGetLastError();
+        return 8;
+    }
+    const int longest = c->h_info[2];
+    return longest <= 64 ? 2 : longest <= 128 ? 4 : 8;
 }
 
 int check_run(const pdb_csr *X, const float *y, const pdb_conflicts *c, const float *w, int loss, int epochs)
@@ -331,29 +388,46 @@ int pdb_sgd_epoch(const pdb_csr *X, const float *y, const pdb_conflicts *c, cons
     if (!h || h->c != c) return PDB_EINVAL;
     cudaStream_t s = (cudaStream_t)stream;
     pdb_conflicts *cm = const_cast<pdb_conflicts *>(c);
+    const int width = register_width(cm);
     cudaEventRecord(cm->ev_sgd0, s);
+    cudaEventRecord(cm->ev_k0, s);
+    cudaEventRecord(cm->ev_k1, s);
     const uint64_t tmo = timeout_ns(opts);
     int32_t n32 = (int32_t)X->n_rows;
     int lossi = (int)loss;
     if (X->n_rows > 0 && n_epochs > 0) {
         if (h->mode == PDB_SCHED_LEVELS) {
-            const void *kern = (const void *)k_sgd_levels;
+            const void *kern = width == 2 ? (const void *)k_sgd_levels<2>
+                               : width == 4 ? (const void *)k_sgd_levels<4> : (const void *)k_sgd_levels<8>;
             int grid = persistent_grid(kern, opts);
             const int64_t *rp = X->row_ptr;
             const int32_t *cl = X->col;
             const float *vl = X->val;
-            void *args[] = {(void *)&n32, (void *)&rp,        (void *)&cl, (void *)&vl,       (void *)&y,
-                            (void *)&h->order,  (void *)&h->level_ptr, (void *)&h->ctl, (void *)&w,
-                            (void *)&lossi,     (void *)&eta, (void *)&n_epochs, (void *)&h->bar,
+            void *args[] = {(void *)&n32,      (void *)&rp,  (void *)&cl,       (void *)&vl,     (void *)&y,
+                            (void *)&h->order, (void *)&h->level_ptr, (void *)&h->ctl, (void *)&w,
+                            (void *)&lossi,    (void *)&eta, (void *)&n_epochs, (void *)&h->bar,
                             (void *)&cm->status, (void *)&tmo};
-            if (cudaLaunchCooperativeKernel(kern, grid, THREADS, args, 0, s) != cudaSuccess) rc = PDB_ECUDA; note_launch();
+            cudaEventRecord(cm->ev_k0, s);
+            if (cudaLaunchCooperativeKernel(kern, grid, THREADS, args, 0, s) != cudaSuccess) rc = PDB_ECUDA;
+            note_launch();
+            cudaEventRecord(cm->ev_k1, s);
         } else {
-            int grid = persistent_grid((const void *)k_sgd_ready, opts);
+            auto kern = width == 2 ? k_sgd_ready<2> : width == 4 ? k_sgd_ready<4> : k_sgd_ready<8>;
+            int grid = persistent_grid((const void *)kern, opts);
+            const int64_t F = X->n_cols;
+            const int chunk = (opts && opts->ticket_chunk > 0) ? opts->ticket_chunk : 2;
+            k_pack<<<grid_1d(F), 256, 0, s>>>(w, F, h->rec, cm->status);
+            note_launch();
+            cudaEventRecord(cm->ev_k0, s);
             for (int ep = 0; ep < n_epochs; ++ep) {
                 cudaMemsetAsync(h->ticket, 0, sizeof(unsigned long long), s);
-                k_sgd_ready<<<grid, THREADS, 0, s>>>(n32, X->row_ptr, X->col, X->val, y, h->gate, h->ctr, w, lossi,
-                                                     eta, h->ticket, cm->status, tmo); note_launch();
+                kern<<<grid, THREADS, 0, s>>>(n32, X->row_ptr, X->col, X->val, y, c->gate, h->rec, lossi, eta,
+                                              h->ticket, chunk, cm->status, tmo);
+                note_launch();
             }
+            cudaEventRecord(cm->ev_k1, s);
+            k_unpack<<<grid_1d(F), 256, 0, s>>>(h->rec, F, w, cm->status);
+            note_launch();
         }
     }
     cudaEventRecord(cm->ev_sgd1, s);

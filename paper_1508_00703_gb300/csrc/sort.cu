@@ -87,6 +87,12 @@ void release(void *p, cudaStream_t s)
 static std::atomic<long long> g_launches{0};
 void note_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
 
+int grid_1d(int64_t n)
+{
+    int64_t b = (n + 255) / 256;
+    return (int)std::max<int64_t>(1, std::min<int64_t>(b, 152 * 32));
+}
+
 int bits_for(int64_t max_key)
 {
     int b = 1;

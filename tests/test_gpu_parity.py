@@ -160,18 +160,18 @@ def test_device_validation(row_ptr, col, code):
 
 
 def test_wait_timeout_is_reported_not_hung():
-    # A ready counter that nothing will ever release: every bounded wait
-    # gives up after the short limit, the kernel returns, the status says so,
-    # and the context stays usable.
+    # One position waits for a version its feature never reaches: every
+    # bounded wait gives up after the short limit, the kernel returns, the
+    # status says so, and the context stays usable.
     name = "tiny"
     p, X, y = _gpu(name)
     c = pdb.pdb_build_conflicts(X)
     s = pdb.pdb_schedule_build(c, pdb.PDB_SCHED_READY)
     pdb.check_status(c)
-    ctr_ptr = pdb.pdb_schedule_ready(s)["ctr"]
-    j = int(p.col[p.row_ptr[5]])                          # a feature that example 5 reads
+    gate_ptr = pdb.pdb_schedule_ready(s)["gate"]
+    pos = int(p.row_ptr[5])                               # first element of example 5
     poison = torch.tensor([12345], dtype=torch.int32, device="cuda")
-    pdb.pdb_memcpy(ctr_ptr + 4 * j, poison.data_ptr(), 4)
+    pdb.pdb_memcpy(gate_ptr + 4 * pos, poison.data_ptr(), 4)
     w = torch.zeros(p.n_cols, dtype=torch.float32, device="cuda")
     pdb.pdb_sgd_epoch(X, y, c, s, w, p.loss, p.eta, 1, opts=dict(wait_timeout_s=0.2))
     assert pdb.pdb_status(c) == pdb.PDB_ETIMEOUT
