@@ -56,6 +56,7 @@ extern "C" {
 #define PDB_ETIMEOUT (-6) /* a bounded device-side wait expired (the kernel stopped, the GPU stays usable) */
 #define PDB_EFAULT (-7)   /* an internal invariant failed on the device */
 #define PDB_ESTATE (-8)   /* wrong handle for this call (e.g. a READY schedule where levels are needed) */
+#define PDB_ETOOBIG (-9)  /* problem larger than the fixed scratch of pdb_sgd_epoch_ready_noalloc */
 
 /* ---------------------------------------------------------------- types */
 
@@ -204,6 +205,30 @@ void pdb_schedule_free(pdb_schedule *s);
 
 /* Text of an error code. */
 const char *pdb_strerror(int code);
+
+/* Allocation-free variant of pdb_sgd_epoch with a READY schedule (the paper
+ * has no counterpart; it exists for callers that must not allocate device
+ * memory while they train: work recorded into a CUDA graph capture, where
+ * cudaMalloc cannot be captured, or a process that has given all device
+ * memory to its own pool).  It allocates nothing: its scratch (one 64-bit
+ * (weight, version) record per feature, a ticket counter and a status word)
+ * is one fixed array inside the library of 2^20 records, about 8 MiB, that
+ * every GPU loading the library holds until the process exits.
+ *   X, y, w     as for pdb_sgd_epoch; X->n_cols must be <= 2^20, else
+ *               PDB_ETOOBIG and nothing runs.
+ *   gate[nnz]   per position, the occurrence rank of its feature with bit 31
+ *               set on the feature's last occurrence -- the array that
+ *               pdb_schedule_ready returns for a READY schedule of X (device,
+ *               caller-owned here).
+ * Same arithmetic and result as pdb_sgd_epoch.  The first call on each
+ * device looks up the array's device address (cudaGetSymbolAddress); make
+ * that first call before any stream capture.  All calls on a device share
+ * the array (each clears what must start at zero): calls whose GPU work
+ * overlaps race, so order them on one stream.  SYNCHRONIZES `stream` and
+ * returns PDB_OK, a kernel-recorded error (PDB_ETIMEOUT, PDB_EFAULT), or a
+ * host error. */
+int pdb_sgd_epoch_ready_noalloc(const pdb_csr *X, const float *y, const uint32_t *gate, float *w, pdb_loss loss,
+                                float eta, int n_epochs, void *stream);
 
 /* ---------------------------------------------------------------- utilities */
 

@@ -26,6 +26,8 @@ NVCC_FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-fmad=false", "-Xcompiler", "-f
 
 PDB_OK, PDB_EINVAL, PDB_ERANGE, PDB_EDUP, PDB_ENOMEM, PDB_ECUDA, PDB_ETIMEOUT, PDB_EFAULT, PDB_ESTATE = \
     0, -1, -2, -3, -4, -5, -6, -7, -8
+PDB_ETOOBIG = -9
+NOALLOC_MAX_COLS = 1 << 20
 PDB_LOSS_LOGISTIC, PDB_LOSS_SQUARED, PDB_LOSS_HINGE = 0, 1, 2
 PDB_SCHED_LEVELS, PDB_SCHED_READY = 0, 1
 
@@ -104,7 +106,8 @@ class pdb_stats(ctypes.Structure):
 EXPORTS = ["pdb_build_conflicts", "pdb_conflicts_arrays", "pdb_schedule_build", "pdb_schedule_levels",
            "pdb_schedule_ready",
            "pdb_sgd_epoch", "pdb_bsp_epoch", "pdb_status", "pdb_get_stats", "pdb_conflicts_free",
-           "pdb_schedule_free", "pdb_strerror", "pdb_memcpy", "pdb_eval_expf", "pdb_launch_count"]
+           "pdb_schedule_free", "pdb_strerror", "pdb_memcpy", "pdb_eval_expf", "pdb_launch_count",
+           "pdb_sgd_epoch_ready_noalloc"]
 
 
 def load(path: str | None = None):
@@ -133,6 +136,7 @@ def load(path: str | None = None):
         lib.pdb_strerror.restype = ctypes.c_char_p
         lib.pdb_memcpy.argtypes = [P, P, ctypes.c_size_t, P]
         lib.pdb_eval_expf.argtypes = [P, P, I64, P]
+        lib.pdb_sgd_epoch_ready_noalloc.argtypes = [ctypes.POINTER(pdb_csr), P, P, P, I32, ctypes.c_float, I32, P]
         lib.pdb_launch_count.argtypes = []
         lib.pdb_launch_count.restype = I64
         _lib = lib
@@ -259,6 +263,17 @@ def pdb_bsp_epoch(X: Csr, y, c: Conflicts, w, loss: int, eta: float, batch: int,
                   stream=None):
     _check(load().pdb_bsp_epoch(ctypes.byref(X.struct), _ptr(y), c.handle, _ptr(w), int(loss), float(eta),
                                 int(batch), int(n_epochs), _opts(opts), _stream(stream)), "pdb_bsp_epoch")
+
+
+def pdb_sgd_epoch_ready_noalloc(X: Csr, y, gate_ptr: int, w, loss: int, eta: float, n_epochs: int,
+                                stream=None) -> int:
+    """READY-schedule SGD epochs that allocate no device memory (scratch is a
+    fixed array inside the library, up to NOALLOC_MAX_COLS features).  For
+    callers that cannot allocate while training, e.g. inside a CUDA graph
+    capture or under a memory pool that owns the whole device.  Synchronizes
+    and returns the status code (PDB_OK on success)."""
+    return int(load().pdb_sgd_epoch_ready_noalloc(ctypes.byref(X.struct), _ptr(y), ctypes.c_void_p(gate_ptr), _ptr(w),
+                                                  int(loss), float(eta), int(n_epochs), _stream(stream)))
 
 
 def pdb_status(c: Conflicts, stream=None) -> int:

@@ -278,6 +278,7 @@ const char *pdb_strerror(int code)
     case PDB_ETIMEOUT: return "device-side wait expired";
     case PDB_EFAULT: return "internal invariant failed on the device";
     case PDB_ESTATE: return "handle in the wrong mode for this call";
+    case PDB_ETOOBIG: return "more features than the allocation-free variant's fixed scratch holds (2^20)";
     default: return "unknown error";
     }
 }

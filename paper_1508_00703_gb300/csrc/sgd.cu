@@ -10,6 +10,7 @@
 #include <cuda_runtime.h>
 
 #include <algorithm>
+#include <mutex>
 
 #include "common.cuh"
 
@@ -512,3 +513,92 @@ int pdb_eval_expf(const float *x, float *out, int64_t n, void *stream)
 }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------- allocation-free READY epoch
+// Some callers cannot allocate device memory while they train: code that
+// runs between the two halves of a CUDA graph capture (cudaMalloc is not a
+// capturable operation), a server that has handed all device memory to its
+// own pool and must not grow or fragment it, or an embedding runtime that
+// forbids the library from owning memory.  For them the READY epoch below
+// keeps its per-feature (weight, version) records, its ticket counter and
+// its status word in one fixed array compiled into the library instead of
+// in a schedule handle.  Every GPU that loads libpdb holds this array
+// (NOALLOC_MAX_COLS * 8 bytes + 256 bytes, about 8 MiB) until the process
+// exits.  All calls on a device share it: two calls whose work overlaps on
+// the GPU corrupt each other, so order them on one stream.
+constexpr int64_t NOALLOC_MAX_COLS = 1 << 20;
+constexpr int64_t NOALLOC_WORDS = NOALLOC_MAX_COLS + 32;   // records, then ticket and status
+static __device__ __align__(256) unsigned long long g_noalloc_scratch[NOALLOC_WORDS];
+
+namespace {
+
+std::mutex g_noalloc_lock;
+unsigned long long *g_noalloc_ptr[64];
+
+// Device address of the scratch array for the current device, looked up
+// once per device (host code only sees a stand-in symbol, not the address).
+unsigned long long *noalloc_scratch()
+{
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
+    std::lock_guard<std::mutex> guard(g_noalloc_lock);
+    if (!g_noalloc_ptr[dev]) {
+        void *p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess) {
+            cudaGetLastError();
+            return nullptr;
+        }
+        g_noalloc_ptr[dev] = (unsigned long long *)p;
+    }
+    return g_noalloc_ptr[dev];
+}
+
+}  // namespace
+
+extern "C" int pdb_sgd_epoch_ready_noalloc(const pdb_csr *X, const float *y, const uint32_t *gate, float *w,
+                                           pdb_loss loss, float eta, int n_epochs, void *stream)
+{
+    if (!X || X->n_rows < 0 || X->n_cols < 0 || X->nnz < 0 || n_epochs < 0) return PDB_EINVAL;
+    if (X->n_cols > NOALLOC_MAX_COLS) return PDB_ETOOBIG;
+    if (X->n_rows >= (1ll << 31) - 1 || X->nnz >= (1ll << 31) - 1) return PDB_EINVAL;
+    if (loss != PDB_LOSS_LOGISTIC && loss != PDB_LOSS_SQUARED && loss != PDB_LOSS_HINGE) return PDB_EINVAL;
+    if (!X->row_ptr || (X->nnz > 0 && (!X->col || !gate)) || (X->n_rows > 0 && !y) || (X->n_cols > 0 && !w))
+        return PDB_EINVAL;
+    unsigned long long *scratch = noalloc_scratch();
+    if (!scratch) return PDB_ECUDA;
+    unsigned long long *rec = scratch;
+    unsigned long long *ticket = scratch + NOALLOC_MAX_COLS;
+    int *status = (int *)(scratch + NOALLOC_MAX_COLS + 1);
+    cudaStream_t s = (cudaStream_t)stream;
+    // the previous call left its status and ticket behind: start from zero
+    if (cudaMemsetAsync(status, 0, sizeof(int), s) != cudaSuccess) return PDB_ECUDA;
+    if (X->n_rows > 0 && n_epochs > 0) {
+        const int64_t F = X->n_cols;
+        const int32_t n32 = (int32_t)X->n_rows;
+        const uint64_t tmo = timeout_ns(nullptr);
+        const int grid = persistent_grid((const void *)k_sgd_ready<8>, nullptr);
+        if (F > 0) {
+            k_pack<<<grid_1d(F), 256, 0, s>>>(w, F, rec, status);
+            note_launch();
+        }
+        for (int ep = 0; ep < n_epochs; ++ep) {
+            cudaMemsetAsync(ticket, 0, sizeof(unsigned long long), s);
+            k_sgd_ready<8><<<grid, THREADS, 0, s>>>(n32, X->row_ptr, X->col, X->val, y, gate, rec, (int)loss, eta,
+                                                    ticket, 2, status, tmo);
+            note_launch();
+        }
+        if (F > 0) {
+            k_unpack<<<grid_1d(F), 256, 0, s>>>(rec, F, w, status);
+            note_launch();
+        }
+    }
+    if (cudaPeekAtLastError() != cudaSuccess) {
+        cudaGetLastError();
+        return PDB_ECUDA;
+    }
+    int st = 0;
+    if (cudaMemcpyAsync(&st, status, sizeof(int), cudaMemcpyDeviceToHost, s) != cudaSuccess ||
+        cudaStreamSynchronize(s) != cudaSuccess)
+        return PDB_ECUDA;
+    return st;
+}
