@@ -69,9 +69,10 @@ __global__ void k_rows_scan(const int64_t *__restrict__ row_ptr, const int32_t *
 }
 
 // Slot order: gate[csc_pos[s]] = rank | last-occurrence bit (the one
-// scatter of the build), the longest chain, and -- only when some row is
-// unsorted -- the repeated-id check: two neighbouring slots of one feature
-// in the same example.
+// scatter of the build; grouping the writes by position first was measured
+// slower: the rate of scattered 4-byte stores, not DRAM, bounds it), the
+// longest chain, and -- only when some row is unsorted -- the repeated-id
+// check: two neighbouring slots of one feature in the same example.
 __global__ void k_slots(const uint32_t *__restrict__ skey, const int32_t *__restrict__ spos, int64_t nnz,
                         const int64_t *__restrict__ feat_ptr, const int32_t *__restrict__ row_of,
                         uint32_t *__restrict__ gate, int *info)

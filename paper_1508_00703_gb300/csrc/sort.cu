@@ -1,13 +1,7 @@
 // Stable LSD radix sort of (uint32 key, int32 value) pairs and segment
 // bounds of sorted keys, plus the small host helpers of libpdb.
 //
-// One pass per 8-bit digit.  A pass is: per-tile digit histogram (tiles of
-// 4096 pairs), a scan of the [tile][digit] counts in digit-major order done
-// hierarchically (chunk column sums, one-block scan of the chunk sums, chunk
-// down-sweep), and a scatter in which each tile ranks its pairs stably
-// (warp match on the digit, per-warp running counts, block prefix), stages
-// them in shared memory in output order and writes each digit's run with
-// consecutive threads.
+// One pass per digit of 8 to 10 bits (details at the radix sort section).
 #include <cuda_runtime.h>
 
 #include <algorithm>
@@ -101,216 +95,294 @@ int bits_for(int64_t max_key)
 }
 
 // ------------------------------------------------------------------ radix sort
+// Stable LSD radix sort, reduce-then-scan per pass (no inter-tile waiting):
+//   1. k_rs_hist:  digit counts of every 4096-pair tile, written tile-major;
+//   2. k_rs_chunk_sum / k_rs_chunk_scan / k_rs_chunk_down: the counts in
+//      digit-major order become the global output offset of each (tile,
+//      digit), computed hierarchically over chunks of 256 tiles;
+//   3. k_rs_scatter: each tile ranks its pairs stably (warp match on the
+//      digit, per-warp running counts, prefix over warps and digits), stages
+//      them in shared memory in output order, and writes every digit's run
+//      with consecutive threads.
+// Digits are D = 8..10 bits, equal for all passes (27-bit ids: 3 passes of 9).
 constexpr int RS_THREADS = 256;
 constexpr int RS_IPT = 16;
-constexpr int RS_TILE = RS_THREADS * RS_IPT;   // 4096 pairs per tile
+constexpr int RS_TILE = RS_THREADS * RS_IPT;   // pairs per tile
 constexpr int RS_CHUNK = 256;                  // tiles per scan chunk
 
+template <int D>
 __global__ __launch_bounds__(RS_THREADS) void k_rs_hist(const uint32_t *__restrict__ keys, int64_t n, int shift,
                                                          uint32_t *__restrict__ hist, const int *status)
 {
+    constexpr int RADIX = 1 << D;
+    __shared__ uint32_t h[WARPS][RADIX];
     if (read_status(status)) return;
-    __shared__ uint32_t h[WARPS][256];
-    for (int i = threadIdx.x; i < WARPS * 256; i += RS_THREADS) (&h[0][0])[i] = 0;
+    for (int i = threadIdx.x; i < WARPS * RADIX; i += RS_THREADS) (&h[0][0])[i] = 0;
+    const int64_t tile0 = (int64_t)blockIdx.x * RS_TILE;
+    const int ntile = (int)min64(RS_TILE, n - tile0);
+    uint32_t k[RS_IPT];
+#pragma unroll
+    for (int i = 0; i < RS_IPT; ++i) {
+        const int idx = i * RS_THREADS + threadIdx.x;
+        k[i] = idx < ntile ? __ldcs(keys + tile0 + idx) : 0u;
+    }
     __syncthreads();
     const int warp = threadIdx.x >> 5;
-    const int64_t base = (int64_t)blockIdx.x * RS_TILE;
-#pragma unroll 4
-    for (int i = 0; i < RS_IPT; ++i) {
-        int64_t idx = base + i * RS_THREADS + threadIdx.x;
-        if (idx < n) atomicAdd(&h[warp][(keys[idx] >> shift) & 255u], 1u);
-    }
-    __syncthreads();
-    uint32_t sum = 0;
 #pragma unroll
-    for (int w = 0; w < WARPS; ++w) sum += h[w][threadIdx.x];
-    hist[(int64_t)blockIdx.x * 256 + threadIdx.x] = sum;
-}
-
-// column sums of the [tile][digit] counts over each chunk of RS_CHUNK tiles
-__global__ __launch_bounds__(256) void k_rs_chunk_sum(const uint32_t *__restrict__ hist, int64_t n_tiles,
-                                                      uint32_t *__restrict__ csum, const int *status)
-{
-    if (read_status(status)) return;
-    int64_t t0 = (int64_t)blockIdx.x * RS_CHUNK;
-    int64_t t1 = min64(n_tiles, t0 + RS_CHUNK);
-    uint32_t s = 0;
-    for (int64_t t = t0; t < t1; ++t) s += hist[t * 256 + threadIdx.x];
-    csum[(int64_t)blockIdx.x * 256 + threadIdx.x] = s;
-}
-
-// one block: cbase[chunk][d] = (pairs with a smaller digit) + (pairs with
-// digit d in earlier chunks)
-__global__ __launch_bounds__(256) void k_rs_chunk_scan(const uint32_t *__restrict__ csum, int64_t n_chunks,
-                                                       uint32_t *__restrict__ cbase, const int *status)
-{
-    if (read_status(status)) return;
-    __shared__ uint32_t tot[256];
-    const int d = threadIdx.x;
-    uint32_t run = 0;
-    for (int64_t c = 0; c < n_chunks; ++c) run += csum[c * 256 + d];
-    tot[d] = run;
+    for (int i = 0; i < RS_IPT; ++i)
+        if (i * RS_THREADS + (int)threadIdx.x < ntile) atomicAdd(&h[warp][(k[i] >> shift) & (RADIX - 1)], 1u);
     __syncthreads();
-    if (d == 0) {
-        uint32_t acc = 0;
-        for (int i = 0; i < 256; ++i) {
-            uint32_t v = tot[i];
-            tot[i] = acc;
-            acc += v;
-        }
+    for (int d = threadIdx.x; d < RADIX; d += RS_THREADS) {
+        uint32_t sum = 0;
+#pragma unroll
+        for (int w = 0; w < WARPS; ++w) sum += h[w][d];
+        hist[(int64_t)blockIdx.x * RADIX + d] = sum;
     }
+}
+
+// column sums of the [tile][digit] counts over each chunk of RS_CHUNK tiles (RADIX threads)
+__global__ void k_rs_chunk_sum(const uint32_t *__restrict__ hist, int64_t n_tiles, int radix,
+                               uint32_t *__restrict__ csum, const int *status)
+{
+    if (read_status(status)) return;
+    const int64_t t0 = (int64_t)blockIdx.x * RS_CHUNK, t1 = min64(n_tiles, t0 + RS_CHUNK);
+    uint32_t s = 0;
+    for (int64_t t = t0; t < t1; ++t) s += hist[t * radix + threadIdx.x];
+    csum[(int64_t)blockIdx.x * radix + threadIdx.x] = s;
+}
+
+// one block of RADIX threads: cbase[chunk][d] = (pairs with a smaller digit)
+// + (pairs with digit d in earlier chunks)
+__global__ void k_rs_chunk_scan(const uint32_t *__restrict__ csum, int64_t n_chunks, int radix,
+                                uint32_t *__restrict__ cbase, const int *status)
+{
+    __shared__ uint32_t wsum[32];
+    if (read_status(status)) return;
+    const int d = threadIdx.x, lane = d & 31, warp = d >> 5;
+    uint32_t tot = 0;
+    for (int64_t c = 0; c < n_chunks; ++c) tot += csum[c * radix + d];
+    uint32_t x = tot;
+    for (int off = 1; off < 32; off <<= 1) {
+        uint32_t y = __shfl_up_sync(FULL, x, off);
+        if (lane >= off) x += y;
+    }
+    if (lane == 31) wsum[warp] = x;
     __syncthreads();
-    run = tot[d];
+    uint32_t run = x - tot;
+    for (int w = 0; w < warp; ++w) run += wsum[w];
     for (int64_t c = 0; c < n_chunks; ++c) {
-        uint32_t v = csum[c * 256 + d];
-        cbase[c * 256 + d] = run;
+        const uint32_t v = csum[c * radix + d];
+        cbase[c * radix + d] = run;
         run += v;
     }
 }
 
 // hist[tile][d] <- global output offset of digit d for that tile
-__global__ __launch_bounds__(256) void k_rs_chunk_down(uint32_t *__restrict__ hist, int64_t n_tiles,
-                                                       const uint32_t *__restrict__ cbase, const int *status)
+__global__ void k_rs_chunk_down(uint32_t *__restrict__ hist, int64_t n_tiles, int radix,
+                                const uint32_t *__restrict__ cbase, const int *status)
 {
     if (read_status(status)) return;
-    int64_t t0 = (int64_t)blockIdx.x * RS_CHUNK;
-    int64_t t1 = min64(n_tiles, t0 + RS_CHUNK);
-    uint32_t run = cbase[(int64_t)blockIdx.x * 256 + threadIdx.x];
-    for (int64_t t = t0; t < t1; ++t) {
-        uint32_t v = hist[t * 256 + threadIdx.x];
-        hist[t * 256 + threadIdx.x] = run;
-        run += v;
+    const int64_t t0 = (int64_t)blockIdx.x * RS_CHUNK, t1 = min64(n_tiles, t0 + RS_CHUNK);
+    uint32_t run = cbase[(int64_t)blockIdx.x * radix + threadIdx.x];
+    for (int64_t t = t0; t < t1; t += 16) {       // 16 loads in flight, then 16 stores
+        uint32_t v[16];
+#pragma unroll
+        for (int u = 0; u < 16; ++u) v[u] = t + u < t1 ? hist[(t + u) * radix + threadIdx.x] : 0u;
+#pragma unroll
+        for (int u = 0; u < 16; ++u)
+            if (t + u < t1) {
+                hist[(t + u) * radix + threadIdx.x] = run;
+                run += v[u];
+            }
     }
 }
 
-__global__ __launch_bounds__(RS_THREADS) void k_rs_scatter(const uint32_t *__restrict__ kin,
-                                                            const int32_t *__restrict__ vin,
-                                                            uint32_t *__restrict__ kout, int32_t *__restrict__ vout,
-                                                            int64_t n, int shift, const uint32_t *__restrict__ offs,
-                                                            const int *status)
+template <int D>
+__global__ __launch_bounds__(RS_THREADS, 3) void k_rs_scatter(const uint32_t *__restrict__ kin,
+                                                               const int32_t *__restrict__ vin,
+                                                               uint32_t *__restrict__ kout, int32_t *__restrict__ vout,
+                                                               int64_t n, int shift, const uint32_t *__restrict__ offs,
+                                                               const int *status)
 {
-    if (read_status(status)) return;
-    __shared__ uint32_t s_wcnt[WARPS][256];
-    __shared__ uint32_t s_tpre[256];
-    __shared__ uint32_t s_base[256];
+    constexpr int RADIX = 1 << D;
+    constexpr unsigned MASK = RADIX - 1;
+    constexpr int PER = (RADIX + RS_THREADS - 1) / RS_THREADS;
+    extern __shared__ uint32_t smem[];
+    uint32_t *s_wcnt = smem;                       // [WARPS][RADIX]
+    uint32_t *s_tpre = s_wcnt + WARPS * RADIX;     // [RADIX] tile counts, then tile-local offsets
+    uint32_t *s_base = s_tpre + RADIX;             // [RADIX] global offset of each digit for this tile
+    uint32_t *s_keys = s_base + RADIX;             // [RS_TILE]
+    int32_t *s_vals = (int32_t *)(s_keys + RS_TILE);   // [RS_TILE] values in output order
+    int32_t *s_vin = s_vals + RS_TILE;                  // [RS_TILE] values in input order
     __shared__ uint32_t s_wtot[WARPS];
-    __shared__ uint32_t s_keys[RS_TILE];
-    __shared__ int32_t s_vals[RS_TILE];
+    if (read_status(status)) return;
 
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    for (int i = tid; i < WARPS * 256; i += RS_THREADS) (&s_wcnt[0][0])[i] = 0;
-    s_base[tid] = offs[(int64_t)blockIdx.x * 256 + tid];
-    __syncthreads();
-
     const int64_t tile0 = (int64_t)blockIdx.x * RS_TILE;
-    const int64_t wbase = tile0 + (int64_t)warp * (32 * RS_IPT);
+    const int ntile = (int)min64(RS_TILE, n - tile0);
+    const uint32_t *tkin = kin + tile0;
+    const int wbase = warp * (32 * RS_IPT);
+    if (vin) {
+        // the tile's values travel to shared memory asynchronously while the keys are ranked
+        // (16-byte copies; the tile start is 16 KB aligned and vin is a 256-byte aligned buffer)
+        const int full = ntile & ~3;
+        for (int c = tid * 4; c < full; c += RS_THREADS * 4) {
+            const unsigned dst = (unsigned)__cvta_generic_to_shared(s_vin + c);
+            asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(vin + tile0 + c) : "memory");
+        }
+        asm volatile("cp.async.commit_group;" ::: "memory");
+        for (int c = full + tid; c < ntile; c += RS_THREADS) s_vin[c] = vin[tile0 + c];
+    }
+    uint32_t key[RS_IPT], pos[RS_IPT];
+#pragma unroll
+    for (int i = 0; i < RS_IPT; ++i) {          // all loads in flight before any ranking
+        const int idx = wbase + i * 32 + lane;
+        key[i] = idx < ntile ? __ldcs(tkin + idx) : 0u;
+    }
+    for (int i = tid; i < WARPS * RADIX; i += RS_THREADS) s_wcnt[i] = 0;
+    for (int d = tid; d < RADIX; d += RS_THREADS) s_base[d] = offs[(int64_t)blockIdx.x * RADIX + d];
+    __syncthreads();
     const unsigned lt = lanemask_lt();
-    uint32_t key[RS_IPT];
-    int32_t val[RS_IPT];
-    uint32_t pos[RS_IPT];
 #pragma unroll
     for (int i = 0; i < RS_IPT; ++i) {
-        int64_t idx = wbase + i * 32 + lane;
-        bool valid = idx < n;
-        key[i] = valid ? kin[idx] : 0u;
-        val[i] = valid ? (vin ? vin[idx] : (int32_t)idx) : 0;
-        unsigned d = valid ? ((key[i] >> shift) & 255u) : 256u;
-        unsigned peers = __match_any_sync(FULL, d);
-        unsigned rank = __popc(peers & lt);
-        unsigned cnt = valid ? s_wcnt[warp][d] : 0u;
+        const int idx = wbase + i * 32 + lane;
+        const bool valid = idx < ntile;
+        const unsigned d = valid ? ((key[i] >> shift) & MASK) : (unsigned)RADIX;
+        const unsigned peers = __match_any_sync(FULL, d);
+        const unsigned rank = __popc(peers & lt);
+        const unsigned cnt = valid ? s_wcnt[warp * RADIX + d] : 0u;
         pos[i] = cnt + rank;
         __syncwarp();
-        if (valid && rank == 0) s_wcnt[warp][d] = cnt + __popc(peers);
+        if (valid && rank == 0) s_wcnt[warp * RADIX + d] = cnt + __popc(peers);
         __syncwarp();
     }
     __syncthreads();
-    // per digit: exclusive prefix over warps, then over digits for the tile
-    {
-        const int d = tid;
+    // per digit: exclusive prefix over the warps and the tile count
+    for (int d = tid; d < RADIX; d += RS_THREADS) {
         uint32_t run = 0;
 #pragma unroll
         for (int w = 0; w < WARPS; ++w) {
-            uint32_t c = s_wcnt[w][d];
-            s_wcnt[w][d] = run;
+            const uint32_t c = s_wcnt[w * RADIX + d];
+            s_wcnt[w * RADIX + d] = run;
             run += c;
         }
-        // block exclusive scan of run over d = 0..255
-        uint32_t x = run;
+        s_tpre[d] = run;
+    }
+    __syncthreads();
+    // tile-local exclusive prefix of the digit counts
+    {
+        uint32_t local[PER], sum = 0;
+#pragma unroll
+        for (int q = 0; q < PER; ++q) {
+            const int d = tid * PER + q;
+            local[q] = d < RADIX ? s_tpre[d] : 0u;
+            sum += local[q];
+        }
+        uint32_t x = sum;
 #pragma unroll
         for (int off = 1; off < 32; off <<= 1) {
-            uint32_t y = __shfl_up_sync(FULL, x, off);
+            const uint32_t y = __shfl_up_sync(FULL, x, off);
             if (lane >= off) x += y;
         }
         if (lane == 31) s_wtot[warp] = x;
         __syncthreads();
-        uint32_t wpre = 0;
+        uint32_t excl = x - sum;
 #pragma unroll
-        for (int w = 0; w < WARPS; ++w) wpre += (w < warp) ? s_wtot[w] : 0u;
-        s_tpre[d] = wpre + x - run;
+        for (int w = 0; w < WARPS; ++w) excl += w < warp ? s_wtot[w] : 0u;
+#pragma unroll
+        for (int q = 0; q < PER; ++q) {
+            const int d = tid * PER + q;
+            if (d < RADIX) s_tpre[d] = excl;
+            excl += local[q];
+        }
     }
+    if (vin) asm volatile("cp.async.wait_group 0;" ::: "memory");
     __syncthreads();
 #pragma unroll
     for (int i = 0; i < RS_IPT; ++i) {
-        int64_t idx = wbase + i * 32 + lane;
-        if (idx < n) {
-            unsigned d = (key[i] >> shift) & 255u;
-            uint32_t li = s_tpre[d] + s_wcnt[warp][d] + pos[i];
+        const int idx = wbase + i * 32 + lane;
+        if (idx < ntile) {
+            const unsigned d = (key[i] >> shift) & MASK;
+            const uint32_t li = s_tpre[d] + s_wcnt[warp * RADIX + d] + pos[i];
             s_keys[li] = key[i];
-            s_vals[li] = val[i];
+            s_vals[li] = vin ? s_vin[idx] : (int32_t)(tile0 + idx);
         }
     }
     __syncthreads();
-    const int64_t ntile = min64(RS_TILE, n - tile0);
 #pragma unroll
     for (int i = 0; i < RS_IPT; ++i) {
-        int li = i * RS_THREADS + tid;
+        const int li = i * RS_THREADS + tid;
         if (li < ntile) {
-            uint32_t k = s_keys[li];
-            unsigned d = (k >> shift) & 255u;
-            uint32_t dest = s_base[d] + (uint32_t)li - s_tpre[d];
+            const uint32_t k = s_keys[li];
+            const unsigned d = (k >> shift) & MASK;
+            const uint32_t dest = s_base[d] + (uint32_t)li - s_tpre[d];
             kout[dest] = k;
             vout[dest] = s_vals[li];
         }
     }
 }
 
-int radix_sort(const uint32_t *keys_in, const int32_t *vals_in, uint32_t *keys_out, int32_t *vals_out,
-               uint32_t *keys_tmp, int32_t *vals_tmp, int64_t n, int key_bits, const int *status, cudaStream_t s)
+template <int D>
+int radix_passes(const uint32_t *keys_in, const int32_t *vals_in, uint32_t *keys_out, int32_t *vals_out,
+                 uint32_t *keys_tmp, int32_t *vals_tmp, int64_t n, int passes, const int *status, cudaStream_t s)
 {
-    if (n <= 0) return PDB_OK;
-    const int passes = std::max(1, (key_bits + 7) / 8);
+    constexpr int RADIX = 1 << D;
+    const size_t smem = sizeof(uint32_t) * ((size_t)(WARPS + 2) * RADIX + 3 * RS_TILE);
+    static bool configured[64] = {};
+    int dev = 0;
+    cudaGetDevice(&dev);
+    if (dev >= 0 && dev < 64 && !configured[dev]) {
+        if (cudaFuncSetAttribute(k_rs_scatter<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) !=
+            cudaSuccess)
+            return PDB_ECUDA;
+        configured[dev] = true;
+    }
     const int64_t n_tiles = (n + RS_TILE - 1) / RS_TILE;
     const int64_t n_chunks = (n_tiles + RS_CHUNK - 1) / RS_CHUNK;
     uint32_t *hist = nullptr, *csum = nullptr, *cbase = nullptr;
-    int rc = alloc((void **)&hist, sizeof(uint32_t) * 256 * n_tiles, s);
-    if (rc == PDB_OK) rc = alloc((void **)&csum, sizeof(uint32_t) * 256 * n_chunks, s);
-    if (rc == PDB_OK) rc = alloc((void **)&cbase, sizeof(uint32_t) * 256 * n_chunks, s);
-    if (rc != PDB_OK) {
-        release(hist, s);
-        release(csum, s);
-        release(cbase, s);
-        return rc;
-    }
-    const uint32_t *kin = keys_in;
-    const int32_t *vin = vals_in;
-    for (int p = 0; p < passes; ++p) {
-        // the last pass must land in *_out
-        bool to_out = ((passes - 1 - p) % 2) == 0;
-        uint32_t *ko = to_out ? keys_out : keys_tmp;
-        int32_t *vo = to_out ? vals_out : vals_tmp;
-        int shift = 8 * p;
-        k_rs_hist<<<(unsigned)n_tiles, RS_THREADS, 0, s>>>(kin, n, shift, hist, status); note_launch();
-        k_rs_chunk_sum<<<(unsigned)n_chunks, 256, 0, s>>>(hist, n_tiles, csum, status); note_launch();
-        k_rs_chunk_scan<<<1, 256, 0, s>>>(csum, n_chunks, cbase, status); note_launch();
-        k_rs_chunk_down<<<(unsigned)n_chunks, 256, 0, s>>>(hist, n_tiles, cbase, status); note_launch();
-        k_rs_scatter<<<(unsigned)n_tiles, RS_THREADS, 0, s>>>(kin, vin, ko, vo, n, shift, hist, status); note_launch();
-        kin = ko;
-        vin = vo;
+    int rc = alloc((void **)&hist, sizeof(uint32_t) * RADIX * n_tiles, s);
+    rc = rc ? rc : alloc((void **)&csum, sizeof(uint32_t) * RADIX * n_chunks, s);
+    rc = rc ? rc : alloc((void **)&cbase, sizeof(uint32_t) * RADIX * n_chunks, s);
+    if (rc == PDB_OK) {
+        const uint32_t *kin = keys_in;
+        const int32_t *vin = vals_in;
+        for (int p = 0; p < passes; ++p) {
+            const bool to_out = ((passes - 1 - p) % 2) == 0;   // the last pass lands in *_out
+            uint32_t *ko = to_out ? keys_out : keys_tmp;
+            int32_t *vo = to_out ? vals_out : vals_tmp;
+            const int shift = D * p;
+            k_rs_hist<D><<<(unsigned)n_tiles, RS_THREADS, 0, s>>>(kin, n, shift, hist, status);
+            note_launch();
+            k_rs_chunk_sum<<<(unsigned)n_chunks, RADIX, 0, s>>>(hist, n_tiles, RADIX, csum, status);
+            note_launch();
+            k_rs_chunk_scan<<<1, RADIX, 0, s>>>(csum, n_chunks, RADIX, cbase, status);
+            note_launch();
+            k_rs_chunk_down<<<(unsigned)n_chunks, RADIX, 0, s>>>(hist, n_tiles, RADIX, cbase, status);
+            note_launch();
+            k_rs_scatter<D><<<(unsigned)n_tiles, RS_THREADS, smem, s>>>(kin, vin, ko, vo, n, shift, hist, status);
+            note_launch();
+            kin = ko;
+            vin = vo;
+        }
     }
     release(hist, s);
     release(csum, s);
     release(cbase, s);
+    if (rc != PDB_OK) return rc;
     return cudaPeekAtLastError() == cudaSuccess ? PDB_OK : PDB_ECUDA;
+}
+
+int radix_sort(const uint32_t *keys_in, const int32_t *vals_in, uint32_t *keys_out, int32_t *vals_out,
+               uint32_t *keys_tmp, int32_t *vals_tmp, int64_t n, int key_bits, const int *status, cudaStream_t s)
+{
+    if (n <= 0) return PDB_OK;
+    // equal digit widths of 8..10 bits: 27-bit ids take 3 passes of 9
+    const int kb = std::max(1, std::min(key_bits, 32));
+    const int passes = (kb + 9) / 10;
+    const int d = std::max(8, (kb + passes - 1) / passes);
+    if (d == 8) return radix_passes<8>(keys_in, vals_in, keys_out, vals_out, keys_tmp, vals_tmp, n, passes, status, s);
+    if (d == 9) return radix_passes<9>(keys_in, vals_in, keys_out, vals_out, keys_tmp, vals_tmp, n, passes, status, s);
+    return radix_passes<10>(keys_in, vals_in, keys_out, vals_out, keys_tmp, vals_tmp, n, passes, status, s);
 }
 
 // ------------------------------------------------------------------ segment bounds

@@ -18,6 +18,8 @@ SMALL = {
     "deepchain-shape": ("deep-chain", dict(n_rows=5000)),
     "long-rows": ("tiny", dict(n_rows=1500, n_cols=5000, k=300, k_lo=200, labels="sign")),
     "wide-ids-4pass": ("low-conflict", dict(n_rows=3000, n_cols=20_000_000, k=50)),
+    "ids-18bit": ("zipf-1m", dict(n_rows=20000, n_cols=200_000)),
+    "ids-20bit": ("zipf-1m", dict(n_rows=20000, n_cols=1_000_000)),
 }
 
 FULL = {
