@@ -45,7 +45,7 @@ def parse_args(argv=None):
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default="low-conflict")
-    ap.add_argument("--mode", choices=["ready", "levels"], default="ready")
+    ap.add_argument("--mode", choices=["auto", "ready", "levels", "chain"], default="auto")
     ap.add_argument("--rows", type=int, default=None, help="override the workload's example count")
     ap.add_argument("--ticket-chunk", type=int, default=0, help="READY engine: examples per ticket (0 = default)")
     ap.add_argument("--blocks-per-sm", type=int, default=0)
@@ -278,7 +278,8 @@ def run_ours(args, rank, world, local_rank):
     overrides = {} if args.rows is None else {"n_rows": args.rows}
     p = synthdata.generate(args.workload, seed=synthdata.DATA_SEED + rank, **overrides)
     E = p.epochs
-    mode = pdb.PDB_SCHED_READY if args.mode == "ready" else pdb.PDB_SCHED_LEVELS
+    mode = {"auto": pdb.PDB_SCHED_AUTO, "ready": pdb.PDB_SCHED_READY, "levels": pdb.PDB_SCHED_LEVELS,
+            "chain": pdb.PDB_SCHED_CHAIN}[args.mode]
     X = pdb.Csr.from_problem(p)
     y = torch.from_numpy(p.y).cuda()
     w = torch.zeros(p.n_cols, dtype=torch.float32, device="cuda")
@@ -331,7 +332,9 @@ def run_ours(args, rank, world, local_rank):
     sgd_bytes_per_launch = ALG_BYTES_PER_NNZ * p.nnz + ALG_BYTES_PER_ROW * p.n_rows
     sgd_launch_ms = ms_kern / E
     sgd_gbs = sgd_bytes_per_launch / (sgd_launch_ms / 1e3) / 1e9
-    kname = "k_sgd_ready" if mode == pdb.PDB_SCHED_READY else "k_sgd_levels"
+    resolved = int(phases[0]["sched_mode"])
+    kname = {pdb.PDB_SCHED_READY: "k_sgd_ready", pdb.PDB_SCHED_LEVELS: "k_sgd_levels",
+             pdb.PDB_SCHED_CHAIN: "k_sgd_chain"}[resolved]
     roofline = {"kernel": kname,
                 "bound": "hbm", "achieved": round(sgd_gbs, 1), "peak": peak, "unit": "GB/s",
                 "frac": round(sgd_gbs / peak, 4), "traffic": recorded_traffic(kname, args.workload),
@@ -342,7 +345,8 @@ def run_ours(args, rank, world, local_rank):
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f32", "data": "synthetic (seeded generator, no dataset)",
-        "config": dict(workload_config(args.workload, p, args.mode),
+        "config": dict(workload_config(args.workload, p,
+                                       {0: "levels", 1: "ready", 2: "chain"}[resolved] + (" (auto)" if args.mode == "auto" else "")),
                        parallelism=f"replicas{world}" if world > 1 else "single GPU",
                        ticket_chunk=args.ticket_chunk or 2),
         "roofline": roofline,

@@ -89,8 +89,18 @@ typedef enum { PDB_LOSS_LOGISTIC = 0, PDB_LOSS_SQUARED = 1, PDB_LOSS_HINGE = 2 }
  *           r reads w_j once the iteration number of j equals r and
  *           publishes r + 1 with its write (the read protocol of Section 5
  *           with the iteration number counted per feature); no barrier at
- *           all.  The number lives in the same 64-bit word as the weight. */
-typedef enum { PDB_SCHED_LEVELS = 0, PDB_SCHED_READY = 1 } pdb_sched_mode;
+ *           all.  The number lives in the same 64-bit word as the weight.
+ *   CHAIN   for conflict graphs that are close to one chain (a feature in
+ *           most examples): one thread block runs the examples strictly in
+ *           data order (Algorithm 1 itself), prefetching ids, values and
+ *           weights ahead and forwarding each new weight whose next
+ *           occurrence is among the next 16 examples through shared memory,
+ *           so a dependency hop costs a few hundred cycles.  Examples of at
+ *           most 256 ids.
+ *   AUTO    CHAIN when the longest per-feature chain exceeds n_rows / 20 and
+ *           every example has at most 256 ids, else READY (waits on the host
+ *           for the conflict build to read those two numbers). */
+typedef enum { PDB_SCHED_LEVELS = 0, PDB_SCHED_READY = 1, PDB_SCHED_CHAIN = 2, PDB_SCHED_AUTO = 3 } pdb_sched_mode;
 
 /* Launch and wait options; a zeroed struct (or NULL) selects the defaults. */
 typedef struct {
@@ -108,6 +118,7 @@ typedef struct {
     int64_t max_chain;       /* most occurrences of one feature (longest per-feature chain) */
     double ms_build, ms_schedule, ms_sgd, ms_bsp;
     double ms_sgd_kernels;   /* pdb_sgd_epoch's update kernels alone (no record packing) */
+    int64_t sched_mode;      /* mode the schedule runs (AUTO resolved); -1 without a schedule */
 } pdb_stats;
 
 typedef struct pdb_conflicts pdb_conflicts; /* opaque, library-owned device arrays */
@@ -147,6 +158,11 @@ int pdb_conflicts_arrays(const pdb_conflicts *c, const int32_t **csc_pos, const 
  *   READY: one 64-bit record per feature, bits(w_j) | version_j << 32,
  *     filled from w by pdb_sgd_epoch; each position waits for the version
  *     equal to its occurrence rank (the conflicts' gate array).
+ *   CHAIN: per position, whether an example among the 16 before it writes
+ *     its feature last (its weight is then forwarded on chip) and where the
+ *     next occurrence sits if within the 16 examples after.
+ *     PDB_ETOOBIG when an example has more than 256 ids.
+ *   AUTO: one of the two above (see pdb_sched_mode).
  * Allocates stream-ordered on `stream`. */
 int pdb_schedule_build(const pdb_conflicts *c, pdb_sched_mode mode, pdb_schedule **out, void *stream);
 

@@ -29,7 +29,7 @@ PDB_OK, PDB_EINVAL, PDB_ERANGE, PDB_EDUP, PDB_ENOMEM, PDB_ECUDA, PDB_ETIMEOUT, P
 PDB_ETOOBIG = -9
 NOALLOC_MAX_COLS = 1 << 20
 PDB_LOSS_LOGISTIC, PDB_LOSS_SQUARED, PDB_LOSS_HINGE = 0, 1, 2
-PDB_SCHED_LEVELS, PDB_SCHED_READY = 0, 1
+PDB_SCHED_LEVELS, PDB_SCHED_READY, PDB_SCHED_CHAIN, PDB_SCHED_AUTO = 0, 1, 2, 3
 
 _lock = threading.Lock()
 _lib = None
@@ -97,7 +97,7 @@ class pdb_stats(ctypes.Structure):
     _fields_ = [("n_rows", ctypes.c_int64), ("n_cols", ctypes.c_int64), ("nnz", ctypes.c_int64),
                 ("n_levels", ctypes.c_int64), ("max_level_width", ctypes.c_int64), ("max_chain", ctypes.c_int64),
                 ("ms_build", ctypes.c_double), ("ms_schedule", ctypes.c_double), ("ms_sgd", ctypes.c_double),
-                ("ms_bsp", ctypes.c_double), ("ms_sgd_kernels", ctypes.c_double)]
+                ("ms_bsp", ctypes.c_double), ("ms_sgd_kernels", ctypes.c_double), ("sched_mode", ctypes.c_int64)]
 
     def as_dict(self):
         return {k: getattr(self, k) for k, _ in self._fields_}

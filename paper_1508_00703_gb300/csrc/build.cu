@@ -279,7 +279,7 @@ const char *pdb_strerror(int code)
     case PDB_ETIMEOUT: return "device-side wait expired";
     case PDB_EFAULT: return "internal invariant failed on the device";
     case PDB_ESTATE: return "handle in the wrong mode for this call";
-    case PDB_ETOOBIG: return "more features than the allocation-free variant's fixed scratch holds (2^20)";
+    case PDB_ETOOBIG: return "problem beyond a fixed limit (allocation-free scratch: 2^20 features; CHAIN: 256 ids per example)";
     default: return "unknown error";
     }
 }
@@ -399,7 +399,7 @@ void pdb_schedule_free(pdb_schedule *s)
 {
     if (!s) return;
     cudaDeviceSynchronize();
-    free_ptrs({s->level, s->order, s->indeg, s->queue, s->level_ptr, s->ctl, s->rec, s->bar, s->ticket});
+    free_ptrs({s->level, s->order, s->indeg, s->queue, s->level_ptr, s->ctl, s->rec, s->link, s->bar, s->ticket});
     if (s->ev0) cudaEventDestroy(s->ev0);
     if (s->ev1) cudaEventDestroy(s->ev1);
     delete s;
@@ -407,10 +407,22 @@ void pdb_schedule_free(pdb_schedule *s)
 
 int pdb_schedule_build(const pdb_conflicts *c, pdb_sched_mode mode, pdb_schedule **out, void *stream)
 {
-    if (!c || !out || (mode != PDB_SCHED_LEVELS && mode != PDB_SCHED_READY)) return PDB_EINVAL;
+    if (!c || !out || mode < PDB_SCHED_LEVELS || mode > PDB_SCHED_AUTO) return PDB_EINVAL;
     *out = nullptr;
     cudaStream_t s = (cudaStream_t)stream;
     pdb_conflicts *cm = const_cast<pdb_conflicts *>(c);
+    if (mode == PDB_SCHED_CHAIN || mode == PDB_SCHED_AUTO) {
+        // both need the longest row (and AUTO the longest chain) recorded by the build
+        if (cudaEventSynchronize(c->ev1) != cudaSuccess) {
+            cudaGetLastError();
+            return PDB_ECUDA;
+        }
+        const bool fits = c->h_info[INFO_MAX_ROW] <= chain_max_row();
+        if (mode == PDB_SCHED_AUTO)
+            mode = (fits && (int64_t)c->h_info[INFO_MAX_CHAIN] * 20 > c->n_rows) ? PDB_SCHED_CHAIN : PDB_SCHED_READY;
+        else if (!fits)
+            return PDB_ETOOBIG;
+    }
     pdb_schedule *h = new (std::nothrow) pdb_schedule();
     if (!h) return PDB_ENOMEM;
     h->c = c;
@@ -430,6 +442,10 @@ int pdb_schedule_build(const pdb_conflicts *c, pdb_sched_mode mode, pdb_schedule
     if (mode == PDB_SCHED_READY) {
         // one (weight, version) record per feature; filled from w by pdb_sgd_epoch
         rc = rc ? rc : alloc((void **)&h->rec, sizeof(unsigned long long) * F, s);
+    } else if (mode == PDB_SCHED_CHAIN) {
+        rc = rc ? rc : materialize_chains(cm, s);
+        rc = rc ? rc : alloc((void **)&h->link, sizeof(uint32_t) * nnz, s);
+        rc = rc ? rc : chain_schedule(c->prev, c->next, c->row_of, c->row_ptr, nnz, h->link, c->status, s);
     } else {
         rc = rc ? rc : materialize_chains(cm, s);
         if (rc == PDB_OK && !cm->npred) {
@@ -535,7 +551,9 @@ int pdb_get_stats(const pdb_conflicts *c, const pdb_schedule *h, pdb_stats *out)
     if (c->timed_sgd && cudaEventElapsedTime(&ms, c->ev_sgd0, c->ev_sgd1) == cudaSuccess) out->ms_sgd = ms;
     if (c->timed_sgd && cudaEventElapsedTime(&ms, c->ev_k0, c->ev_k1) == cudaSuccess) out->ms_sgd_kernels = ms;
     if (c->timed_bsp && cudaEventElapsedTime(&ms, c->ev_bsp0, c->ev_bsp1) == cudaSuccess) out->ms_bsp = ms;
+    out->sched_mode = -1;
     if (h) {
+        out->sched_mode = h->mode;
         if (h->timed && cudaEventElapsedTime(&ms, h->ev0, h->ev1) == cudaSuccess) out->ms_schedule = ms;
         if (h->mode == PDB_SCHED_LEVELS) {
             LevelCtl ctl;

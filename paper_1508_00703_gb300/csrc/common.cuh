@@ -28,6 +28,13 @@ int alloc(void **p, size_t bytes, cudaStream_t s);   // stream-ordered, 256-byte
 void release(void *p, cudaStream_t s);
 int bits_for(int64_t max_key);                        // bits to hold values 0..max_key (>= 1)
 int grid_1d(int64_t n);                               // blocks of 256 threads for a grid-stride loop
+
+// chain engine (chain.cu)
+int chain_max_row();
+int chain_schedule(const int32_t *prev, const int32_t *next, const int32_t *row_of, const int64_t *row_ptr,
+                   int64_t nnz, uint32_t *link, const int *status, cudaStream_t s);
+int chain_run(const pdb_csr *X, const float *y, const uint32_t *link, float *w, int loss, float eta, int epochs,
+              int max_row, int *status, cudaStream_t s);
 void note_launch();                                   // count one kernel launch (pdb_launch_count)
 
 // Stable LSD radix sort of (key, value) pairs, 8-bit digits.  vals_in ==
@@ -214,6 +221,7 @@ struct pdb_schedule {
     int64_t *level_ptr;
     LevelCtl *ctl;            // device
     unsigned long long *rec;  // READY: per feature (weight bits | version << 32)
+    uint32_t *link;           // CHAIN: per position, receive flag and push target
     pdb::GridBarrier *bar;    // barrier for the level-synchronous engine
     unsigned long long *ticket;
     cudaEvent_t ev0, ev1;

@@ -412,6 +412,10 @@ int pdb_sgd_epoch(const pdb_csr *X, const float *y, const pdb_conflicts *c, cons
             if (cudaLaunchCooperativeKernel(kern, grid, THREADS, args, 0, s) != cudaSuccess) rc = PDB_ECUDA;
             note_launch();
             cudaEventRecord(cm->ev_k1, s);
+        } else if (h->mode == PDB_SCHED_CHAIN) {
+            cudaEventRecord(cm->ev_k0, s);
+            rc = chain_run(X, y, h->link, w, lossi, eta, n_epochs, c->h_info[2], cm->status, s);
+            cudaEventRecord(cm->ev_k1, s);
         } else {
             auto kern = width == 2 ? k_sgd_ready<2> : width == 4 ? k_sgd_ready<4> : k_sgd_ready<8>;
             int grid = persistent_grid((const void *)kern, opts);

@@ -29,13 +29,14 @@ def _arr(ptr, n, dtype):
     return pdb.device_array(ptr, n, dtype).cpu().numpy()
 
 
-@pytest.mark.parametrize("name", ["tiny", "zipf-1m", "low-conflict"])
-def test_full_size_chains_and_ready_weights(name):
+@pytest.mark.parametrize("name", ["tiny", "zipf-1m", "low-conflict", "deep-chain", "ctr"])
+def test_full_size_chains_and_auto_weights(name):
+    # AUTO picks what bench.py runs: READY for tiny and low-conflict, CHAIN for the Zipf workloads
     p = synthdata.generate(name)
     X = pdb.Csr.from_problem(p)
     y = torch.from_numpy(p.y).cuda()
     c = pdb.pdb_build_conflicts(X)
-    s = pdb.pdb_schedule_build(c, pdb.PDB_SCHED_READY)
+    s = pdb.pdb_schedule_build(c, pdb.PDB_SCHED_AUTO)
     w = torch.zeros(p.n_cols, dtype=torch.float32, device="cuda")
     pdb.pdb_sgd_epoch(X, y, c, s, w, p.loss, p.eta, p.epochs)
     pdb.check_status(c)

@@ -97,14 +97,37 @@ def _sgd(name, mode, opts=None):
     return w.cpu().numpy()
 
 
-@pytest.mark.parametrize("mode", ["levels", "ready"])
+MODES = {"levels": pdb.PDB_SCHED_LEVELS, "ready": pdb.PDB_SCHED_READY, "chain": pdb.PDB_SCHED_CHAIN}
+
+
+@pytest.mark.parametrize("mode", list(MODES))
 @pytest.mark.parametrize("name", ALL)
 def test_sgd_weights(name, mode):
-    m = pdb.PDB_SCHED_LEVELS if mode == "levels" else pdb.PDB_SCHED_READY
-    got = _sgd(name, m)
+    p = C.problem(name)
+    longest = int(np.max(np.diff(p.row_ptr))) if p.n_rows else 0
+    if mode == "chain" and longest > 256:
+        with pytest.raises(pdb.PdbError) as e:
+            _sgd(name, MODES[mode])
+        assert e.value.code == pdb.PDB_ETOOBIG
+        return
+    got = _sgd(name, MODES[mode])
     ref = C.oracle_sgd(name)
     assert C.rel_err(got, ref) <= TOL
     assert np.array_equal(got, ref)       # same fp32 operation order on both sides
+
+
+@pytest.mark.parametrize("name,expect", [("tiny", "ready"), ("lowconflict-shape", "ready"),
+                                         ("zipf-shape", "chain"), ("deepchain-shape", "chain"),
+                                         ("ctr-shape-binary", "chain"), ("one-feature-chain", "chain")])
+def test_auto_schedule_choice(name, expect):
+    p, X, y = _gpu(name)
+    c = pdb.pdb_build_conflicts(X)
+    s = pdb.pdb_schedule_build(c, pdb.PDB_SCHED_AUTO)
+    assert pdb.pdb_get_stats(c, s)["sched_mode"] == MODES[expect]
+    w = torch.zeros(p.n_cols, dtype=torch.float32, device="cuda")
+    pdb.pdb_sgd_epoch(X, y, c, s, w, p.loss, p.eta, p.epochs)
+    pdb.check_status(c)
+    assert np.array_equal(w.cpu().numpy(), C.oracle_sgd(name))
 
 
 def test_sgd_small_grid_and_repeat_calls():
@@ -112,7 +135,7 @@ def test_sgd_small_grid_and_repeat_calls():
     name = "zipf-shape"
     p, X, y = _gpu(name)
     c = pdb.pdb_build_conflicts(X)
-    for mode in (pdb.PDB_SCHED_LEVELS, pdb.PDB_SCHED_READY):
+    for mode in (pdb.PDB_SCHED_LEVELS, pdb.PDB_SCHED_READY, pdb.PDB_SCHED_CHAIN):
         s = pdb.pdb_schedule_build(c, mode)
         w = torch.zeros(p.n_cols, dtype=torch.float32, device="cuda")
         pdb.pdb_sgd_epoch(X, y, c, s, w, p.loss, p.eta, 1, opts=dict(blocks_per_sm=1))
