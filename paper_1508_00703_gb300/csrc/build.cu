@@ -68,14 +68,15 @@ __global__ void k_rows_scan(const int64_t *__restrict__ row_ptr, const int32_t *
     if (lane == 0 && longest > 0) atomicMax(info + INFO_MAX_ROW, longest);
 }
 
-// Slot order: gate[csc_pos[s]] = rank | last-occurrence bit (the one
-// scatter of the build; grouping the writes by position first was measured
-// slower: the rate of scattered 4-byte stores, not DRAM, bounds it), the
+// Slot order: the gate word of every slot, rank | last-occurrence bit, the
 // longest chain, and -- only when some row is unsorted -- the repeated-id
-// check: two neighbouring slots of one feature in the same example.
+// check: two neighbouring slots of one feature in the same example.  The
+// gate words go to position order either directly (gate[csc_pos[s]], one
+// scattered 4-byte store per slot) or, for large inputs, in slot order
+// (gsort[s]) for the partitioned scatter below.
 __global__ void k_slots(const uint32_t *__restrict__ skey, const int32_t *__restrict__ spos, int64_t nnz,
                         const int64_t *__restrict__ feat_ptr, const int32_t *__restrict__ row_of,
-                        uint32_t *__restrict__ gate, int *info)
+                        uint32_t *__restrict__ gate, uint32_t *__restrict__ gsort, int *info)
 {
     if (read_status(info)) return;
     const bool check_dup = *(volatile int *)(info + INFO_UNSORTED) != 0;
@@ -86,13 +87,46 @@ __global__ void k_slots(const uint32_t *__restrict__ skey, const int32_t *__rest
         const int32_t p = spos[s];
         const bool last = s == nnz - 1 || skey[s + 1] != j;
         const int64_t r = s - feat_ptr[j];
-        gate[p] = (uint32_t)r | (last ? 0x80000000u : 0u);
+        const uint32_t g = (uint32_t)r | (last ? 0x80000000u : 0u);
+        if (gsort)
+            gsort[s] = g;
+        else
+            gate[p] = g;
         if (last) longest = max(longest, (int)(r + 1));
         if (check_dup && s > 0 && skey[s - 1] == j) dup |= row_of[spos[s - 1]] == row_of[p];
     }
     for (int off = 16; off >= 1; off >>= 1) longest = max(longest, __shfl_xor_sync(FULL, longest, off));
     if ((threadIdx.x & 31) == 0 && longest > 0) atomicMax(info + INFO_MAX_CHAIN, longest);
     if (__any_sync(FULL, dup) && (threadIdx.x & 31) == 0) set_status(info, PDB_EDUP);
+}
+
+// Last step of the gate scatter for large inputs.  The (position, gate)
+// pairs arrive sorted on the position bits above SB, so block b of the pair
+// array holds exactly the positions [b * 2^SB, (b + 1) * 2^SB) in some order
+// (positions are a permutation of the slots).  One thread block inverts that
+// piece in shared memory and writes it out contiguously: no ranking, and
+// DRAM sees whole lines instead of one scattered 4-byte store per slot.
+constexpr int SCATTER_SB = 14;                 // 2^14 slots = 64 KB of shared memory per block
+constexpr int SCATTER_THREADS = 512;
+__global__ __launch_bounds__(SCATTER_THREADS) void k_scatter_block(const uint32_t *__restrict__ ppos,
+                                                                  const uint32_t *__restrict__ pgate, int64_t nnz,
+                                                                  uint32_t *__restrict__ gate, int *info)
+{
+    extern __shared__ uint32_t piece[];
+    if (read_status(info)) return;
+    const int64_t base = (int64_t)blockIdx.x << SCATTER_SB;
+    const int cnt = (int)min64((int64_t)1 << SCATTER_SB, nnz - base);
+    bool bad = false;
+    for (int i = threadIdx.x; i < cnt; i += SCATTER_THREADS) {
+        const uint32_t off = __ldcs(ppos + base + i) - (uint32_t)base;
+        if (off < (uint32_t)cnt)
+            piece[off] = __ldcs(pgate + base + i);
+        else
+            bad = true;
+    }
+    if (bad) set_status(info, PDB_EFAULT);
+    __syncthreads();
+    for (int i = threadIdx.x; i < cnt; i += SCATTER_THREADS) gate[base + i] = piece[i];
 }
 
 // Position order: rank, previous and next occurrence of each position's feature.
@@ -349,8 +383,43 @@ int pdb_build_conflicts(const pdb_csr *X, pdb_conflicts **out, void *stream)
     }
     if (rc == PDB_OK) rc = segment_bounds(skey, nnz, F, nullptr, c->feat_ptr, c->info, s);
     if (rc == PDB_OK && nnz > 0) {
-        k_slots<<<grid_1d(nnz), 256, 0, s>>>(skey, c->csc_pos, nnz, c->feat_ptr, c->row_of, c->gate, c->info);
+        // up to 2^22 slots the gate array (16 MB) stays in L2 and the direct
+        // scatter is cheapest; above, sort the gate words back to position
+        // order (k_scatter_block)
+        const int pbits = bits_for(nnz - 1);
+        const bool partition = pbits > 22;
+        k_slots<<<grid_1d(nnz), 256, 0, s>>>(skey, c->csc_pos, nnz, c->feat_ptr, c->row_of, c->gate,
+                                             partition ? (uint32_t *)tval : nullptr, c->info);
         note_launch();
+        if (partition) {
+            // (position, gate) pairs sorted on the position bits above SCATTER_SB; skey is free after k_slots
+            uint32_t *pk = nullptr;
+            int32_t *pv = nullptr;
+            rc = alloc((void **)&pk, sizeof(uint32_t) * nnz, s);
+            rc = rc ? rc : alloc((void **)&pv, sizeof(int32_t) * nnz, s);
+            if (rc == PDB_OK)
+                rc = radix_sort_bits((const uint32_t *)c->csc_pos, tval, pk, pv, tkey, (int32_t *)skey, nnz,
+                                     SCATTER_SB, pbits, c->info, s);
+            if (rc == PDB_OK) {
+                const size_t smem = sizeof(uint32_t) << SCATTER_SB;
+                static bool configured[64] = {};
+                if (c->device >= 0 && c->device < 64 && !configured[c->device]) {
+                    if (cudaFuncSetAttribute(k_scatter_block, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) !=
+                        cudaSuccess)
+                        rc = PDB_ECUDA;
+                    else
+                        configured[c->device] = true;
+                }
+                if (rc == PDB_OK) {
+                    const int64_t blocks = ((nnz - 1) >> SCATTER_SB) + 1;
+                    k_scatter_block<<<(unsigned)blocks, SCATTER_THREADS, smem, s>>>(pk, (const uint32_t *)pv, nnz,
+                                                                                     c->gate, c->info);
+                    note_launch();
+                }
+            }
+            release(pk, s);
+            release(pv, s);
+        }
     }
     release(skey, s);
     release(tkey, s);

@@ -44,6 +44,10 @@ void note_launch();                                   // count one kernel launch
 int radix_sort(const uint32_t *keys_in, const int32_t *vals_in, uint32_t *keys_out, int32_t *vals_out,
                uint32_t *keys_tmp, int32_t *vals_tmp, int64_t n, int key_bits, const int *status,
                cudaStream_t s);
+// stable sort on key bits [lo_bit, hi_bit) only (the bits below stay in input order)
+int radix_sort_bits(const uint32_t *keys_in, const int32_t *vals_in, uint32_t *keys_out, int32_t *vals_out,
+                    uint32_t *keys_tmp, int32_t *vals_tmp, int64_t n, int lo_bit, int hi_bit, const int *status,
+                    cudaStream_t s);
 
 // ptr[k] = first index i of the sorted keys with keys[i] >= k, k = 0..n_bins
 // (n_bins read from *n_bins_dev when that is non-null).
