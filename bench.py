@@ -45,7 +45,7 @@ def parse_args(argv=None):
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default="low-conflict")
-    ap.add_argument("--mode", choices=["auto", "ready", "levels", "chain"], default="auto")
+    ap.add_argument("--mode", choices=["auto", "ready", "levels", "chain", "window"], default="auto")
     ap.add_argument("--rows", type=int, default=None, help="override the workload's example count")
     ap.add_argument("--ticket-chunk", type=int, default=0, help="READY engine: examples per ticket (0 = default)")
     ap.add_argument("--blocks-per-sm", type=int, default=0)
@@ -223,7 +223,8 @@ def recorded_traffic(kernel: str, workload: str):
     if not (m_b and m_h):
         return None
     h = hashlib.sha256()
-    for f in ("sgd.cu", "common.cuh"):
+    sources = {"k_sgd_window": "window.cu", "k_sgd_chain": "chain.cu"}.get(kernel, "sgd.cu")
+    for f in (sources, "common.cuh"):
         with open(os.path.join(ROOT, "paper_1508_00703_gb300", "csrc", f), "rb") as fh:
             h.update(fh.read())
     return float(m_b.group(1)) if h.hexdigest() == m_h.group(1) else None
@@ -279,7 +280,7 @@ def run_ours(args, rank, world, local_rank):
     p = synthdata.generate(args.workload, seed=synthdata.DATA_SEED + rank, **overrides)
     E = p.epochs
     mode = {"auto": pdb.PDB_SCHED_AUTO, "ready": pdb.PDB_SCHED_READY, "levels": pdb.PDB_SCHED_LEVELS,
-            "chain": pdb.PDB_SCHED_CHAIN}[args.mode]
+            "chain": pdb.PDB_SCHED_CHAIN, "window": pdb.PDB_SCHED_WINDOW}[args.mode]
     X = pdb.Csr.from_problem(p)
     y = torch.from_numpy(p.y).cuda()
     w = torch.zeros(p.n_cols, dtype=torch.float32, device="cuda")
@@ -334,7 +335,7 @@ def run_ours(args, rank, world, local_rank):
     sgd_gbs = sgd_bytes_per_launch / (sgd_launch_ms / 1e3) / 1e9
     resolved = int(phases[0]["sched_mode"])
     kname = {pdb.PDB_SCHED_READY: "k_sgd_ready", pdb.PDB_SCHED_LEVELS: "k_sgd_levels",
-             pdb.PDB_SCHED_CHAIN: "k_sgd_chain"}[resolved]
+             pdb.PDB_SCHED_CHAIN: "k_sgd_chain", pdb.PDB_SCHED_WINDOW: "k_sgd_window"}[resolved]
     roofline = {"kernel": kname,
                 "bound": "hbm", "achieved": round(sgd_gbs, 1), "peak": peak, "unit": "GB/s",
                 "frac": round(sgd_gbs / peak, 4), "traffic": recorded_traffic(kname, args.workload),
@@ -346,7 +347,8 @@ def run_ours(args, rank, world, local_rank):
         "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f32", "data": "synthetic (seeded generator, no dataset)",
         "config": dict(workload_config(args.workload, p,
-                                       {0: "levels", 1: "ready", 2: "chain"}[resolved] + (" (auto)" if args.mode == "auto" else "")),
+                                       {0: "levels", 1: "ready", 2: "chain", 4: "window"}[resolved]
+                                       + (" (auto)" if args.mode == "auto" else "")),
                        parallelism=f"replicas{world}" if world > 1 else "single GPU",
                        ticket_chunk=args.ticket_chunk or 2),
         "roofline": roofline,

@@ -56,7 +56,8 @@ extern "C" {
 #define PDB_ETIMEOUT (-6) /* a bounded device-side wait expired (the kernel stopped, the GPU stays usable) */
 #define PDB_EFAULT (-7)   /* an internal invariant failed on the device */
 #define PDB_ESTATE (-8)   /* wrong handle for this call (e.g. a READY schedule where levels are needed) */
-#define PDB_ETOOBIG (-9)  /* problem larger than the fixed scratch of pdb_sgd_epoch_ready_noalloc */
+#define PDB_ETOOBIG (-9)  /* beyond a fixed limit: the scratch of pdb_sgd_epoch_ready_noalloc, CHAIN's
+                             row length, or a feature occurring 2^29 times or more */
 
 /* ---------------------------------------------------------------- types */
 
@@ -97,10 +98,25 @@ typedef enum { PDB_LOSS_LOGISTIC = 0, PDB_LOSS_SQUARED = 1, PDB_LOSS_HINGE = 2 }
  *           occurrence is among the next 16 examples through shared memory,
  *           so a dependency hop costs a few hundred cycles.  Examples of at
  *           most 256 ids.
+ *   WINDOW  for conflict graphs whose consecutive occurrences of a feature
+ *           mostly lie far apart: w stays a plain float array.  A position
+ *           whose previous occurrence lies at least `near` positions back
+ *           (a distance fixed by the build, >= 2^22) reads w_j once the
+ *           completion watermark -- every example before it finished --
+ *           has passed that occurrence; a nearer one waits for feature j's
+ *           iteration number as under READY, kept in a separate word that
+ *           only near writers release.
  *   AUTO    CHAIN when the longest per-feature chain exceeds n_rows / 20 and
- *           every example has at most 256 ids, else READY (waits on the host
- *           for the conflict build to read those two numbers). */
-typedef enum { PDB_SCHED_LEVELS = 0, PDB_SCHED_READY = 1, PDB_SCHED_CHAIN = 2, PDB_SCHED_AUTO = 3 } pdb_sched_mode;
+ *           every example has at most 256 ids; else WINDOW when at most 1/8
+ *           of the positions have a near next occurrence; else READY (waits
+ *           on the host for the conflict build to read those numbers). */
+typedef enum {
+    PDB_SCHED_LEVELS = 0,
+    PDB_SCHED_READY = 1,
+    PDB_SCHED_CHAIN = 2,
+    PDB_SCHED_AUTO = 3,
+    PDB_SCHED_WINDOW = 4
+} pdb_sched_mode;
 
 /* Launch and wait options; a zeroed struct (or NULL) selects the defaults. */
 typedef struct {
@@ -134,6 +150,14 @@ typedef struct pdb_schedule pdb_schedule;   /* opaque, library-owned device arra
  *   feat_ptr[F+1]   feature j occupies csc_pos[feat_ptr[j] .. feat_ptr[j+1])
  *   prev[p], next[p] previous / next position holding col[p], -1 if none
  *   rank[p]         number of earlier positions holding col[p]
+ * It also marks, per position, whether the previous and the next
+ * occurrence lie within a distance `near` (the WINDOW schedule's input; see
+ * pdb_schedule_ready) and counts those pairs: near = 2^22 positions, or
+ * k * 2^15 rounded up to a power of two for a mean example length k > 128,
+ * or the value of the environment variable PDB_NEAR (>= 1) when set at
+ * this call.  Any near >= 1 gives the same SGD result; it only decides which
+ * positions wait on the watermark.
+ * A feature occurring 2^29 times or more is reported as PDB_ETOOBIG.
  * *out receives a new handle (free with pdb_conflicts_free) even when the
  * device later reports a CSR error through pdb_status.  The handle keeps
  * referring to X's arrays (D is immutable, Definition 1): they must stay
@@ -162,7 +186,9 @@ int pdb_conflicts_arrays(const pdb_conflicts *c, const int32_t **csc_pos, const 
  *     its feature last (its weight is then forwarded on chip) and where the
  *     next occurrence sits if within the 16 examples after.
  *     PDB_ETOOBIG when an example has more than 256 ids.
- *   AUTO: one of the two above (see pdb_sched_mode).
+ *   WINDOW: per feature a 32-bit iteration number, per example a finished
+ *     flag, and the watermark; the positions' near flags are in the gate.
+ *   AUTO: CHAIN, WINDOW or READY (see pdb_sched_mode).
  * Allocates stream-ordered on `stream`. */
 int pdb_schedule_build(const pdb_conflicts *c, pdb_sched_mode mode, pdb_schedule **out, void *stream);
 
@@ -172,11 +198,14 @@ int pdb_schedule_build(const pdb_conflicts *c, pdb_sched_mode mode, pdb_schedule
 int pdb_schedule_levels(const pdb_schedule *s, const int32_t **level, const int32_t **order,
                         const int64_t **level_ptr, int64_t *n_levels, void *stream);
 
-/* READY schedule arrays (borrowed device pointers, any may be NULL):
- * gate[nnz] the version each position waits for (its occurrence rank) with
- * bit 31 set on the last occurrence of its feature, and records[n_cols]
- * (weight bits | version << 32, meaningful while pdb_sgd_epoch runs).
- * PDB_ESTATE for a LEVELS schedule. */
+/* READY and WINDOW schedule arrays (borrowed device pointers, any may be
+ * NULL): gate[nnz], per position bits 0..28 the version it waits for (its
+ * occurrence rank), bit 29 set when the next occurrence of its feature lies
+ * within the build's `near` distance, bit 30 when the previous one does,
+ * bit 31 on the last occurrence of its feature; and, READY only,
+ * records[n_cols] (weight bits | version << 32, meaningful while
+ * pdb_sgd_epoch runs; NULL under WINDOW).  PDB_ESTATE for LEVELS and CHAIN
+ * schedules. */
 int pdb_schedule_ready(const pdb_schedule *s, const uint32_t **gate, const uint64_t **records);
 
 /* n_epochs passes of SGD over X in data order (Algorithm 1 with one
@@ -232,8 +261,9 @@ const char *pdb_strerror(int code);
  * every GPU loading the library holds until the process exits.
  *   X, y, w     as for pdb_sgd_epoch; X->n_cols must be <= 2^20, else
  *               PDB_ETOOBIG and nothing runs.
- *   gate[nnz]   per position, the occurrence rank of its feature with bit 31
- *               set on the feature's last occurrence -- the array that
+ *   gate[nnz]   per position, the gate word (occurrence rank of its feature
+ *               in bits 0..28, bit 31 on the feature's last occurrence,
+ *               bits 29-30 ignored here) -- the array that
  *               pdb_schedule_ready returns for a READY schedule of X (device,
  *               caller-owned here).
  * Same arithmetic and result as pdb_sgd_epoch.  The first call on each

@@ -29,7 +29,7 @@ PDB_OK, PDB_EINVAL, PDB_ERANGE, PDB_EDUP, PDB_ENOMEM, PDB_ECUDA, PDB_ETIMEOUT, P
 PDB_ETOOBIG = -9
 NOALLOC_MAX_COLS = 1 << 20
 PDB_LOSS_LOGISTIC, PDB_LOSS_SQUARED, PDB_LOSS_HINGE = 0, 1, 2
-PDB_SCHED_LEVELS, PDB_SCHED_READY, PDB_SCHED_CHAIN, PDB_SCHED_AUTO = 0, 1, 2, 3
+PDB_SCHED_LEVELS, PDB_SCHED_READY, PDB_SCHED_CHAIN, PDB_SCHED_AUTO, PDB_SCHED_WINDOW = 0, 1, 2, 3, 4
 
 _lock = threading.Lock()
 _lib = None

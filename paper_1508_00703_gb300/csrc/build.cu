@@ -27,7 +27,7 @@ using namespace pdb;
 
 namespace {
 
-enum { INFO_STATUS = 0, INFO_MAX_CHAIN = 1, INFO_MAX_ROW = 2, INFO_UNSORTED = 3, INFO_WORDS = 4 };
+enum { INFO_STATUS = 0, INFO_MAX_CHAIN = 1, INFO_MAX_ROW = 2, INFO_UNSORTED = 3, INFO_NEAR = 4, INFO_WORDS = 5 };
 
 // row_ptr[0] = 0, row_ptr[N] = nnz, nondecreasing (Definition 1: D is a list of examples)
 __global__ void k_validate_rows(const int64_t *__restrict__ row_ptr, int64_t n_rows, int64_t nnz, int *info)
@@ -75,29 +75,39 @@ __global__ void k_rows_scan(const int64_t *__restrict__ row_ptr, const int32_t *
 // scattered 4-byte store per slot) or, for large inputs, in slot order
 // (gsort[s]) for the partitioned scatter below.
 __global__ void k_slots(const uint32_t *__restrict__ skey, const int32_t *__restrict__ spos, int64_t nnz,
-                        const int64_t *__restrict__ feat_ptr, const int32_t *__restrict__ row_of,
+                        const int64_t *__restrict__ feat_ptr, const int32_t *__restrict__ row_of, int64_t near,
                         uint32_t *__restrict__ gate, uint32_t *__restrict__ gsort, int *info)
 {
     if (read_status(info)) return;
     const bool check_dup = *(volatile int *)(info + INFO_UNSORTED) != 0;
-    int longest = 0;
-    bool dup = false;
+    int longest = 0, n_near = 0;
+    bool dup = false, big = false;
     for (int64_t s = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; s < nnz; s += (int64_t)gridDim.x * blockDim.x) {
         const uint32_t j = skey[s];
         const int32_t p = spos[s];
         const bool last = s == nnz - 1 || skey[s + 1] != j;
         const int64_t r = s - feat_ptr[j];
-        const uint32_t g = (uint32_t)r | (last ? 0x80000000u : 0u);
+        const bool near_prev = r > 0 && (int64_t)p - spos[s - 1] < near;
+        const bool near_next = !last && (int64_t)spos[s + 1] - p < near;
+        big |= r > (int64_t)GATE_RANK;
+        n_near += near_next;
+        const uint32_t g = ((uint32_t)r & GATE_RANK) | (near_next ? GATE_NEAR_NEXT : 0u) |
+                           (near_prev ? GATE_NEAR_PREV : 0u) | (last ? GATE_LAST : 0u);
         if (gsort)
             gsort[s] = g;
         else
             gate[p] = g;
         if (last) longest = max(longest, (int)(r + 1));
-        if (check_dup && s > 0 && skey[s - 1] == j) dup |= row_of[spos[s - 1]] == row_of[p];
+        if (check_dup && r > 0) dup |= row_of[spos[s - 1]] == row_of[p];
     }
-    for (int off = 16; off >= 1; off >>= 1) longest = max(longest, __shfl_xor_sync(FULL, longest, off));
+    for (int off = 16; off >= 1; off >>= 1) {
+        longest = max(longest, __shfl_xor_sync(FULL, longest, off));
+        n_near += __shfl_xor_sync(FULL, n_near, off);
+    }
     if ((threadIdx.x & 31) == 0 && longest > 0) atomicMax(info + INFO_MAX_CHAIN, longest);
+    if ((threadIdx.x & 31) == 0 && n_near > 0) atomicAdd(info + INFO_NEAR, n_near);
     if (__any_sync(FULL, dup) && (threadIdx.x & 31) == 0) set_status(info, PDB_EDUP);
+    if (__any_sync(FULL, big) && (threadIdx.x & 31) == 0) set_status(info, PDB_ETOOBIG);
 }
 
 // Last step of the gate scatter for large inputs.  The (position, gate)
@@ -138,11 +148,11 @@ __global__ void k_materialize(const int32_t *__restrict__ col, const uint32_t *_
     if (read_status(info)) return;
     for (int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; p < nnz; p += (int64_t)gridDim.x * blockDim.x) {
         const uint32_t g = gate[p];
-        const int32_t r = (int32_t)(g & 0x7fffffffu);
+        const int32_t r = (int32_t)(g & GATE_RANK);
         const int64_t s = feat_ptr[col[p]] + r;
         rank[p] = r;
         prev[p] = r > 0 ? csc_pos[s - 1] : -1;
-        next[p] = (g >> 31) ? -1 : csc_pos[s + 1];
+        next[p] = (g & GATE_LAST) ? -1 : csc_pos[s + 1];
     }
 }
 
@@ -313,7 +323,9 @@ const char *pdb_strerror(int code)
     case PDB_ETIMEOUT: return "device-side wait expired";
     case PDB_EFAULT: return "internal invariant failed on the device";
     case PDB_ESTATE: return "handle in the wrong mode for this call";
-    case PDB_ETOOBIG: return "problem beyond a fixed limit (allocation-free scratch: 2^20 features; CHAIN: 256 ids per example)";
+    case PDB_ETOOBIG:
+        return "problem beyond a fixed limit (allocation-free scratch: 2^20 features; CHAIN: 256 ids per example; "
+               "a feature in 2^29 positions or more)";
     default: return "unknown error";
     }
 }
@@ -346,6 +358,20 @@ int pdb_build_conflicts(const pdb_csr *X, pdb_conflicts **out, void *stream)
     c->col = X->col;
     c->val = X->val;
     const int64_t N = X->n_rows, F = X->n_cols, nnz = X->nnz;
+    // WINDOW distance: several times the positions one persistent grid holds
+    // in flight (~15k examples), at least 2^22
+    {
+        const int64_t k_mean = N > 0 ? (nnz + N - 1) / N : 1;
+        int64_t near = (int64_t)1 << 22;
+        while (near < k_mean * ((int64_t)1 << 15) && near < ((int64_t)1 << 29)) near <<= 1;
+        // PDB_NEAR overrides it (any value >= 1 gives the same result; small
+        // values exercise the watermark path on small inputs)
+        if (const char *env = std::getenv("PDB_NEAR")) {
+            const long long v = std::atoll(env);
+            if (v >= 1) near = std::min<int64_t>(v, (int64_t)1 << 30);
+        }
+        c->near = near;
+    }
     for (cudaEvent_t *e : {&c->ev0, &c->ev1, &c->ev_sgd0, &c->ev_sgd1, &c->ev_bsp0, &c->ev_bsp1, &c->ev_k0, &c->ev_k1})
         if (cudaEventCreate(e) != cudaSuccess) {
             pdb_conflicts_free(c);
@@ -388,7 +414,7 @@ int pdb_build_conflicts(const pdb_csr *X, pdb_conflicts **out, void *stream)
         // order (k_scatter_block)
         const int pbits = bits_for(nnz - 1);
         const bool partition = pbits > 22;
-        k_slots<<<grid_1d(nnz), 256, 0, s>>>(skey, c->csc_pos, nnz, c->feat_ptr, c->row_of, c->gate,
+        k_slots<<<grid_1d(nnz), 256, 0, s>>>(skey, c->csc_pos, nnz, c->feat_ptr, c->row_of, c->near, c->gate,
                                              partition ? (uint32_t *)tval : nullptr, c->info);
         note_launch();
         if (partition) {
@@ -468,7 +494,8 @@ void pdb_schedule_free(pdb_schedule *s)
 {
     if (!s) return;
     cudaDeviceSynchronize();
-    free_ptrs({s->level, s->order, s->indeg, s->queue, s->level_ptr, s->ctl, s->rec, s->link, s->bar, s->ticket});
+    free_ptrs({s->level, s->order, s->indeg, s->queue, s->level_ptr, s->ctl, s->rec, s->link, s->bar, s->ticket,
+               s->prog, s->wctl});
     if (s->ev0) cudaEventDestroy(s->ev0);
     if (s->ev1) cudaEventDestroy(s->ev1);
     delete s;
@@ -476,7 +503,7 @@ void pdb_schedule_free(pdb_schedule *s)
 
 int pdb_schedule_build(const pdb_conflicts *c, pdb_sched_mode mode, pdb_schedule **out, void *stream)
 {
-    if (!c || !out || mode < PDB_SCHED_LEVELS || mode > PDB_SCHED_AUTO) return PDB_EINVAL;
+    if (!c || !out || mode < PDB_SCHED_LEVELS || mode > PDB_SCHED_WINDOW) return PDB_EINVAL;
     *out = nullptr;
     cudaStream_t s = (cudaStream_t)stream;
     pdb_conflicts *cm = const_cast<pdb_conflicts *>(c);
@@ -487,8 +514,12 @@ int pdb_schedule_build(const pdb_conflicts *c, pdb_sched_mode mode, pdb_schedule
             return PDB_ECUDA;
         }
         const bool fits = c->h_info[INFO_MAX_ROW] <= chain_max_row();
+        // AUTO: one chain dominates -> CHAIN; near occurrence pairs rare
+        // (at most 1/8 of the positions) -> WINDOW; else READY
         if (mode == PDB_SCHED_AUTO)
-            mode = (fits && (int64_t)c->h_info[INFO_MAX_CHAIN] * 20 > c->n_rows) ? PDB_SCHED_CHAIN : PDB_SCHED_READY;
+            mode = (fits && (int64_t)c->h_info[INFO_MAX_CHAIN] * 20 > c->n_rows) ? PDB_SCHED_CHAIN
+                   : (int64_t)c->h_info[INFO_NEAR] * 8 <= c->nnz                  ? PDB_SCHED_WINDOW
+                                                                                 : PDB_SCHED_READY;
         else if (!fits)
             return PDB_ETOOBIG;
     }
@@ -511,6 +542,17 @@ int pdb_schedule_build(const pdb_conflicts *c, pdb_sched_mode mode, pdb_schedule
     if (mode == PDB_SCHED_READY) {
         // one (weight, version) record per feature; filled from w by pdb_sgd_epoch
         rc = rc ? rc : alloc((void **)&h->rec, sizeof(unsigned long long) * F, s);
+    } else if (mode == PDB_SCHED_WINDOW) {
+        // near hand-off records (tag 0 = none: tags carry a nonzero epoch
+        // stamp), one progress word per warp the device can hold resident,
+        // the watermark (progress and watermark reset every epoch)
+        int sms = 0;
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, c->device);
+        h->prog_cap = (int64_t)std::max(sms, 1) * 64;
+        rc = rc ? rc : alloc((void **)&h->rec, sizeof(unsigned long long) * std::max<int64_t>(F, 1), s);
+        if (rc == PDB_OK) cudaMemsetAsync(h->rec, 0, sizeof(unsigned long long) * std::max<int64_t>(F, 1), s);
+        rc = rc ? rc : alloc((void **)&h->prog, sizeof(unsigned) * h->prog_cap, s);
+        rc = rc ? rc : alloc((void **)&h->wctl, sizeof(WindowCtl), s);
     } else if (mode == PDB_SCHED_CHAIN) {
         rc = rc ? rc : materialize_chains(cm, s);
         rc = rc ? rc : alloc((void **)&h->link, sizeof(uint32_t) * nnz, s);
@@ -596,9 +638,9 @@ int pdb_schedule_levels(const pdb_schedule *h, const int32_t **level, const int3
 int pdb_schedule_ready(const pdb_schedule *h, const uint32_t **gate, const uint64_t **records)
 {
     if (!h) return PDB_EINVAL;
-    if (h->mode != PDB_SCHED_READY) return PDB_ESTATE;
+    if (h->mode != PDB_SCHED_READY && h->mode != PDB_SCHED_WINDOW) return PDB_ESTATE;
     if (gate) *gate = h->c->gate;
-    if (records) *records = (const uint64_t *)h->rec;
+    if (records) *records = (const uint64_t *)h->rec;   // NULL under WINDOW
     return PDB_OK;
 }
 

@@ -188,6 +188,26 @@ __device__ __forceinline__ float warp_combine(float a)
     return a;
 }
 
+// Gate word of a position (the conflicts' per-position schedule input):
+// bits 0..28 occurrence rank of its feature, bit 29 the next occurrence lies
+// within `near` positions, bit 30 the previous one does, bit 31 last
+// occurrence of the feature.
+constexpr uint32_t GATE_RANK = 0x1fffffffu;
+constexpr uint32_t GATE_NEAR_NEXT = 1u << 29;
+constexpr uint32_t GATE_NEAR_PREV = 1u << 30;
+constexpr uint32_t GATE_LAST = 1u << 31;
+
+// WINDOW engine control block (device), zeroed before every epoch
+struct WindowCtl {
+    unsigned long long ticket;  // next example to hand out
+    long long wpos;             // every example starting below this position has finished
+};
+
+int window_run(const pdb_csr *X, const float *y, const uint32_t *gate, float *w, unsigned long long *rec,
+               unsigned *epoch_count, unsigned *prog, int64_t prog_cap, WindowCtl *ctl, int64_t near, int loss,
+               float eta, int n_epochs, int width, const pdb_opts *opts, int *status, uint64_t timeout,
+               cudaStream_t s);
+
 }  // namespace pdb
 
 // ------------------------------------------------------------------ handles
@@ -199,11 +219,13 @@ struct pdb_conflicts {
     const float *val;
     int32_t *csc_pos;        // positions grouped by feature, data order inside a feature
     int64_t *feat_ptr;       // [F+1]
-    uint32_t *gate;          // per position: occurrence rank, bit 31 = last occurrence of the feature
+    uint32_t *gate;          // per position: occurrence rank and flags (GATE_* below)
+    int64_t near;            // distance (positions) under which an occurrence pair counts as near
     int32_t *row_of;         // example of each position
     int32_t *prev, *next, *rank;  // materialized from the above on first request
     int32_t *npred;          // per example: occurrences with an earlier occurrence (LEVELS)
-    int *info;               // device: [0] status, [1] max chain, [2] longest row, [3] any unsorted row
+    int *info;               // device: [0] status, [1] max chain, [2] longest row, [3] any unsorted row,
+                             // [4] near occurrence pairs
     int *h_info;             // pinned host copy of info, filled at the end of the build
     cudaEvent_t ev0, ev1, ev_sgd0, ev_sgd1, ev_bsp0, ev_bsp1, ev_k0, ev_k1;
     bool timed_build, timed_sgd, timed_bsp;
@@ -224,8 +246,12 @@ struct pdb_schedule {
     int32_t *level, *order, *indeg, *queue;
     int64_t *level_ptr;
     LevelCtl *ctl;            // device
-    unsigned long long *rec;  // READY: per feature (weight bits | version << 32)
+    unsigned long long *rec;  // READY: per feature (weight bits | version << 32); WINDOW: near hand-offs
     uint32_t *link;           // CHAIN: per position, receive flag and push target
+    unsigned epochs_run;      // WINDOW: epochs run so far (epoch stamp of the record tags)
+    unsigned *prog;           // WINDOW: progress word per worker warp
+    int64_t prog_cap;
+    pdb::WindowCtl *wctl;     // WINDOW: ticket and watermark
     pdb::GridBarrier *bar;    // barrier for the level-synchronous engine
     unsigned long long *ticket;
     cudaEvent_t ev0, ev1;

@@ -108,7 +108,7 @@ __global__ __launch_bounds__(THREADS) void k_sgd_levels(int32_t n_rows, const in
 // Constraint: the previous writer is done) -- and publishes the new weight
 // together with version r + 1 in one 64-bit store (Write Constraint: its own
 // read, the only read of that version, came first).  The last occurrence of
-// j in the epoch (gate bit 31) writes version 0 for the next epoch.  Both
+// j in the epoch (GATE_LAST) writes version 0 for the next epoch.  Both
 // halves travel in one single-copy-atomic access, so no fence is needed.
 // Examples are taken in data order from a ticket counter, `chunk`
 // consecutive ones at a time and run in order by the warp that took them,
@@ -189,8 +189,8 @@ __device__ __forceinline__ bool ready_example(int t, const int64_t *__restrict__
             j[r] = i < k ? col[b + i] : 0;
             x[r] = i < k ? (val ? val[b + i] : 1.0f) : 0.0f;
             uint32_t g = i < k ? gate[b + i] : 0u;
-            want[r] = g & 0x7fffffffu;
-            next[r] = (g >> 31) ? 0u : want[r] + 1u;
+            want[r] = g & GATE_RANK;
+            next[r] = (g & GATE_LAST) ? 0u : want[r] + 1u;
             wv[r] = 0.0f;
         }
         bool ok = gather_ready<R>(rec, j, want, wv, lane, k, status, timeout);
@@ -213,7 +213,7 @@ __device__ __forceinline__ bool ready_example(int t, const int64_t *__restrict__
     bool ok = true;
     for (int i = lane; i < k && ok; i += 32) {
         int j1[1] = {col[b + i]};
-        unsigned w1[1] = {gate[b + i] & 0x7fffffffu};
+        unsigned w1[1] = {gate[b + i] & GATE_RANK};
         float v1[1];
         ok = gather_ready<1>(rec, j1, w1, v1, 0, 1, status, timeout);
         if (ok) acc = __fmaf_rn(v1[0], val ? val[b + i] : 1.0f, acc);
@@ -226,7 +226,7 @@ __device__ __forceinline__ bool ready_example(int t, const int64_t *__restrict__
         const float xx = val ? val[b + i] : 1.0f;
         const uint32_t g = gate[b + i];
         const float wo = __uint_as_float((unsigned)ld_rec(rec + jj));
-        st_rec(rec + jj, __fsub_rn(wo, __fmul_rn(c, xx)), (g >> 31) ? 0u : (g & 0x7fffffffu) + 1u);
+        st_rec(rec + jj, __fsub_rn(wo, __fmul_rn(c, xx)), (g & GATE_LAST) ? 0u : (g & GATE_RANK) + 1u);
     }
     return true;
 }
@@ -415,6 +415,12 @@ int pdb_sgd_epoch(const pdb_csr *X, const float *y, const pdb_conflicts *c, cons
         } else if (h->mode == PDB_SCHED_CHAIN) {
             cudaEventRecord(cm->ev_k0, s);
             rc = chain_run(X, y, h->link, w, lossi, eta, n_epochs, c->h_info[2], cm->status, s);
+            cudaEventRecord(cm->ev_k1, s);
+        } else if (h->mode == PDB_SCHED_WINDOW) {
+            cudaEventRecord(cm->ev_k0, s);
+            pdb_schedule *hm = const_cast<pdb_schedule *>(h);
+            rc = window_run(X, y, c->gate, w, h->rec, &hm->epochs_run, h->prog, h->prog_cap, h->wctl, c->near, lossi,
+                            eta, n_epochs, width, opts, cm->status, tmo, s);
             cudaEventRecord(cm->ev_k1, s);
         } else {
             auto kern = width == 2 ? k_sgd_ready<2> : width == 4 ? k_sgd_ready<4> : k_sgd_ready<8>;

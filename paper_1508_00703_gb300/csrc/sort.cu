@@ -243,13 +243,16 @@ __global__ __launch_bounds__(RS_THREADS, 3) void k_rs_scatter(const uint32_t *__
     for (int d = tid; d < RADIX; d += RS_THREADS) s_base[d] = offs[(int64_t)blockIdx.x * RADIX + d];
     __syncthreads();
     const unsigned lt = lanemask_lt();
+    // 1. lanes holding the same digit, for all the thread's elements at once
+    //    (one ballot per digit bit plus the valid bit, intersected; the
+    //    ballots of different elements are independent, so they overlap):
+    //    rank among the equal lanes, run length, leader flag
+    uint32_t info[RS_IPT];
 #pragma unroll
     for (int i = 0; i < RS_IPT; ++i) {
         const int idx = wbase + i * 32 + lane;
         const bool valid = idx < ntile;
         const unsigned d = valid ? ((key[i] >> shift) & MASK) : (unsigned)RADIX;
-        // lanes holding the same digit: one ballot per digit bit (plus the
-        // valid bit), intersected -- cheaper than a warp match instruction
         unsigned peers = __ballot_sync(FULL, valid);
         if (!valid) peers = ~peers;
 #pragma unroll
@@ -257,11 +260,18 @@ __global__ __launch_bounds__(RS_THREADS, 3) void k_rs_scatter(const uint32_t *__
             const unsigned m = __ballot_sync(FULL, (d >> b) & 1u);
             peers &= ((d >> b) & 1u) ? m : ~m;
         }
-        const unsigned rank = __popc(peers & lt);
+        info[i] = d | (__popc(peers & lt) << 16) | (__popc(peers) << 24);
+    }
+    // 2. per-warp running count of each digit (the only serial part)
+#pragma unroll
+    for (int i = 0; i < RS_IPT; ++i) {
+        const unsigned d = info[i] & 0xffffu;
+        const unsigned rank = (info[i] >> 16) & 0xffu;
+        const bool valid = d < (unsigned)RADIX;
         const unsigned cnt = valid ? s_wcnt[warp * RADIX + d] : 0u;
         pos[i] = cnt + rank;
         __syncwarp();
-        if (valid && rank == 0) s_wcnt[warp * RADIX + d] = cnt + __popc(peers);
+        if (valid && rank == 0) s_wcnt[warp * RADIX + d] = cnt + (info[i] >> 24);
         __syncwarp();
     }
     __syncthreads();
@@ -300,7 +310,10 @@ __global__ __launch_bounds__(RS_THREADS, 3) void k_rs_scatter(const uint32_t *__
 #pragma unroll
         for (int q = 0; q < PER; ++q) {
             const int d = tid * PER + q;
-            if (d < RADIX) s_tpre[d] = excl;
+            if (d < RADIX) {
+                s_tpre[d] = excl;
+                s_base[d] -= excl;    // output index = s_base[d] + (tile-local index)
+            }
             excl += local[q];
         }
     }
@@ -323,7 +336,7 @@ __global__ __launch_bounds__(RS_THREADS, 3) void k_rs_scatter(const uint32_t *__
         if (li < ntile) {
             const uint32_t k = s_keys[li];
             const unsigned d = (k >> shift) & MASK;
-            const uint32_t dest = s_base[d] + (uint32_t)li - s_tpre[d];
+            const uint32_t dest = s_base[d] + (uint32_t)li;
             kout[dest] = k;
             vout[dest] = s_vals[li];
         }

@@ -1,0 +1,348 @@
+// Window engine: pdb_sgd_epoch under a WINDOW schedule.
+//
+// When consecutive occurrences of a feature mostly lie far apart in the data
+// (ids drawn from many more features than one batch of concurrent examples
+// touches), almost every Read Constraint of Section 4.4 is already met by the
+// time an example runs: the previous writer finished long ago.  This engine
+// pays for the constraint only where it can bind:
+//
+//   * a position whose previous occurrence lies at least `near` positions
+//     back ("far") reads w_j from the plain fp32 array, once the example has
+//     seen the completion watermark pass that distance: every example below
+//     the watermark has finished and its writes are visible;
+//   * a position whose previous occurrence lies closer ("near", gate bit 30)
+//     takes the weight from that occurrence through a 64-bit record of
+//     feature j, bits(w_j) | tag << 32, as under READY (the read protocol of
+//     Section 5): one load both checks the tag and returns the weight.  The
+//     tag is the reader's occurrence rank plus an epoch stamp in bits 29-31,
+//     so records left by an earlier epoch never match and need no reset.
+//
+// Each position writes its new weight exactly once: into the record when its
+// next occurrence is near (gate bit 29; the near reader takes it from
+// there), else into w_j (read by a far successor, or final).  So w_j always
+// holds the weight of the latest writer whose successor is far, which is the
+// one a far reader needs; no position pays for both.
+//
+// Watermark: examples are taken in data order from a ticket counter, a
+// chunk of consecutive ones per warp.  Each worker warp keeps one progress
+// word: when it takes chunk c it publishes c (release, after a fence that
+// covers the weight stores of its earlier chunks), meaning "every chunk I
+// took before c is finished"; it publishes UINT_MAX when it runs out of
+// tickets.  The minimum over the warps is a chunk below which every chunk is
+// finished.  Block 0 of the grid does no examples: it sweeps the progress
+// words and publishes the first position of that chunk as `wpos` (release).
+// An example refreshes its view of `wpos` with one acquire load issued while
+// its ids and values are still in flight.
+//
+// Deadlock freedom: the oldest unfinished example waits for nothing -- its
+// near predecessors are finished, and its watermark condition is capped at
+// the first position of its own chunk, which the watermark reaches once all
+// earlier chunks are done and their warps have moved on.  Every wait,
+// including the sweeper's, is bounded by the timeout.
+#include <cuda_runtime.h>
+
+#include "common.cuh"
+
+using namespace pdb;
+
+namespace {
+
+__device__ __forceinline__ long long ld_acquire_s64(const long long *p)
+{
+    long long v;
+    asm volatile("ld.acquire.gpu.global.s64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
+    return v;
+}
+__device__ __forceinline__ unsigned ld_relaxed_u32(const unsigned *p)
+{
+    unsigned v;
+    asm volatile("ld.relaxed.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+__device__ __forceinline__ unsigned long long ld_rec(const unsigned long long *p)
+{
+    unsigned long long v;
+    asm volatile("ld.relaxed.gpu.global.b64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
+    return v;
+}
+__device__ __forceinline__ void st_rec(unsigned long long *p, float w, unsigned tag)
+{
+    const unsigned long long v = (unsigned long long)__float_as_uint(w) | ((unsigned long long)tag << 32);
+    asm volatile("st.relaxed.gpu.global.b64 [%0], %1;" ::"l"(p), "l"(v) : "memory");
+}
+__device__ __forceinline__ void fence_acq_rel() { asm volatile("fence.acq_rel.gpu;" ::: "memory"); }
+__device__ __forceinline__ void max_release(long long *p, long long v)
+{
+    asm volatile("red.release.gpu.global.max.s64 [%0], %1;" ::"l"(p), "l"(v) : "memory");
+}
+
+// gives up when the failure is elsewhere (status set) or the wait ran out
+__device__ __forceinline__ bool keep_waiting(unsigned &spins, uint64_t t0, int *status, uint64_t timeout)
+{
+    if ((++spins & 15u) != 0) return true;
+    if (read_status(status)) return false;
+    if (globaltimer() - t0 > timeout) {
+        set_status(status, PDB_ETIMEOUT);
+        return false;
+    }
+    return true;
+}
+
+// Waits until the watermark has reached `need` (positions) or gives up.
+// `known` holds this lane's last acquired watermark (it only grows).
+__device__ __noinline__ bool wait_watermark(const WindowCtl *ctl, long long need, long long &known, int *status,
+                                            uint64_t timeout)
+{
+    const uint64_t t0 = globaltimer();
+    unsigned spins = 0, nap = 64;
+    while (known < need) {
+        __nanosleep(nap);
+        nap = nap < 1024 ? 2 * nap : 1024;
+        known = ld_acquire_s64(&ctl->wpos);
+        if (known < need && !keep_waiting(spins, t0, status, timeout)) return false;
+    }
+    return true;
+}
+
+// Gathers this lane's weights: far ones from w (their watermark condition
+// already checked), near ones from the records, waiting for each wanted tag.
+template <int R>
+__device__ __forceinline__ bool gather_window(const float *w, const unsigned long long *rec, const int *j,
+                                              const uint32_t *g, unsigned stamp, float *wv, int lane, int k,
+                                              int *status, uint64_t timeout)
+{
+    unsigned pending = 0;
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+        wv[r] = 0.0f;
+        if (r * 32 + lane < k) {
+            if (g[r] & GATE_NEAR_PREV) {
+                const unsigned long long v = ld_rec(rec + j[r]);
+                wv[r] = __uint_as_float((unsigned)v);
+                if ((unsigned)(v >> 32) != ((g[r] & GATE_RANK) | stamp)) pending |= 1u << r;
+            } else {
+                wv[r] = __ldcg(w + j[r]);
+            }
+        }
+    }
+    if (pending == 0) return true;
+    const uint64_t t0 = globaltimer();
+    unsigned spins = 0, nap = 32;
+    while (pending) {
+        __nanosleep(nap);
+        nap = nap < 512 ? 2 * nap : 512;
+#pragma unroll
+        for (int r = 0; r < R; ++r)
+            if (pending & (1u << r)) {
+                const unsigned long long v = ld_rec(rec + j[r]);
+                if ((unsigned)(v >> 32) == ((g[r] & GATE_RANK) | stamp)) {
+                    wv[r] = __uint_as_float((unsigned)v);
+                    pending &= ~(1u << r);
+                }
+            }
+        if (pending && !keep_waiting(spins, t0, status, timeout)) return false;
+    }
+    return true;
+}
+
+// the new weight goes where the next occurrence will look for it
+__device__ __forceinline__ void publish(int j, uint32_t g, float nw, float *w, unsigned long long *rec,
+                                        unsigned stamp)
+{
+    if (g & GATE_NEAR_NEXT)
+        st_rec(rec + j, nw, ((g & GATE_RANK) + 1u) | stamp);
+    else
+        __stcg(w + j, nw);
+}
+
+// a previous occurrence that is not near: read from w after the watermark
+__device__ __forceinline__ bool is_far(uint32_t g) { return (g & GATE_RANK) != 0 && !(g & GATE_NEAR_PREV); }
+
+template <int R>
+__device__ __forceinline__ bool window_example(int t, int64_t floor_pos, const int64_t *__restrict__ row_ptr,
+                                               const int32_t *__restrict__ col, const float *__restrict__ val,
+                                               const float *__restrict__ y, const uint32_t *__restrict__ gate,
+                                               float *w, unsigned long long *rec, unsigned stamp,
+                                               const WindowCtl *ctl, int64_t near, int loss, float eta,
+                                               long long &known, int *status, uint64_t timeout)
+{
+    const int lane = threadIdx.x & 31;
+    const int64_t b = row_ptr[t];
+    const int k = (int)(row_ptr[t + 1] - b);
+    const float yt = y[t];
+    // a far previous occurrence sits at or before p - near (p < b + k) and
+    // before this example's chunk: below `need`
+    const long long need = (long long)min64(floor_pos, b + k - near);
+    if (k <= 32 * R) {
+        int j[R];
+        float x[R], wv[R];
+        uint32_t g[R];
+#pragma unroll
+        for (int r = 0; r < R; ++r) {
+            const int i = r * 32 + lane;
+            j[r] = i < k ? __ldcs(col + b + i) : 0;
+            x[r] = i < k ? (val ? __ldcs(val + b + i) : 1.0f) : 0.0f;
+            g[r] = i < k ? __ldcs(gate + b + i) : 0u;
+        }
+        // refresh the watermark while the loads above are in flight
+        if (known < need) known = ld_acquire_s64(&ctl->wpos);
+        bool far = false;
+#pragma unroll
+        for (int r = 0; r < R; ++r) far |= r * 32 + lane < k && is_far(g[r]);
+        bool ok = !far || known >= need || wait_watermark(ctl, need, known, status, timeout);
+        ok = ok && gather_window<R>(w, rec, j, g, stamp, wv, lane, k, status, timeout);
+        if (!__all_sync(FULL, ok)) return false;
+        float acc = 0.0f;
+#pragma unroll
+        for (int r = 0; r < R; ++r)
+            if (r * 32 + lane < k) acc = __fmaf_rn(wv[r], x[r], acc);
+        const float m = warp_combine(acc);
+        const float c = __fmul_rn(eta, dev_grad(loss, m, yt));
+#pragma unroll
+        for (int r = 0; r < R; ++r)
+            if (r * 32 + lane < k) publish(j[r], g[r], __fsub_rn(wv[r], __fmul_rn(c, x[r])), w, rec, stamp);
+        __syncwarp();   // the next example of the chunk may read these weights from another lane
+        return true;
+    }
+    // long example: gather element by element, then a second pass (no other
+    // example writes these features before this one does, so the second
+    // read of w or of a record returns the same weight)
+    if (known < need) known = ld_acquire_s64(&ctl->wpos);
+    float acc = 0.0f;
+    bool ok = true;
+    for (int i = lane; i < k && ok; i += 32) {
+        const int jj[1] = {col[b + i]};
+        const uint32_t gg[1] = {gate[b + i]};
+        float v1[1];
+        ok = !is_far(gg[0]) || known >= need || wait_watermark(ctl, need, known, status, timeout);
+        ok = ok && gather_window<1>(w, rec, jj, gg, stamp, v1, 0, 1, status, timeout);
+        if (ok) acc = __fmaf_rn(v1[0], val ? val[b + i] : 1.0f, acc);
+    }
+    if (!__all_sync(FULL, ok)) return false;
+    const float m = warp_combine(acc);
+    const float c = __fmul_rn(eta, dev_grad(loss, m, yt));
+    for (int i = lane; i < k; i += 32) {
+        const int jj = col[b + i];
+        const uint32_t gg = gate[b + i];
+        const float xx = val ? val[b + i] : 1.0f;
+        const float wo = (gg & GATE_NEAR_PREV) ? __uint_as_float((unsigned)ld_rec(rec + jj)) : __ldcg(w + jj);
+        publish(jj, gg, __fsub_rn(wo, __fmul_rn(c, xx)), w, rec, stamp);
+    }
+    __syncwarp();
+    return true;
+}
+
+// Block 0: sweep the worker warps' progress words until every chunk is
+// finished, publishing the watermark after each sweep.  Relaxed loads then
+// one fence: an acquire of all of them without serializing the loads.
+__device__ void sweep(int32_t n_rows, const int64_t *__restrict__ row_ptr, const unsigned *prog, int n_workers,
+                      unsigned n_chunks, int chunk, WindowCtl *ctl, int *status, uint64_t timeout)
+{
+    __shared__ unsigned s_min[WARPS];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    unsigned last = 0;
+    uint64_t t_last = globaltimer();
+    for (;;) {
+        unsigned m = 0xffffffffu;
+        for (int i = threadIdx.x; i < n_workers; i += THREADS) m = min(m, ld_relaxed_u32(prog + i));
+        fence_acq_rel();
+        for (int off = 16; off >= 1; off >>= 1) m = min(m, __shfl_xor_sync(FULL, m, off));
+        if (lane == 0) s_min[warp] = m;
+        __syncthreads();
+        unsigned wm = s_min[0];
+#pragma unroll
+        for (int q = 1; q < WARPS; ++q) wm = min(wm, s_min[q]);
+        wm = min(wm, n_chunks);
+        if (threadIdx.x == 0 && wm > last)
+            max_release(&ctl->wpos, (long long)row_ptr[min64(n_rows, (int64_t)wm * chunk)]);
+        if (wm >= n_chunks) return;
+        const uint64_t now = globaltimer();
+        if (wm > last) {
+            last = wm;
+            t_last = now;
+        }
+        const bool timed_out = now - t_last > timeout;
+        if (read_status(status) != 0 || timed_out) {
+            if (threadIdx.x == 0 && timed_out) set_status(status, PDB_ETIMEOUT);
+            return;
+        }
+        __syncthreads();     // s_min is rewritten by the next sweep
+        __nanosleep(256);
+    }
+}
+
+// this warp's progress word: every chunk it took before `value` is finished
+// and its weights are visible (fence by every lane, then one release store)
+__device__ __forceinline__ void publish_progress(unsigned *slot, unsigned value)
+{
+    fence_acq_rel();
+    __syncwarp();
+    if ((threadIdx.x & 31) == 0) st_release(slot, value);
+}
+
+template <int R>
+__global__ __launch_bounds__(THREADS) void k_sgd_window(int32_t n_rows, const int64_t *__restrict__ row_ptr,
+                                                        const int32_t *__restrict__ col,
+                                                        const float *__restrict__ val, const float *__restrict__ y,
+                                                        const uint32_t *__restrict__ gate, float *w,
+                                                        unsigned long long *rec, unsigned stamp, unsigned *prog,
+                                                        WindowCtl *ctl, int64_t near, int loss, float eta, int chunk,
+                                                        int *status, uint64_t timeout)
+{
+    if (read_status(status)) return;
+    const unsigned n_chunks = (unsigned)((n_rows + (int64_t)chunk - 1) / chunk);
+    const int n_workers = (gridDim.x - 1) * WARPS;
+    if (blockIdx.x == 0) {
+        sweep(n_rows, row_ptr, prog, n_workers, n_chunks, chunk, ctl, status, timeout);
+        return;
+    }
+    const int lane = threadIdx.x & 31;
+    unsigned *slot = prog + (blockIdx.x - 1) * WARPS + (threadIdx.x >> 5);
+    long long known = 0;
+    for (;;) {
+        unsigned long long tk = 0;
+        if (lane == 0) tk = atomicAdd(&ctl->ticket, (unsigned long long)chunk);
+        tk = __shfl_sync(FULL, tk, 0);
+        if (tk >= (unsigned long long)n_rows) {
+            publish_progress(slot, 0xffffffffu);
+            return;
+        }
+        publish_progress(slot, (unsigned)(tk / chunk));
+        const int t1 = (int)min64((int64_t)n_rows, (int64_t)tk + chunk);
+        const int64_t floor_pos = row_ptr[tk];
+        for (int t = (int)tk; t < t1; ++t)
+            if (!window_example<R>(t, floor_pos, row_ptr, col, val, y, gate, w, rec, stamp, ctl, near, loss, eta,
+                                   known, status, timeout))
+                return;
+    }
+}
+
+}  // namespace
+
+namespace pdb {
+
+int window_run(const pdb_csr *X, const float *y, const uint32_t *gate, float *w, unsigned long long *rec,
+               unsigned *epoch_count, unsigned *prog, int64_t prog_cap, WindowCtl *ctl, int64_t near, int loss,
+               float eta, int n_epochs, int width, const pdb_opts *opts, int *status, uint64_t timeout,
+               cudaStream_t s)
+{
+    const int32_t n = (int32_t)X->n_rows;
+    const int chunk = (opts && opts->ticket_chunk > 0) ? opts->ticket_chunk : 2;
+    auto kern = width == 2 ? k_sgd_window<2> : width == 4 ? k_sgd_window<4> : k_sgd_window<8>;
+    int grid = persistent_grid((const void *)kern, opts);
+    if (grid < 2) grid = 2;                         // the sweeper block plus at least one worker block
+    if ((int64_t)(grid - 1) * WARPS > prog_cap) return PDB_EFAULT;
+    for (int ep = 0; ep < n_epochs; ++ep) {
+        // record tags carry an epoch stamp 1..7 (bits 29-31), different in
+        // consecutive epochs of this schedule, so stale records never match
+        const unsigned stamp = (1u + (*epoch_count)++ % 7u) << 29;
+        cudaMemsetAsync(prog, 0, sizeof(unsigned) * (size_t)(grid - 1) * WARPS, s);
+        cudaMemsetAsync(ctl, 0, sizeof(WindowCtl), s);
+        kern<<<grid, THREADS, 0, s>>>(n, X->row_ptr, X->col, X->val, y, gate, w, rec, stamp, prog, ctl, near, loss,
+                                      eta, chunk, status, timeout);
+        note_launch();
+    }
+    return cudaPeekAtLastError() == cudaSuccess ? PDB_OK : PDB_ECUDA;
+}
+
+}  // namespace pdb

@@ -97,7 +97,17 @@ def _sgd(name, mode, opts=None):
     return w.cpu().numpy()
 
 
-MODES = {"levels": pdb.PDB_SCHED_LEVELS, "ready": pdb.PDB_SCHED_READY, "chain": pdb.PDB_SCHED_CHAIN}
+MODES = {"levels": pdb.PDB_SCHED_LEVELS, "ready": pdb.PDB_SCHED_READY, "chain": pdb.PDB_SCHED_CHAIN,
+         "window": pdb.PDB_SCHED_WINDOW}
+
+
+@pytest.fixture
+def near(monkeypatch):
+    # the conflict build reads PDB_NEAR at each call: small distances make most
+    # occurrence pairs "far", so small inputs run the watermark path
+    def set_near(v):
+        monkeypatch.setenv("PDB_NEAR", str(v))
+    return set_near
 
 
 @pytest.mark.parametrize("mode", list(MODES))
@@ -114,6 +124,40 @@ def test_sgd_weights(name, mode):
     ref = C.oracle_sgd(name)
     assert C.rel_err(got, ref) <= TOL
     assert np.array_equal(got, ref)       # same fp32 operation order on both sides
+
+
+@pytest.mark.parametrize("near_dist", [1, 7, 300, 5000])
+@pytest.mark.parametrize("name", ["tiny", "lowconflict-shape", "ragged-empty-rows", "zipf-shape", "long-rows",
+                                  "ctr-shape-binary", "one-feature-chain", "exp-saturation"])
+def test_window_watermark_path(name, near_dist, near):
+    # WINDOW with most pairs far (watermark) or a mix of far and near pairs
+    near(near_dist)
+    got = _sgd(name, pdb.PDB_SCHED_WINDOW, opts=dict(wait_timeout_s=20.0))
+    ref = C.oracle_sgd(name)
+    assert C.rel_err(got, ref) <= TOL
+    assert np.array_equal(got, ref)
+
+
+def test_window_chunk_sizes(near):
+    near(50)
+    name = "lowconflict-shape"
+    ref = C.oracle_sgd(name)
+    for chunk in (1, 3, 16):
+        got = _sgd(name, pdb.PDB_SCHED_WINDOW, opts=dict(ticket_chunk=chunk, blocks_per_sm=1))
+        assert np.array_equal(got, ref), chunk
+
+
+def test_auto_picks_window_when_near_pairs_are_rare(near):
+    near(64)
+    name = "lowconflict-shape"
+    p, X, y = _gpu(name)
+    c = pdb.pdb_build_conflicts(X)
+    s = pdb.pdb_schedule_build(c, pdb.PDB_SCHED_AUTO)
+    assert pdb.pdb_get_stats(c, s)["sched_mode"] == pdb.PDB_SCHED_WINDOW
+    w = torch.zeros(p.n_cols, dtype=torch.float32, device="cuda")
+    pdb.pdb_sgd_epoch(X, y, c, s, w, p.loss, p.eta, p.epochs)
+    pdb.check_status(c)
+    assert np.array_equal(w.cpu().numpy(), C.oracle_sgd(name))
 
 
 @pytest.mark.parametrize("name,expect", [("tiny", "ready"), ("lowconflict-shape", "ready"),
@@ -135,7 +179,7 @@ def test_sgd_small_grid_and_repeat_calls():
     name = "zipf-shape"
     p, X, y = _gpu(name)
     c = pdb.pdb_build_conflicts(X)
-    for mode in (pdb.PDB_SCHED_LEVELS, pdb.PDB_SCHED_READY, pdb.PDB_SCHED_CHAIN):
+    for mode in (pdb.PDB_SCHED_LEVELS, pdb.PDB_SCHED_READY, pdb.PDB_SCHED_CHAIN, pdb.PDB_SCHED_WINDOW):
         s = pdb.pdb_schedule_build(c, mode)
         w = torch.zeros(p.n_cols, dtype=torch.float32, device="cuda")
         pdb.pdb_sgd_epoch(X, y, c, s, w, p.loss, p.eta, 1, opts=dict(blocks_per_sm=1))
@@ -200,3 +244,25 @@ def test_wait_timeout_is_reported_not_hung():
     assert pdb.pdb_status(c) == pdb.PDB_ETIMEOUT
     t = torch.arange(10, device="cuda").sum().item()     # the device still works
     assert t == 45
+
+
+@pytest.mark.parametrize("near_dist", [1 << 22, 1])
+def test_window_wait_timeout_is_reported_not_hung(near_dist, near):
+    # WINDOW: one position waits for an iteration number nobody publishes, so
+    # its chunk never finishes; with all pairs far (near_dist 1) every later
+    # example also waits on the stalled watermark.  The waits give up after
+    # the limit, the kernel returns and the status says so.
+    near(near_dist)
+    name = "tiny"
+    p, X, y = _gpu(name)
+    c = pdb.pdb_build_conflicts(X)
+    s = pdb.pdb_schedule_build(c, pdb.PDB_SCHED_WINDOW)
+    pdb.check_status(c)
+    gate_ptr = pdb.pdb_schedule_ready(s)["gate"]
+    pos = int(p.row_ptr[5])
+    poison = torch.tensor([12345 | (1 << 30)], dtype=torch.int32, device="cuda")   # rank 12345, near previous
+    pdb.pdb_memcpy(gate_ptr + 4 * pos, poison.data_ptr(), 4)
+    w = torch.zeros(p.n_cols, dtype=torch.float32, device="cuda")
+    pdb.pdb_sgd_epoch(X, y, c, s, w, p.loss, p.eta, 1, opts=dict(wait_timeout_s=0.2))
+    assert pdb.pdb_status(c) == pdb.PDB_ETIMEOUT
+    assert torch.arange(10, device="cuda").sum().item() == 45
