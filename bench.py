@@ -386,15 +386,22 @@ def run_e2e(args, p, mode, pdb, torch, world):
     h2d = sum(t.numel() * t.element_size() for t in (h_row, h_col, h_val, h_y, h_w0) if t is not None)
     d2h = h_w.numel() * h_w.element_size()
 
+    side = torch.cuda.Stream()
+
     def step():
+        # the conflict build needs only row_ptr and col: the values, labels
+        # and initial weights travel on a second stream while it runs
         d_row.copy_(h_row, non_blocking=True)
         d_col.copy_(h_col, non_blocking=True)
-        if d_val is not None:
-            d_val.copy_(h_val, non_blocking=True)
-        d_y.copy_(h_y, non_blocking=True)
-        d_w.copy_(h_w0, non_blocking=True)
+        side.wait_stream(stream)
+        with torch.cuda.stream(side):
+            if d_val is not None:
+                d_val.copy_(h_val, non_blocking=True)
+            d_y.copy_(h_y, non_blocking=True)
+            d_w.copy_(h_w0, non_blocking=True)
         c = pdb.pdb_build_conflicts(X, stream)
         s = pdb.pdb_schedule_build(c, mode, stream)
+        stream.wait_stream(side)
         pdb.pdb_sgd_epoch(X, d_y, c, s, d_w, p.loss, p.eta, p.epochs,
                           opts=dict(ticket_chunk=args.ticket_chunk, blocks_per_sm=args.blocks_per_sm), stream=stream)
         h_w.copy_(d_w, non_blocking=True)

@@ -41,11 +41,11 @@ __global__ void k_validate_rows(const int64_t *__restrict__ row_ptr, int64_t n_r
     }
 }
 
-// One warp per example: ids in [0, n_cols) (else ERANGE), row_of, the
-// longest row, and whether the row's ids are strictly increasing (a row
-// that is cannot hold a repeated id; only unsorted rows need the slot check).
+// One warp per example: ids in [0, n_cols) (else ERANGE), the longest row,
+// and whether the row's ids are strictly increasing (a row that is cannot
+// hold a repeated id; only unsorted rows need the slot check).
 __global__ void k_rows_scan(const int64_t *__restrict__ row_ptr, const int32_t *__restrict__ col, int64_t n_rows,
-                            int64_t n_cols, int32_t *__restrict__ row_of, int *info)
+                            int64_t n_cols, int *info)
 {
     if (read_status(info)) return;
     const int lane = threadIdx.x & 31;
@@ -60,12 +60,39 @@ __global__ void k_rows_scan(const int64_t *__restrict__ row_ptr, const int32_t *
             int32_t j = col[p];
             bad |= j < 0 || (int64_t)j >= n_cols;
             unsorted |= p > b && col[p - 1] >= j;
-            row_of[p] = (int32_t)t;
         }
     }
     if (__any_sync(FULL, bad) && lane == 0) set_status(info, PDB_ERANGE);
     if (__any_sync(FULL, unsorted) && lane == 0) atomicExch(info + INFO_UNSORTED, 1);
     if (lane == 0 && longest > 0) atomicMax(info + INFO_MAX_ROW, longest);
+}
+
+// example of each position (built on first use: LEVELS, CHAIN, BSP)
+__global__ void k_row_of(const int64_t *__restrict__ row_ptr, int64_t n_rows, int32_t *__restrict__ row_of,
+                         const int *info)
+{
+    if (read_status(info)) return;
+    const int lane = threadIdx.x & 31;
+    const int64_t gw = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    for (int64_t t = gw; t < n_rows; t += nw) {
+        const int64_t b = row_ptr[t], e = row_ptr[t + 1];
+        for (int64_t p = b + lane; p < e; p += 32) row_of[p] = (int32_t)t;
+    }
+}
+
+// the example holding position p: the last t with row_ptr[t] <= p
+__device__ __forceinline__ int64_t find_row(const int64_t *__restrict__ row_ptr, int64_t n_rows, int64_t p)
+{
+    int64_t lo = 0, hi = n_rows - 1;
+    while (lo < hi) {
+        const int64_t mid = (lo + hi + 1) >> 1;
+        if (row_ptr[mid] <= p)
+            lo = mid;
+        else
+            hi = mid - 1;
+    }
+    return lo;
 }
 
 // Slot order: the gate word of every slot, rank | last-occurrence bit, the
@@ -75,7 +102,8 @@ __global__ void k_rows_scan(const int64_t *__restrict__ row_ptr, const int32_t *
 // scattered 4-byte store per slot) or, for large inputs, in slot order
 // (gsort[s]) for the partitioned scatter below.
 __global__ void k_slots(const uint32_t *__restrict__ skey, const int32_t *__restrict__ spos, int64_t nnz,
-                        const int64_t *__restrict__ feat_ptr, const int32_t *__restrict__ row_of, int64_t near,
+                        const int64_t *__restrict__ feat_ptr, const int64_t *__restrict__ row_ptr, int64_t n_rows,
+                        int64_t near,
                         uint32_t *__restrict__ gate, uint32_t *__restrict__ gsort, int *info)
 {
     if (read_status(info)) return;
@@ -98,7 +126,7 @@ __global__ void k_slots(const uint32_t *__restrict__ skey, const int32_t *__rest
         else
             gate[p] = g;
         if (last) longest = max(longest, (int)(r + 1));
-        if (check_dup && r > 0) dup |= row_of[spos[s - 1]] == row_of[p];
+        if (check_dup && r > 0) dup |= find_row(row_ptr, n_rows, spos[s - 1]) == find_row(row_ptr, n_rows, p);
     }
     for (int off = 16; off >= 1; off >>= 1) {
         longest = max(longest, __shfl_xor_sync(FULL, longest, off));
@@ -274,11 +302,37 @@ int check_csr(const pdb_csr *X)
     return PDB_OK;
 }
 
+// Callers synchronize the device first.  The arrays go back to the
+// stream-ordered pool (kept, not returned to the driver), so freeing costs no
+// device-wide synchronization and the next build reuses the memory.
 void free_ptrs(std::initializer_list<void *> ptrs)
 {
     for (void *p : ptrs)
-        if (p) cudaFree(p);
+        if (p) cudaFreeAsync(p, 0);
 }
+
+}  // namespace
+
+namespace pdb {
+
+// row_of of every position (idempotent; enqueued on s)
+int ensure_row_of(pdb_conflicts *c, cudaStream_t s)
+{
+    if (c->row_of) return PDB_OK;
+    int32_t *row_of = nullptr;
+    int rc = alloc((void **)&row_of, sizeof(int32_t) * std::max<int64_t>(c->nnz, 1), s);
+    if (rc != PDB_OK) return rc;
+    if (c->n_rows > 0) {
+        k_row_of<<<grid_1d(c->n_rows * 32), 256, 0, s>>>(c->row_ptr, c->n_rows, row_of, c->status);
+        note_launch();
+    }
+    c->row_of = row_of;
+    return cudaPeekAtLastError() == cudaSuccess ? PDB_OK : PDB_ECUDA;
+}
+
+}  // namespace pdb
+
+namespace {
 
 // prev/next/rank of every position (idempotent; enqueued on s)
 int materialize_chains(pdb_conflicts *c, cudaStream_t s)
@@ -387,7 +441,6 @@ int pdb_build_conflicts(const pdb_csr *X, pdb_conflicts **out, void *stream)
     rc = alloc((void **)&c->info, sizeof(int) * INFO_WORDS, s);
     rc = rc ? rc : alloc((void **)&c->csc_pos, sizeof(int32_t) * nnz, s);
     rc = rc ? rc : alloc((void **)&c->gate, sizeof(uint32_t) * nnz, s);
-    rc = rc ? rc : alloc((void **)&c->row_of, sizeof(int32_t) * nnz, s);
     rc = rc ? rc : alloc((void **)&c->feat_ptr, sizeof(int64_t) * (F + 1), s);
     uint32_t *skey = nullptr, *tkey = nullptr;
     int32_t *tval = nullptr;
@@ -400,7 +453,7 @@ int pdb_build_conflicts(const pdb_csr *X, pdb_conflicts **out, void *stream)
         k_validate_rows<<<grid_1d(N + 1), 256, 0, s>>>(X->row_ptr, N, nnz, c->info);
         note_launch();
         if (N > 0) {
-            k_rows_scan<<<grid_1d(N * 32), 256, 0, s>>>(X->row_ptr, X->col, N, F, c->row_of, c->info);
+            k_rows_scan<<<grid_1d(N * 32), 256, 0, s>>>(X->row_ptr, X->col, N, F, c->info);
             note_launch();
         }
         // (feature, position) pairs sorted by feature, stable: positions stay in data order
@@ -414,7 +467,7 @@ int pdb_build_conflicts(const pdb_csr *X, pdb_conflicts **out, void *stream)
         // order (k_scatter_block)
         const int pbits = bits_for(nnz - 1);
         const bool partition = pbits > 22;
-        k_slots<<<grid_1d(nnz), 256, 0, s>>>(skey, c->csc_pos, nnz, c->feat_ptr, c->row_of, c->near, c->gate,
+        k_slots<<<grid_1d(nnz), 256, 0, s>>>(skey, c->csc_pos, nnz, c->feat_ptr, X->row_ptr, N, c->near, c->gate,
                                              partition ? (uint32_t *)tval : nullptr, c->info);
         note_launch();
         if (partition) {
@@ -556,9 +609,11 @@ int pdb_schedule_build(const pdb_conflicts *c, pdb_sched_mode mode, pdb_schedule
     } else if (mode == PDB_SCHED_CHAIN) {
         rc = rc ? rc : materialize_chains(cm, s);
         rc = rc ? rc : alloc((void **)&h->link, sizeof(uint32_t) * nnz, s);
+        rc = rc ? rc : ensure_row_of(cm, s);
         rc = rc ? rc : chain_schedule(c->prev, c->next, c->row_of, c->row_ptr, nnz, h->link, c->status, s);
     } else {
         rc = rc ? rc : materialize_chains(cm, s);
+        rc = rc ? rc : ensure_row_of(cm, s);
         if (rc == PDB_OK && !cm->npred) {
             rc = alloc((void **)&cm->npred, sizeof(int32_t) * N, s);
             if (rc == PDB_OK && N > 0) {

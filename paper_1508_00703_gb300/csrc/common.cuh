@@ -203,6 +203,8 @@ struct WindowCtl {
     long long wpos;             // every example starting below this position has finished
 };
 
+int ensure_row_of(pdb_conflicts *c, cudaStream_t s);   // builds c->row_of on first use (stream-ordered)
+
 int window_run(const pdb_csr *X, const float *y, const uint32_t *gate, float *w, unsigned long long *rec,
                unsigned *epoch_count, unsigned *prog, int64_t prog_cap, WindowCtl *ctl, int64_t near, int loss,
                float eta, int n_epochs, int width, const pdb_opts *opts, int *status, uint64_t timeout,
@@ -221,7 +223,7 @@ struct pdb_conflicts {
     int64_t *feat_ptr;       // [F+1]
     uint32_t *gate;          // per position: occurrence rank and flags (GATE_* below)
     int64_t near;            // distance (positions) under which an occurrence pair counts as near
-    int32_t *row_of;         // example of each position
+    int32_t *row_of;         // example of each position (built on first use)
     int32_t *prev, *next, *rank;  // materialized from the above on first request
     int32_t *npred;          // per example: occurrences with an earlier occurrence (LEVELS)
     int *info;               // device: [0] status, [1] max chain, [2] longest row, [3] any unsorted row,

@@ -479,7 +479,8 @@ int pdb_bsp_epoch(const pdb_csr *X, const float *y, const pdb_conflicts *c, floa
         rc = rc ? rc : alloc((void **)&bar, sizeof(GridBarrier), s);
         if (rc == PDB_OK) {
             cudaMemsetAsync(bar, 0, sizeof(GridBarrier), s);
-            if (nnz > 0) {
+            if (nnz > 0) rc = ensure_row_of(cm, s);
+            if (rc == PDB_OK && nnz > 0) {
                 k_bsp_keys<<<grid_1d(nnz), 256, 0, s>>>(c->csc_pos, c->row_of, nnz, batch, key, cm->status); note_launch();
                 // stable by batch: inside a batch the feature-major CSC order survives
                 rc = radix_sort(key, c->csc_pos, skey, bpos, tkey, tval, nnz, bits_for(n_batches - 1), cm->status, s);

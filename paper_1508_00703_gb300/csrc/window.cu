@@ -25,11 +25,13 @@
 //
 // Watermark: examples are taken in data order from a ticket counter, a
 // chunk of consecutive ones per warp.  Each worker warp keeps one progress
-// word: when it takes chunk c it publishes c (release, after a fence that
-// covers the weight stores of its earlier chunks), meaning "every chunk I
-// took before c is finished"; it publishes UINT_MAX when it runs out of
-// tickets.  The minimum over the warps is a chunk below which every chunk is
-// finished.  Block 0 of the grid does no examples: it sweeps the progress
+// word: once it has taken chunk c (and issued the loads of its first
+// example) it publishes c (release, after a fence that covers the weight
+// stores of its earlier chunks), meaning "every chunk I took before c is
+// finished"; it publishes UINT_MAX when it runs out of tickets.  Until then
+// the word still holds the previous chunk, which is only more conservative.
+// The minimum over the warps is a chunk below which every chunk is finished.
+// Block 0 of the grid does no examples: it sweeps the progress
 // words and publishes the first position of that chunk as `wpos` (release).
 // An example refreshes its view of `wpos` with one acquire load issued while
 // its ids and values are still in flight.
@@ -158,13 +160,27 @@ __device__ __forceinline__ void publish(int j, uint32_t g, float nw, float *w, u
 // a previous occurrence that is not near: read from w after the watermark
 __device__ __forceinline__ bool is_far(uint32_t g) { return (g & GATE_RANK) != 0 && !(g & GATE_NEAR_PREV); }
 
+// this warp's progress word: every chunk it took before `value` is finished
+// and its weights are visible (fence by every lane, then one release store)
+__device__ __forceinline__ void publish_progress(unsigned *slot, unsigned value)
+{
+    fence_acq_rel();
+    __syncwarp();
+    if ((threadIdx.x & 31) == 0) st_release(slot, value);
+}
+
+// One example.  The first example of a chunk publishes the warp's progress
+// (slot != nullptr) right after issuing its ids and values: the fence then
+// waits for the earlier chunk's weight stores while those loads are in
+// flight anyway.
 template <int R>
 __device__ __forceinline__ bool window_example(int t, int64_t floor_pos, const int64_t *__restrict__ row_ptr,
                                                const int32_t *__restrict__ col, const float *__restrict__ val,
                                                const float *__restrict__ y, const uint32_t *__restrict__ gate,
                                                float *w, unsigned long long *rec, unsigned stamp,
                                                const WindowCtl *ctl, int64_t near, int loss, float eta,
-                                               long long &known, int *status, uint64_t timeout)
+                                               long long &known, unsigned *slot, unsigned progress, int *status,
+                                               uint64_t timeout)
 {
     const int lane = threadIdx.x & 31;
     const int64_t b = row_ptr[t];
@@ -184,6 +200,7 @@ __device__ __forceinline__ bool window_example(int t, int64_t floor_pos, const i
             x[r] = i < k ? (val ? __ldcs(val + b + i) : 1.0f) : 0.0f;
             g[r] = i < k ? __ldcs(gate + b + i) : 0u;
         }
+        if (slot) publish_progress(slot, progress);
         // refresh the watermark while the loads above are in flight
         if (known < need) known = ld_acquire_s64(&ctl->wpos);
         bool far = false;
@@ -207,6 +224,7 @@ __device__ __forceinline__ bool window_example(int t, int64_t floor_pos, const i
     // long example: gather element by element, then a second pass (no other
     // example writes these features before this one does, so the second
     // read of w or of a record returns the same weight)
+    if (slot) publish_progress(slot, progress);
     if (known < need) known = ld_acquire_s64(&ctl->wpos);
     float acc = 0.0f;
     bool ok = true;
@@ -271,15 +289,6 @@ __device__ void sweep(int32_t n_rows, const int64_t *__restrict__ row_ptr, const
     }
 }
 
-// this warp's progress word: every chunk it took before `value` is finished
-// and its weights are visible (fence by every lane, then one release store)
-__device__ __forceinline__ void publish_progress(unsigned *slot, unsigned value)
-{
-    fence_acq_rel();
-    __syncwarp();
-    if ((threadIdx.x & 31) == 0) st_release(slot, value);
-}
-
 template <int R>
 __global__ __launch_bounds__(THREADS) void k_sgd_window(int32_t n_rows, const int64_t *__restrict__ row_ptr,
                                                         const int32_t *__restrict__ col,
@@ -307,12 +316,11 @@ __global__ __launch_bounds__(THREADS) void k_sgd_window(int32_t n_rows, const in
             publish_progress(slot, 0xffffffffu);
             return;
         }
-        publish_progress(slot, (unsigned)(tk / chunk));
         const int t1 = (int)min64((int64_t)n_rows, (int64_t)tk + chunk);
         const int64_t floor_pos = row_ptr[tk];
         for (int t = (int)tk; t < t1; ++t)
             if (!window_example<R>(t, floor_pos, row_ptr, col, val, y, gate, w, rec, stamp, ctl, near, loss, eta,
-                                   known, status, timeout))
+                                   known, t == (int)tk ? slot : nullptr, (unsigned)(tk / chunk), status, timeout))
                 return;
     }
 }
