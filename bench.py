@@ -49,6 +49,8 @@ def parse_args(argv=None):
     ap.add_argument("--rows", type=int, default=None, help="override the workload's example count")
     ap.add_argument("--ticket-chunk", type=int, default=0, help="READY engine: examples per ticket (0 = default)")
     ap.add_argument("--blocks-per-sm", type=int, default=0)
+    ap.add_argument("--bsp", type=int, default=0,
+                    help="time pdb_bsp_epoch with this mini-batch instead of pdb_sgd_epoch (-1: the workload's own)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=10.0, help="target length of the CPU oracle sample")
@@ -287,9 +289,14 @@ def run_ours(args, rank, world, local_rank):
     stream = torch.cuda.current_stream()
     opts = dict(ticket_chunk=args.ticket_chunk, blocks_per_sm=args.blocks_per_sm)
 
+    batch = (p.bsp_batch or 4096) if args.bsp < 0 else args.bsp
+
     def step():
         w.zero_()
         c = pdb.pdb_build_conflicts(X, stream)
+        if batch:
+            pdb.pdb_bsp_epoch(X, y, c, w, p.loss, p.eta, batch, E, opts=opts, stream=stream)
+            return c, None
         s = pdb.pdb_schedule_build(c, mode, stream)
         pdb.pdb_sgd_epoch(X, y, c, s, w, p.loss, p.eta, E, opts=opts, stream=stream)
         return c, s
@@ -325,8 +332,8 @@ def run_ours(args, rank, world, local_rank):
     pdb.check_status(c, stream)
     del c, s
 
-    ms_sgd = statistics.median(ph["ms_sgd"] for ph in phases)
-    ms_kern = statistics.median(ph["ms_sgd_kernels"] for ph in phases)
+    ms_sgd = statistics.median(ph["ms_bsp" if batch else "ms_sgd"] for ph in phases)
+    ms_kern = statistics.median(ph["ms_bsp" if batch else "ms_sgd_kernels"] for ph in phases)
     ms_build = statistics.median(ph["ms_build"] for ph in phases)
     ms_sched = statistics.median(ph["ms_schedule"] for ph in phases)
     peak, peak_kind = measured_peak_hbm()
@@ -334,7 +341,7 @@ def run_ours(args, rank, world, local_rank):
     sgd_launch_ms = ms_kern / E
     sgd_gbs = sgd_bytes_per_launch / (sgd_launch_ms / 1e3) / 1e9
     resolved = int(phases[0]["sched_mode"])
-    kname = {pdb.PDB_SCHED_READY: "k_sgd_ready", pdb.PDB_SCHED_LEVELS: "k_sgd_levels",
+    kname = {pdb.PDB_SCHED_READY: "k_sgd_ready", pdb.PDB_SCHED_LEVELS: "k_sgd_levels", -1: "k_bsp",
              pdb.PDB_SCHED_CHAIN: "k_sgd_chain", pdb.PDB_SCHED_WINDOW: "k_sgd_window"}[resolved]
     roofline = {"kernel": kname,
                 "bound": "hbm", "achieved": round(sgd_gbs, 1), "peak": peak, "unit": "GB/s",
@@ -347,19 +354,26 @@ def run_ours(args, rank, world, local_rank):
         "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f32", "data": "synthetic (seeded generator, no dataset)",
         "config": dict(workload_config(args.workload, p,
+                                       f"bsp, mini-batch {batch}" if batch else
                                        {0: "levels", 1: "ready", 2: "chain", 4: "window"}[resolved]
                                        + (" (auto)" if args.mode == "auto" else "")),
                        parallelism=f"replicas{world}" if world > 1 else "single GPU",
                        ticket_chunk=args.ticket_chunk or 2),
         "roofline": roofline,
-        "phases_ms": {"build_conflicts": ms_build, "schedule": ms_sched, "sgd_all_epochs": ms_sgd,
-                      "sgd_update_kernels": ms_kern},
+        "phases_ms": ({"build_conflicts": ms_build, "bsp_all_epochs": ms_sgd} if batch else
+                      {"build_conflicts": ms_build, "schedule": ms_sched, "sgd_all_epochs": ms_sgd,
+                       "sgd_update_kernels": ms_kern}),
         "sgd_only": {"value": units / (ms_sgd / 1e3), "unit": UNIT},
         "gpu_launches": int(launches),
         "clocks": clk.summary(),
     }
 
-    if not args.no_e2e:
+    if batch:
+        roofline["kernel"] = "k_bsp (whole pdb_bsp_epoch call per epoch: batch sort, gather, cooperative kernel)"
+        result["metric"] = METRIC.replace("serially-equivalent sparse SGD", f"BSP mini-batch ({batch}) SGD")
+        del result["sgd_only"]
+        result["bsp_only"] = {"value": units / (ms_sgd / 1e3), "unit": UNIT}
+    if not args.no_e2e and not batch:
         result["e2e"] = run_e2e(args, p, mode, pdb, torch, world)
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         result["cpu_baseline"] = cpu_baseline(p, args.cpu_seconds)

@@ -13,10 +13,15 @@
 //                multiply-adds, then the xor-shuffle combine), and pushes
 //                each new weight whose next occurrence lies in one of the
 //                next D examples straight into that example's weight slot;
-//   warps 1-3,5-7 prefetch with cp.async (row bounds 7 steps ahead; ids,
+//   warps 1-3, 5 prefetch one example of a step each with cp.async (ids,
 //                values, labels and link words 4 steps ahead; the weights
-//                nobody will push 2 steps ahead) and write the new weights of
-//                the previous step through to global memory.
+//                nobody will push 2 steps ahead), lanes striding over the
+//                example's elements;
+//   warps 6, 7   write the new weights of the previous step that are not
+//                pushed through to global memory, and copy row bounds 7
+//                steps ahead;
+//   warp 4       only joins the barriers: warps map to the SM's four
+//                schedulers by index mod 4, and warp 0 keeps its own.
 //
 // A pipeline step handles G = 4 consecutive examples, so the fixed cost of a
 // step (barrier, copy bookkeeping) is shared by four hops.
@@ -44,11 +49,6 @@ constexpr int CH_SLOTS = 32;                // example slots (power of two, > (C
 constexpr int CH_MAXK = 256;                // longest example this engine takes
 constexpr int CH_RP = 64;                   // row_ptr ring (power of two, > (CH_L + 2) * CH_G + 1)
 constexpr int CH_THREADS = 256;
-// Warps are spread over the SM's four schedulers by warp index mod 4, so
-// warp 4 would compete with the computing warp 0 for issue slots: it only
-// joins the barriers.  Warps 1-3 and 5-7 prefetch.
-constexpr int CH_PF = CH_THREADS - 64;      // prefetching threads
-constexpr int CH_PER = (CH_G * CH_MAXK + CH_PF - 1) / CH_PF;   // positions per prefetching thread per step
 // link word of a position: bit 31 = its weight will be pushed by an earlier
 // example (skip the gather); bit 30 = push the new weight to the next
 // occurrence, which is element (bits 0..15) of the example (bits 16..23)
@@ -59,15 +59,48 @@ static_assert(CH_SLOTS > (CH_DS + 2) * CH_G && CH_RP > (CH_L + 2) * CH_G + 1, "r
 static_assert(CH_D < 256 && CH_MAXK <= 65536, "link word fields");
 static_assert((CH_G & (CH_G - 1)) == 0, "examples per step must be a power of two");
 
+// ids, values and link words are copied in 16-byte pieces from the aligned
+// element before the example's first one: element i sits at index off + i,
+// off = (first position) mod 4 (0 when an input array is not 16-byte aligned)
+constexpr int CH_ROW = CH_MAXK + 4;
 struct ChainSmem {
-    int32_t col[CH_SLOTS][CH_MAXK];
-    float val[CH_SLOTS][CH_MAXK];
-    uint32_t link[CH_SLOTS][CH_MAXK];
+    int32_t col[CH_SLOTS][CH_ROW];
+    float val[CH_SLOTS][CH_ROW];
+    uint32_t link[CH_SLOTS][CH_ROW];
     float wp[CH_SLOTS][CH_MAXK];    // weight each element reads (gathered or pushed)
-    float out[CH_SLOTS][CH_MAXK];   // weight each element writes
+    float out[CH_SLOTS][CH_MAXK];   // weight of the elements whose next occurrence is not pushed
     int64_t rp[CH_RP];
     float y[CH_SLOTS];
+    __align__(16) float part[32];   // the compute warp's 32 partial sums
 };
+
+// The xor-butterfly combine of warp_combine (for off = 16, 8, 4, 2, 1 every
+// lane adds the partial of lane ^ off), evaluated from shared memory: every
+// lane reads the 32 partials and adds them in the same tree -- level by
+// level, partial l plus partial l + half -- which is the value lane 0 ends
+// with after the shuffles (fp32 addition is commutative, so every lane of
+// the shuffle version holds it too).  Two shared-memory round trips instead
+// of five dependent shuffles.
+__device__ __forceinline__ float combine_smem(float a, float *part)
+{
+    part[threadIdx.x & 31] = a;
+    __syncwarp();
+    float v[32];
+    const float4 *p4 = reinterpret_cast<const float4 *>(part);
+#pragma unroll
+    for (int q = 0; q < 8; ++q) {
+        const float4 f = p4[q];
+        v[4 * q] = f.x;
+        v[4 * q + 1] = f.y;
+        v[4 * q + 2] = f.z;
+        v[4 * q + 3] = f.w;
+    }
+#pragma unroll
+    for (int half = 16; half >= 1; half >>= 1)
+#pragma unroll
+        for (int l = 0; l < half; ++l) v[l] = __fadd_rn(v[l], v[l + half]);
+    return v[0];
+}
 
 __device__ __forceinline__ void cp4(void *smem_dst, const void *gsrc)
 {
@@ -79,37 +112,38 @@ __device__ __forceinline__ void cp8(void *smem_dst, const void *gsrc)
     const unsigned d = (unsigned)__cvta_generic_to_shared(smem_dst);
     asm volatile("cp.async.ca.shared.global [%0], [%1], 8;" ::"r"(d), "l"(gsrc) : "memory");
 }
+__device__ __forceinline__ void cp16(void *smem_dst, const void *gsrc)
+{
+    const unsigned d = (unsigned)__cvta_generic_to_shared(smem_dst);
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(d), "l"(gsrc) : "memory");
+}
+// copies elements [a0, b + k) of a 4-byte array into dst[0 ..): with vec
+// (every source array 16-byte aligned) in 16-byte pieces from the aligned
+// a0 = b - off up to the last aligned position and then the tail one element
+// at a time; without, all of it one element at a time (off = 0)
+__device__ __forceinline__ void cp_row(void *dst, const void *src, int64_t b, int k, int off, bool vec, int lane)
+{
+    const int64_t a0 = b - off;
+    const int64_t a1 = vec ? ((b + k) & ~(int64_t)3) : a0;
+    const int n16 = a1 > a0 ? (int)((a1 - a0) >> 2) : 0;
+    for (int c = lane; c < n16; c += 32)
+        cp16((uint32_t *)dst + 4 * c, (const uint32_t *)src + a0 + 4 * c);
+    for (int64_t e = (a1 > b ? a1 : b) + lane; e < b + k; e += 32)
+        cp4((uint32_t *)dst + (e - a0), (const uint32_t *)src + e);
+}
 __device__ __forceinline__ void cp_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
 __device__ __forceinline__ void cp_wait_b() { asm volatile("cp.async.wait_group %0;" ::"n"(CH_BS - 1) : "memory"); }
 __device__ __forceinline__ void cp_wait_all() { asm volatile("cp.async.wait_group 0;" ::: "memory"); }
 
-// The positions of the CH_G examples of step t are contiguous: [rp[t*G], rp[t*G+G]).
-// Element e of that range belongs to example r (found among the G bounds) at index i.
-struct StepRange {
-    int64_t b0;
-    int total;
-    int64_t bound[CH_G + 1];
-};
-
-__device__ __forceinline__ bool step_range(const ChainSmem &S, int t, int N, StepRange &R)
+// bounds [b, b + k) of example r from the row_ptr ring (false outside
+// 0..N-1) and the offset of its elements in the 16-byte-copied rows
+__device__ __forceinline__ bool row_bounds(const ChainSmem &S, int r, int N, bool vec, int64_t &b, int &k, int &off)
 {
-    const int r0 = t * CH_G;
-    if (t < 0 || r0 >= N) return false;
-#pragma unroll
-    for (int j = 0; j <= CH_G; ++j) R.bound[j] = S.rp[min(r0 + j, N) & (CH_RP - 1)];
-    R.b0 = R.bound[0];
-    R.total = (int)(R.bound[CH_G] - R.b0);
+    if (r < 0 || r >= N) return false;
+    b = S.rp[r & (CH_RP - 1)];
+    k = (int)(S.rp[(r + 1) & (CH_RP - 1)] - b);
+    off = vec ? (int)(b & 3) : 0;
     return true;
-}
-
-__device__ __forceinline__ void locate(const StepRange &R, int t, int e, int &row, int &i)
-{
-    const int64_t pos = R.b0 + e;
-    int j = 0;
-#pragma unroll
-    for (int q = 1; q < CH_G; ++q) j += pos >= R.bound[q];
-    row = t * CH_G + j;
-    i = (int)(pos - R.bound[j]);
 }
 
 template <int R>
@@ -118,95 +152,81 @@ __global__ __launch_bounds__(CH_THREADS, 1) void k_sgd_chain(int32_t n_rows, con
                                                              const float *__restrict__ val,
                                                              const float *__restrict__ y,
                                                              const uint32_t *__restrict__ link, float *w, int loss,
-                                                             float eta, int epochs, int *status)
+                                                             float eta, int epochs, bool vec, int *status)
 {
     extern __shared__ __align__(16) unsigned char smem_raw[];
     ChainSmem &S = *reinterpret_cast<ChainSmem *>(smem_raw);
     if (read_status(status)) return;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    const bool compute = warp == 0, idle = warp == 4;
-    const int ptid = tid - (warp < 4 ? 32 : 64);
+    // warp 0 computes; warps 1, 2, 3, 5 prefetch example g = 0..3 of a step
+    // (ids, values, link words, then weights); warps 6, 7 write the weights of
+    // the previous step through (two examples each) and copy row bounds; warp
+    // 4 only joins the barriers (it shares warp 0's scheduler)
+    const bool compute = warp == 0;
+    const int gA = warp >= 1 && warp <= 3 ? warp - 1 : warp == 5 ? 3 : -1;
+    const int gW = warp == 6 ? 0 : warp == 7 ? 2 : -1;
     const int N = n_rows;
     const int steps = (N + CH_G - 1) / CH_G;
 
     for (int ep = 0; ep < epochs; ++ep) {
         for (int t = -CH_L; t <= steps; ++t) {
-            if (!compute && !idle) {
-                StepRange R;
-                // stage W: new weights of step t - 1 through to global memory; a weight that a
-                // later example of the same step writes again is left to that example (two
-                // stores of one step to one address would race)
-                if (step_range(S, t - 1, N, R)) {
-#pragma unroll
-                    for (int u = 0; u < CH_PER; ++u) {
-                        const int e = ptid + u * CH_PF;
-                        if (e < R.total) {
-                            int row, i;
-                            locate(R, t - 1, e, row, i);
-                            const int slot = row & (CH_SLOTS - 1);
-                            const uint32_t l = S.link[slot][i];
-                            const bool rewritten = (l & LK_PUSH) && (row & (CH_G - 1)) + (int)((l >> 16) & 0xffu) < CH_G;
-                            if (!rewritten) w[S.col[slot][i]] = S.out[slot][i];
-                        }
+            if (gW >= 0) {
+                // stage W: new weights of step t - 1 that no example among the next D takes
+                // on chip go through to global memory (a pushed weight is re-written by its
+                // receiver, so two stores of one step never hit one address)
+                for (int g = gW; g < gW + 2; ++g) {
+                    const int r = (t - 1) * CH_G + g;
+                    int64_t b;
+                    int k, off;
+                    if (row_bounds(S, r, N, vec, b, k, off)) {
+                        const int slot = r & (CH_SLOTS - 1);
+                        for (int i = lane; i < k; i += 32)
+                            if (!(S.link[slot][off + i] & LK_PUSH)) w[S.col[slot][off + i]] = S.out[slot][i];
                     }
                 }
                 // stage R: row_ptr entries [(t+L)G, (t+L)G + G) with L = DS + BS + 1, so that
                 // stage A of step t finds the bounds of step t + DS (and the entry after it) complete
+                if (warp == 6 && lane < CH_G) {
+                    const int r = (t + CH_L) * CH_G + lane;
+                    if (r >= 0 && r <= N) cp8(&S.rp[r & (CH_RP - 1)], row_ptr + r);
+                }
+            } else if (gA >= 0) {
+                // stage A: ids, values, link words and label of example g of step t + DS
                 {
-                    const int r = (t + CH_L) * CH_G + ptid;
-                    if (ptid < CH_G && r >= 0 && r <= N) cp8(&S.rp[r & (CH_RP - 1)], row_ptr + r);
-                }
-                // stage A: ids, values, link words and labels of step t + DS
-                if (step_range(S, t + CH_DS, N, R)) {
-#pragma unroll
-                    for (int u = 0; u < CH_PER; ++u) {
-                        const int e = ptid + u * CH_PF;
-                        if (e < R.total) {
-                            int row, i;
-                            locate(R, t + CH_DS, e, row, i);
-                            const int slot = row & (CH_SLOTS - 1);
-                            const int64_t pos = R.b0 + e;
-                            cp4(&S.col[slot][i], col + pos);
-                            cp4(&S.link[slot][i], link + pos);
-                            if (val) cp4(&S.val[slot][i], val + pos);
-                        }
+                    const int r = (t + CH_DS) * CH_G + gA;
+                    int64_t b;
+                    int k, off;
+                    if (row_bounds(S, r, N, vec, b, k, off)) {
+                        const int slot = r & (CH_SLOTS - 1);
+                        cp_row(S.col[slot], col, b, k, off, vec, lane);
+                        cp_row(S.link[slot], link, b, k, off, vec, lane);
+                        if (val) cp_row(S.val[slot], val, b, k, off, vec, lane);
+                        if (lane == 0) cp4(&S.y[slot], y + r);
                     }
-                    const int r = (t + CH_DS) * CH_G + ptid;
-                    if (ptid < CH_G && r < N) cp4(&S.y[r & (CH_SLOTS - 1)], y + r);
                 }
-                // stage B: weights of step t + BS that no recent example will push (the
-                // thread that copied a position in stage A handles it here)
-                if (step_range(S, t + CH_BS, N, R)) {
-                    uint32_t l[CH_PER];
-                    int32_t j[CH_PER];
-                    int sl[CH_PER], ix[CH_PER];
-#pragma unroll
-                    for (int u = 0; u < CH_PER; ++u) {
-                        const int e = ptid + u * CH_PF;
-                        l[u] = LK_RECV;
-                        j[u] = 0;
-                        sl[u] = 0;
-                        ix[u] = 0;
-                        if (e < R.total) {
-                            int row, i;
-                            locate(R, t + CH_BS, e, row, i);
-                            sl[u] = row & (CH_SLOTS - 1);
-                            ix[u] = i;
-                            l[u] = S.link[sl[u]][i];
-                            j[u] = S.col[sl[u]][i];
-                        }
+                // stage B: weights of example g of step t + BS that no recent example pushes
+                {
+                    const int r = (t + CH_BS) * CH_G + gA;
+                    int64_t b;
+                    int k, off;
+                    if (row_bounds(S, r, N, vec, b, k, off)) {
+                        const int slot = r & (CH_SLOTS - 1);
+                        for (int i = lane; i < k; i += 32)
+                            if (!(S.link[slot][off + i] & LK_RECV)) cp4(&S.wp[slot][i], w + S.col[slot][off + i]);
                     }
-#pragma unroll
-                    for (int u = 0; u < CH_PER; ++u)
-                        if (!(l[u] & LK_RECV)) cp4(&S.wp[sl[u]][ix[u]], w + j[u]);
                 }
+            }
+            if (!compute) {
                 cp_commit();
                 cp_wait_b();
             } else if (t >= 0 && t < steps) {
                 // compute the G examples of step t in data order
                 for (int r = t * CH_G; r < min(N, t * CH_G + CH_G); ++r) {
                     const int slot = r & (CH_SLOTS - 1);
-                    const int k = (int)(S.rp[(r + 1) & (CH_RP - 1)] - S.rp[r & (CH_RP - 1)]);
+                    int64_t b;
+                    int k, off;
+                    row_bounds(S, r, N, vec, b, k, off);
+                    const float yr = S.y[slot];
                     float xv[R], wv[R];
                     uint32_t lk[R];
                     float acc = 0.0f;
@@ -214,22 +234,23 @@ __global__ __launch_bounds__(CH_THREADS, 1) void k_sgd_chain(int32_t n_rows, con
                     for (int q = 0; q < R; ++q) {
                         const int i = q * 32 + lane;
                         if (i < k) {
-                            xv[q] = val ? S.val[slot][i] : 1.0f;
+                            xv[q] = val ? S.val[slot][off + i] : 1.0f;
                             wv[q] = S.wp[slot][i];
-                            lk[q] = S.link[slot][i];
+                            lk[q] = S.link[slot][off + i];
                             acc = __fmaf_rn(wv[q], xv[q], acc);
                         }
                     }
-                    const float m = warp_combine(acc);
-                    const float c = __fmul_rn(eta, dev_grad(loss, m, S.y[slot]));
+                    const float m = combine_smem(acc, S.part);
+                    const float c = __fmul_rn(eta, dev_grad(loss, m, yr));
 #pragma unroll
                     for (int q = 0; q < R; ++q) {
                         const int i = q * 32 + lane;
                         if (i < k) {
                             const float nw = __fsub_rn(wv[q], __fmul_rn(c, xv[q]));
-                            S.out[slot][i] = nw;
                             if (lk[q] & LK_PUSH)
                                 S.wp[(r + (int)((lk[q] >> 16) & 0xffu)) & (CH_SLOTS - 1)][lk[q] & 0xffffu] = nw;
+                            else
+                                S.out[slot][i] = nw;
                         }
                     }
                     __syncwarp();
@@ -293,8 +314,10 @@ int chain_run(const pdb_csr *X, const float *y, const uint32_t *link, float *w, 
             return PDB_ECUDA;
         configured[dev][variant] = true;
     }
+    // 16-byte row copies need 16-byte aligned ids, values and link words
+    const bool vec = ((uintptr_t)X->col & 15) == 0 && ((uintptr_t)X->val & 15) == 0 && ((uintptr_t)link & 15) == 0;
     kern<<<1, CH_THREADS, sizeof(ChainSmem), s>>>((int32_t)X->n_rows, X->row_ptr, X->col, X->val, y, link, w, loss,
-                                                  eta, epochs, status);
+                                                  eta, epochs, vec, status);
     note_launch();
     return cudaPeekAtLastError() == cudaSuccess ? PDB_OK : PDB_ECUDA;
 }

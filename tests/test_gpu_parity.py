@@ -174,6 +174,28 @@ def test_auto_schedule_choice(name, expect):
     assert np.array_equal(w.cpu().numpy(), C.oracle_sgd(name))
 
 
+@pytest.mark.parametrize("mode", ["chain", "window", "ready"])
+@pytest.mark.parametrize("shift", [1, 2, 3])
+def test_unaligned_input_arrays(mode, shift):
+    # ids and values that do not start on a 16-byte boundary (views into
+    # larger buffers): the engines that stage rows in 16-byte pieces must
+    # fall back to element copies and give the same weights
+    name = "zipf-shape"
+    p = C.problem(name)
+    col_buf = torch.zeros(p.nnz + shift, dtype=torch.int32, device="cuda")
+    val_buf = torch.zeros(p.nnz + shift, dtype=torch.float32, device="cuda")
+    col_buf[shift:] = torch.from_numpy(p.col).cuda()
+    val_buf[shift:] = torch.from_numpy(p.val).cuda()
+    X = pdb.Csr(torch.from_numpy(p.row_ptr).cuda(), col_buf[shift:], val_buf[shift:], p.n_cols)
+    y = torch.from_numpy(p.y).cuda()
+    c = pdb.pdb_build_conflicts(X)
+    s = pdb.pdb_schedule_build(c, MODES[mode])
+    w = torch.zeros(p.n_cols, dtype=torch.float32, device="cuda")
+    pdb.pdb_sgd_epoch(X, y, c, s, w, p.loss, p.eta, p.epochs)
+    pdb.check_status(c)
+    assert np.array_equal(w.cpu().numpy(), C.oracle_sgd(name))
+
+
 def test_sgd_small_grid_and_repeat_calls():
     # a one-block-per-SM grid, and a second call continuing from the first
     name = "zipf-shape"
