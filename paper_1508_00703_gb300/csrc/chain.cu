@@ -131,6 +131,10 @@ __device__ __forceinline__ void cp_row(void *dst, const void *src, int64_t b, in
     for (int64_t e = (a1 > b ? a1 : b) + lane; e < b + k; e += 32)
         cp4((uint32_t *)dst + (e - a0), (const uint32_t *)src + e);
 }
+__device__ __forceinline__ void st_shared(unsigned addr, float v)
+{
+    asm volatile("st.shared.f32 [%0], %1;" ::"r"(addr), "f"(v) : "memory");
+}
 __device__ __forceinline__ void cp_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
 __device__ __forceinline__ void cp_wait_b() { asm volatile("cp.async.wait_group %0;" ::"n"(CH_BS - 1) : "memory"); }
 __device__ __forceinline__ void cp_wait_all() { asm volatile("cp.async.wait_group 0;" ::: "memory"); }
@@ -163,6 +167,8 @@ __global__ __launch_bounds__(CH_THREADS, 1) void k_sgd_chain(int32_t n_rows, con
     // the previous step through (two examples each) and copy row bounds; warp
     // 4 only joins the barriers (it shares warp 0's scheduler)
     const bool compute = warp == 0;
+    const unsigned wp_base = (unsigned)__cvta_generic_to_shared(&S.wp[0][0]);
+    const unsigned out_base = (unsigned)__cvta_generic_to_shared(&S.out[0][0]);
     const int gA = warp >= 1 && warp <= 3 ? warp - 1 : warp == 5 ? 3 : -1;
     const int gW = warp == 6 ? 0 : warp == 7 ? 2 : -1;
     const int N = n_rows;
@@ -246,11 +252,13 @@ __global__ __launch_bounds__(CH_THREADS, 1) void k_sgd_chain(int32_t n_rows, con
                     for (int q = 0; q < R; ++q) {
                         const int i = q * 32 + lane;
                         if (i < k) {
-                            const float nw = __fsub_rn(wv[q], __fmul_rn(c, xv[q]));
-                            if (lk[q] & LK_PUSH)
-                                S.wp[(r + (int)((lk[q] >> 16) & 0xffu)) & (CH_SLOTS - 1)][lk[q] & 0xffffu] = nw;
-                            else
-                                S.out[slot][i] = nw;
+                            // one store per element, no branch: into the receiver's slot of
+                            // wp when pushed, else into out (written through by warps 6, 7)
+                            const unsigned tslot = (r + ((lk[q] >> 16) & 0xffu)) & (CH_SLOTS - 1);
+                            const unsigned a_push = wp_base + 4u * (tslot * CH_MAXK + (lk[q] & 0xffffu));
+                            const unsigned a_out = out_base + 4u * (slot * CH_MAXK + i);
+                            st_shared((lk[q] & LK_PUSH) ? a_push : a_out,
+                                      __fsub_rn(wv[q], __fmul_rn(c, xv[q])));
                         }
                     }
                     __syncwarp();
