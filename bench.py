@@ -51,6 +51,8 @@ def parse_args(argv=None):
     ap.add_argument("--blocks-per-sm", type=int, default=0)
     ap.add_argument("--bsp", type=int, default=0,
                     help="time pdb_bsp_epoch with this mini-batch instead of pdb_sgd_epoch (-1: the workload's own)")
+    ap.add_argument("--delay", type=int, default=None,
+                    help="time pdb_ssp_epoch (admissible delay, READY schedule) with this delay instead")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=10.0, help="target length of the CPU oracle sample")
@@ -297,6 +299,10 @@ def run_ours(args, rank, world, local_rank):
         if batch:
             pdb.pdb_bsp_epoch(X, y, c, w, p.loss, p.eta, batch, E, opts=opts, stream=stream)
             return c, None
+        if args.delay is not None:
+            s = pdb.pdb_schedule_build(c, pdb.PDB_SCHED_READY, stream)
+            pdb.pdb_ssp_epoch(X, y, c, s, w, p.loss, p.eta, E, args.delay, opts=opts, stream=stream)
+            return c, s
         s = pdb.pdb_schedule_build(c, mode, stream)
         pdb.pdb_sgd_epoch(X, y, c, s, w, p.loss, p.eta, E, opts=opts, stream=stream)
         return c, s
@@ -341,7 +347,9 @@ def run_ours(args, rank, world, local_rank):
     sgd_launch_ms = ms_kern / E
     sgd_gbs = sgd_bytes_per_launch / (sgd_launch_ms / 1e3) / 1e9
     resolved = int(phases[0]["sched_mode"])
-    kname = {pdb.PDB_SCHED_READY: "k_sgd_ready", pdb.PDB_SCHED_LEVELS: "k_sgd_levels", -1: "k_bsp",
+    if args.delay is not None:
+        resolved = -2
+    kname = {pdb.PDB_SCHED_READY: "k_sgd_ready", pdb.PDB_SCHED_LEVELS: "k_sgd_levels", -1: "k_bsp", -2: "k_sgd_ssp",
              pdb.PDB_SCHED_CHAIN: "k_sgd_chain", pdb.PDB_SCHED_WINDOW: "k_sgd_window"}[resolved]
     roofline = {"kernel": kname,
                 "bound": "hbm", "achieved": round(sgd_gbs, 1), "peak": peak, "unit": "GB/s",
@@ -355,6 +363,7 @@ def run_ours(args, rank, world, local_rank):
         "vs_baseline": None, "dtype": "f32", "data": "synthetic (seeded generator, no dataset)",
         "config": dict(workload_config(args.workload, p,
                                        f"bsp, mini-batch {batch}" if batch else
+                                       f"admissible delay {args.delay} (READY records)" if args.delay is not None else
                                        {0: "levels", 1: "ready", 2: "chain", 4: "window"}[resolved]
                                        + (" (auto)" if args.mode == "auto" else "")),
                        parallelism=f"replicas{world}" if world > 1 else "single GPU",
@@ -368,12 +377,17 @@ def run_ours(args, rank, world, local_rank):
         "clocks": clk.summary(),
     }
 
+    if args.delay is not None:
+        result["metric"] = METRIC.replace("serially-equivalent sparse SGD",
+                                          f"admissible-delay ({args.delay}) sparse SGD")
+        if args.delay > 0:
+            result["config"]["note"] = "delay > 0: not serially equivalent, result depends on timing"
     if batch:
         roofline["kernel"] = "k_bsp (whole pdb_bsp_epoch call per epoch: batch sort, gather, cooperative kernel)"
         result["metric"] = METRIC.replace("serially-equivalent sparse SGD", f"BSP mini-batch ({batch}) SGD")
         del result["sgd_only"]
         result["bsp_only"] = {"value": units / (ms_sgd / 1e3), "unit": UNIT}
-    if not args.no_e2e and not batch:
+    if not args.no_e2e and not batch and args.delay is None:
         result["e2e"] = run_e2e(args, p, mode, pdb, torch, world)
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         result["cpu_baseline"] = cpu_baseline(p, args.cpu_seconds)

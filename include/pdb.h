@@ -226,6 +226,26 @@ int pdb_schedule_ready(const pdb_schedule *s, const uint32_t **gate, const uint6
 int pdb_sgd_epoch(const pdb_csr *X, const float *y, const pdb_conflicts *c, const pdb_schedule *s, float *w,
                   pdb_loss loss, float eta, int n_epochs, const pdb_opts *opts, void *stream);
 
+/* SGD with admissible delay (Section 7): like pdb_sgd_epoch under a READY
+ * schedule, with the asynchronous Read and Write Constraints counted per
+ * feature.  The occurrence of feature j with rank r reads w_j once at least
+ * r - delay writes of j are done, and writes once at least r - delay + 1
+ * occurrences of j have read; its write applies its step to the current
+ * w_j (an atomic fp32 add of -(eta*g)*x_j, then the write is counted), so
+ * every example's update is applied exactly once.  w is updated in place.
+ *   delay = 0    the sequential result, bitwise equal to pdb_sgd_epoch
+ *   delay > 0    reads may be up to `delay` occurrences stale; the result
+ *                depends on timing and is not deterministic
+ *   delay >= the longest chain  no waits at all (Hogwild with atomic updates)
+ *   coef         optional device array of n_epochs * n_rows floats (NULL for
+ *                none): the step eta*g each example applied, epoch-major,
+ *                for auditing a delayed run
+ * s must be a READY schedule of c (PDB_ESTATE otherwise); delay < 0 is
+ * PDB_EINVAL.  Every wait is bounded (pdb_opts.wait_timeout_s). */
+int pdb_ssp_epoch(const pdb_csr *X, const float *y, const pdb_conflicts *c, const pdb_schedule *s, float *w,
+                  pdb_loss loss, float eta, int n_epochs, int64_t delay, float *coef, const pdb_opts *opts,
+                  void *stream);
+
 /* BSP comparison (Algorithm 2a with `batch` examples between barriers):
  * per batch [b*B, min((b+1)*B, N)) every example computes c_i = eta *
  * dloss/dm at the weights of the batch start (read barrier), then each

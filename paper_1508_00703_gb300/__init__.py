@@ -107,7 +107,7 @@ EXPORTS = ["pdb_build_conflicts", "pdb_conflicts_arrays", "pdb_schedule_build", 
            "pdb_schedule_ready",
            "pdb_sgd_epoch", "pdb_bsp_epoch", "pdb_status", "pdb_get_stats", "pdb_conflicts_free",
            "pdb_schedule_free", "pdb_strerror", "pdb_memcpy", "pdb_eval_expf", "pdb_launch_count",
-           "pdb_sgd_epoch_ready_noalloc"]
+           "pdb_sgd_epoch_ready_noalloc", "pdb_ssp_epoch"]
 
 
 def load(path: str | None = None):
@@ -137,6 +137,8 @@ def load(path: str | None = None):
         lib.pdb_memcpy.argtypes = [P, P, ctypes.c_size_t, P]
         lib.pdb_eval_expf.argtypes = [P, P, I64, P]
         lib.pdb_sgd_epoch_ready_noalloc.argtypes = [ctypes.POINTER(pdb_csr), P, P, P, I32, ctypes.c_float, I32, P]
+        lib.pdb_ssp_epoch.argtypes = [ctypes.POINTER(pdb_csr), P, P, P, P, I32, ctypes.c_float, I32, I64, P,
+                                      ctypes.POINTER(pdb_opts), P]
         lib.pdb_launch_count.argtypes = []
         lib.pdb_launch_count.restype = I64
         _lib = lib
@@ -257,6 +259,13 @@ def pdb_sgd_epoch(X: Csr, y, c: Conflicts, s: Schedule, w, loss: int, eta: float
                   stream=None):
     _check(load().pdb_sgd_epoch(ctypes.byref(X.struct), _ptr(y), c.handle, s.handle, _ptr(w), int(loss), float(eta),
                                 int(n_epochs), _opts(opts), _stream(stream)), "pdb_sgd_epoch")
+
+
+def pdb_ssp_epoch(X: Csr, y, c: Conflicts, s: Schedule, w, loss: int, eta: float, n_epochs: int, delay: int,
+                  coef=None, opts=None, stream=None):
+    _check(load().pdb_ssp_epoch(ctypes.byref(X.struct), _ptr(y), c.handle, s.handle, _ptr(w), int(loss), float(eta),
+                                int(n_epochs), int(delay), _ptr(coef), _opts(opts), _stream(stream)),
+           "pdb_ssp_epoch")
 
 
 def pdb_bsp_epoch(X: Csr, y, c: Conflicts, w, loss: int, eta: float, batch: int, n_epochs: int, opts=None,

@@ -203,6 +203,10 @@ struct WindowCtl {
     long long wpos;             // every example starting below this position has finished
 };
 
+int ssp_run(const pdb_csr *X, const float *y, const uint32_t *gate, float *w, unsigned *writes, unsigned *reads,
+            unsigned long long *ticket, long long delay, float *coef, int loss, float eta, int n_epochs, int width,
+            const pdb_opts *opts, int *status, uint64_t timeout, cudaStream_t s);
+
 int ensure_row_of(pdb_conflicts *c, cudaStream_t s);   // builds c->row_of on first use (stream-ordered)
 
 int window_run(const pdb_csr *X, const float *y, const uint32_t *gate, float *w, unsigned long long *rec,
@@ -249,6 +253,7 @@ struct pdb_schedule {
     int64_t *level_ptr;
     LevelCtl *ctl;            // device
     unsigned long long *rec;  // READY: per feature (weight bits | version << 32); WINDOW: near hand-offs
+    unsigned *reads, *writes; // READY under pdb_ssp_epoch: reads / writes of each feature this epoch (first use)
     uint32_t *link;           // CHAIN: per position, receive flag and push target
     unsigned epochs_run;      // WINDOW: epochs run so far (epoch stamp of the record tags)
     unsigned *prog;           // WINDOW: progress word per worker warp

@@ -448,6 +448,36 @@ int pdb_sgd_epoch(const pdb_csr *X, const float *y, const pdb_conflicts *c, cons
     return rc;
 }
 
+int pdb_ssp_epoch(const pdb_csr *X, const float *y, const pdb_conflicts *c, const pdb_schedule *h, float *w,
+                  pdb_loss loss, float eta, int n_epochs, int64_t delay, float *coef, const pdb_opts *opts,
+                  void *stream)
+{
+    int rc = check_run(X, y, c, w, loss, n_epochs);
+    if (rc != PDB_OK) return rc;
+    if (!h || h->c != c || delay < 0) return PDB_EINVAL;
+    if (h->mode != PDB_SCHED_READY) return PDB_ESTATE;
+    cudaStream_t s = (cudaStream_t)stream;
+    pdb_conflicts *cm = const_cast<pdb_conflicts *>(c);
+    pdb_schedule *hm = const_cast<pdb_schedule *>(h);
+    const int width = register_width(cm);
+    if (!hm->reads) {
+        rc = alloc((void **)&hm->reads, sizeof(unsigned) * std::max<int64_t>(X->n_cols, 1), s);
+        rc = rc ? rc : alloc((void **)&hm->writes, sizeof(unsigned) * std::max<int64_t>(X->n_cols, 1), s);
+        if (rc != PDB_OK) return rc;
+    }
+    cudaEventRecord(cm->ev_sgd0, s);
+    cudaEventRecord(cm->ev_k0, s);
+    if (X->n_rows > 0 && n_epochs > 0)
+        rc = ssp_run(X, y, c->gate, w, hm->writes, hm->reads, h->ticket, (long long)std::min<int64_t>(delay, 1ll << 40),
+                     coef, (int)loss, eta, n_epochs, width, opts, cm->status, timeout_ns(opts), s);
+    cudaEventRecord(cm->ev_k1, s);
+    cudaEventRecord(cm->ev_sgd1, s);
+    cm->timed_sgd = true;
+    if (rc == PDB_OK && cudaPeekAtLastError() != cudaSuccess) rc = PDB_ECUDA;
+    if (rc != PDB_OK) cudaGetLastError();
+    return rc;
+}
+
 int pdb_bsp_epoch(const pdb_csr *X, const float *y, const pdb_conflicts *c, float *w, pdb_loss loss, float eta,
                   int64_t batch, int n_epochs, const pdb_opts *opts, void *stream)
 {

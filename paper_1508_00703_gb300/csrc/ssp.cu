@@ -1,0 +1,190 @@
+// Admissible-delay engine: pdb_ssp_epoch (Section 7).
+//
+// The asynchronous Read and Write Constraints of Section 7, per feature as
+// everywhere else in this library (an iteration = one example, a chunk = one
+// feature, iteration numbers counted per feature):
+//
+//   read   the occurrence of feature j with rank r may read w_j once at least
+//          r - delta writes of j are done (its view is at most delta
+//          occurrences stale);
+//   write  it may write once at least r - delta + 1 occurrences of j have
+//          read (no reader lags the writer by more than delta), and it
+//          applies its step to the current w_j with an atomic fp32 add of
+//          -(eta*g*x_j), then counts the write (release): no update is lost
+//          even when a later occurrence wrote first, and nothing retries.
+//
+// delta = 0 is the sequential computation: the reader of rank r sees exactly
+// r writes, nobody else writes between its read and its write, and
+// w + (-(c*x)) rounds exactly as the sequential w - c*x, so the result is
+// the READY engine's bit for bit.  delta > 0 admits more interleavings;
+// results then depend on timing (not deterministic).  delta >= the longest
+// chain is Hogwild with atomic updates (the paper's delta = infinity).
+//
+// Deadlock freedom: examples are taken in data order; the oldest unfinished
+// example finds every earlier occurrence of its features read and written,
+// so both of its waits pass.  Every wait is bounded by the timeout.
+#include <cuda_runtime.h>
+
+#include "common.cuh"
+
+using namespace pdb;
+
+namespace {
+
+__device__ __forceinline__ unsigned ld_acquire_u32(const unsigned *p)
+{
+    unsigned v;
+    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+// count one read or write of the feature, after the access it counts (release)
+__device__ __forceinline__ void count_release(unsigned *p)
+{
+    asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(p) : "memory");
+}
+
+__device__ __forceinline__ bool keep_waiting(unsigned &spins, uint64_t t0, int *status, uint64_t timeout)
+{
+    if ((++spins & 15u) != 0) return true;
+    if (read_status(status)) return false;
+    if (globaltimer() - t0 > timeout) {
+        set_status(status, PDB_ETIMEOUT);
+        return false;
+    }
+    return true;
+}
+
+// waits until counter >= need (need <= 0: at once)
+__device__ __forceinline__ bool wait_count(const unsigned *counter, long long need, int *status, uint64_t timeout)
+{
+    if (need <= 0 || (long long)ld_acquire_u32(counter) >= need) return true;
+    const uint64_t t0 = globaltimer();
+    unsigned spins = 0, nap = 32;
+    for (;;) {
+        __nanosleep(nap);
+        nap = nap < 512 ? 2 * nap : 512;
+        if ((long long)ld_acquire_u32(counter) >= need) return true;
+        if (!keep_waiting(spins, t0, status, timeout)) return false;
+    }
+}
+
+// w_j once at least `need` writes of j are done, then count the read
+__device__ __forceinline__ bool read_admitted(const float *w, const unsigned *writes, unsigned *reads, int j,
+                                              long long need, float &wv, int *status, uint64_t timeout)
+{
+    if (!wait_count(writes + j, need, status, timeout)) return false;
+    wv = __ldcg(w + j);
+    count_release(reads + j);
+    return true;
+}
+
+// w_j -= step once at least `need` reads of j are done, then count the write
+__device__ __forceinline__ bool write_admitted(float *w, unsigned *writes, const unsigned *reads, int j,
+                                               long long need, float step, int *status, uint64_t timeout)
+{
+    if (!wait_count(reads + j, need, status, timeout)) return false;
+    atomicAdd(w + j, -step);
+    count_release(writes + j);
+    return true;
+}
+
+template <int R>
+__global__ __launch_bounds__(THREADS) void k_sgd_ssp(int32_t n_rows, const int64_t *__restrict__ row_ptr,
+                                                     const int32_t *__restrict__ col, const float *__restrict__ val,
+                                                     const float *__restrict__ y, const uint32_t *__restrict__ gate,
+                                                     float *w, unsigned *writes, unsigned *reads, long long delay,
+                                                     float *coef, int loss, float eta, unsigned long long *ticket,
+                                                     int chunk, int *status, uint64_t timeout)
+{
+    if (read_status(status)) return;
+    const int lane = threadIdx.x & 31;
+    for (;;) {
+        unsigned long long tk = 0;
+        if (lane == 0) tk = atomicAdd(ticket, (unsigned long long)chunk);
+        tk = __shfl_sync(FULL, tk, 0);
+        if (tk >= (unsigned long long)n_rows) return;
+        const int t1 = (int)min64((int64_t)n_rows, (int64_t)tk + chunk);
+        for (int t = (int)tk; t < t1; ++t) {
+            const int64_t b = row_ptr[t];
+            const int k = (int)(row_ptr[t + 1] - b);
+            const float yt = y[t];
+            bool ok = true;
+            float acc = 0.0f;
+            if (k <= 32 * R) {
+                int j[R];
+                float x[R], wv[R];
+                long long rank[R];
+#pragma unroll
+                for (int r = 0; r < R; ++r) {
+                    const int i = r * 32 + lane;
+                    j[r] = i < k ? col[b + i] : 0;
+                    x[r] = i < k ? (val ? val[b + i] : 1.0f) : 0.0f;
+                    rank[r] = i < k ? (long long)(gate[b + i] & GATE_RANK) : 0;
+                    wv[r] = 0.0f;
+                }
+#pragma unroll
+                for (int r = 0; r < R; ++r)
+                    if (r * 32 + lane < k && ok) {
+                        ok = read_admitted(w, writes, reads, j[r], rank[r] - delay, wv[r], status, timeout);
+                    }
+                if (!__all_sync(FULL, ok)) return;
+#pragma unroll
+                for (int r = 0; r < R; ++r)
+                    if (r * 32 + lane < k) acc = __fmaf_rn(wv[r], x[r], acc);
+                const float m = warp_combine(acc);
+                const float c = __fmul_rn(eta, dev_grad(loss, m, yt));
+                if (coef && lane == 0) coef[t] = c;
+#pragma unroll
+                for (int r = 0; r < R; ++r)
+                    if (r * 32 + lane < k && ok)
+                        ok = write_admitted(w, writes, reads, j[r], rank[r] - delay + 1, __fmul_rn(c, x[r]), status,
+                                            timeout);
+                if (!__all_sync(FULL, ok)) return;
+                continue;
+            }
+            // long example: element by element
+            for (int i = lane; i < k && ok; i += 32) {
+                const int jj = col[b + i];
+                float v1 = 0.0f;
+                ok = read_admitted(w, writes, reads, jj, (long long)(gate[b + i] & GATE_RANK) - delay, v1, status,
+                                   timeout);
+                if (ok) acc = __fmaf_rn(v1, val ? val[b + i] : 1.0f, acc);
+            }
+            if (!__all_sync(FULL, ok)) return;
+            const float m = warp_combine(acc);
+            const float c = __fmul_rn(eta, dev_grad(loss, m, yt));
+            if (coef && lane == 0) coef[t] = c;
+            for (int i = lane; i < k && ok; i += 32)
+                ok = write_admitted(w, writes, reads, col[b + i], (long long)(gate[b + i] & GATE_RANK) - delay + 1,
+                                    __fmul_rn(c, val ? val[b + i] : 1.0f), status, timeout);
+            if (!__all_sync(FULL, ok)) return;
+        }
+    }
+}
+
+}  // namespace
+
+namespace pdb {
+
+int ssp_run(const pdb_csr *X, const float *y, const uint32_t *gate, float *w, unsigned *writes, unsigned *reads,
+            unsigned long long *ticket, long long delay, float *coef, int loss, float eta, int n_epochs, int width,
+            const pdb_opts *opts, int *status, uint64_t timeout, cudaStream_t s)
+{
+    const int32_t n = (int32_t)X->n_rows;
+    const int64_t F = X->n_cols;
+    const int chunk = (opts && opts->ticket_chunk > 0) ? opts->ticket_chunk : 2;
+    auto kern = width == 2 ? k_sgd_ssp<2> : width == 4 ? k_sgd_ssp<4> : k_sgd_ssp<8>;
+    const int grid = persistent_grid((const void *)kern, opts);
+    for (int ep = 0; ep < n_epochs; ++ep) {
+        cudaMemsetAsync(writes, 0, sizeof(unsigned) * (size_t)F, s);
+        cudaMemsetAsync(reads, 0, sizeof(unsigned) * (size_t)F, s);
+        cudaMemsetAsync(ticket, 0, sizeof(unsigned long long), s);
+        kern<<<grid, THREADS, 0, s>>>(n, X->row_ptr, X->col, X->val, y, gate, w, writes, reads, delay,
+                                      coef ? coef + (int64_t)ep * n : nullptr, loss, eta, ticket, chunk, status,
+                                      timeout);
+        note_launch();
+    }
+    return cudaPeekAtLastError() == cudaSuccess ? PDB_OK : PDB_ECUDA;
+}
+
+}  // namespace pdb
