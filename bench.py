@@ -318,13 +318,17 @@ def run_ours(args, rank, world, local_rank):
     launches0 = pdb.pdb_launch_count()
     with ClockSampler(local_rank) as clk:
         ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        marks = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps + 1)]
         ev0.record(stream)
-        for _ in range(args.steps):
+        marks[0].record(stream)
+        for i in range(args.steps):
             c, s = step()
+            marks[i + 1].record(stream)
             phases.append(pdb.pdb_get_stats(c, s))   # synchronizes; frees the step's handles below
             del c, s
         ev1.record(stream)
         torch.cuda.synchronize()
+    per_step = sorted(marks[i].elapsed_time(marks[i + 1]) for i in range(args.steps))
     barrier(world)
     launches = pdb.pdb_launch_count() - launches0
     ms_step = ev0.elapsed_time(ev1) / args.steps
@@ -373,6 +377,9 @@ def run_ours(args, rank, world, local_rank):
                       {"build_conflicts": ms_build, "schedule": ms_sched, "sgd_all_epochs": ms_sgd,
                        "sgd_update_kernels": ms_kern}),
         "sgd_only": {"value": units / (ms_sgd / 1e3), "unit": UNIT},
+        # per-step device times (the paper's protocol: trimmed mean without the 2 fastest and 2 slowest)
+        "step_ms": {"trimmed_mean": statistics.mean(per_step[2:-2] if len(per_step) > 4 else per_step),
+                    "median": statistics.median(per_step), "min": per_step[0], "max": per_step[-1]},
         "gpu_launches": int(launches),
         "clocks": clk.summary(),
     }
