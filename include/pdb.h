@@ -96,8 +96,10 @@ typedef enum { PDB_LOSS_LOGISTIC = 0, PDB_LOSS_SQUARED = 1, PDB_LOSS_HINGE = 2 }
  *           data order (Algorithm 1 itself), prefetching ids, values and
  *           weights ahead and forwarding each new weight whose next
  *           occurrence is among the next 16 examples through shared memory,
- *           so a dependency hop costs a few hundred cycles.  Examples of at
- *           most 256 ids.
+ *           so a dependency hop costs a few hundred cycles (examples of at
+ *           most 256 ids).  Longer examples run with all n_cols weights
+ *           resident in shared memory instead, when they fit (about 55,000
+ *           features; dense examples of ~1000 features); else PDB_ETOOBIG.
  *   WINDOW  for conflict graphs whose consecutive occurrences of a feature
  *           mostly lie far apart: w stays a plain float array.  A position
  *           whose previous occurrence lies at least `near` positions back
@@ -107,7 +109,7 @@ typedef enum { PDB_LOSS_LOGISTIC = 0, PDB_LOSS_SQUARED = 1, PDB_LOSS_HINGE = 2 }
  *           iteration number as under READY, kept in a separate word that
  *           only near writers release.
  *   AUTO    CHAIN when the longest per-feature chain exceeds n_rows / 20 and
- *           every example has at most 256 ids; else WINDOW when at most 1/8
+ *           CHAIN takes the rows (see above); else WINDOW when at most 1/8
  *           of the positions have a near next occurrence; else READY (waits
  *           on the host for the conflict build to read those numbers). */
 typedef enum {
@@ -184,8 +186,9 @@ int pdb_conflicts_arrays(const pdb_conflicts *c, const int32_t **csc_pos, const 
  *     equal to its occurrence rank (the conflicts' gate array).
  *   CHAIN: per position, whether an example among the 16 before it writes
  *     its feature last (its weight is then forwarded on chip) and where the
- *     next occurrence sits if within the 16 examples after.
- *     PDB_ETOOBIG when an example has more than 256 ids.
+ *     next occurrence sits if within the 16 examples after; nothing when the
+ *     longest example has more than 256 ids and the weights fit in shared
+ *     memory (resident); PDB_ETOOBIG when they do not.
  *   WINDOW: per feature a 32-bit iteration number, per example a finished
  *     flag, and the watermark; the positions' near flags are in the gate.
  *   AUTO: CHAIN, WINDOW or READY (see pdb_sched_mode).

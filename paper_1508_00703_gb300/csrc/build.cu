@@ -378,8 +378,8 @@ const char *pdb_strerror(int code)
     case PDB_EFAULT: return "internal invariant failed on the device";
     case PDB_ESTATE: return "handle in the wrong mode for this call";
     case PDB_ETOOBIG:
-        return "problem beyond a fixed limit (allocation-free scratch: 2^20 features; CHAIN: 256 ids per example; "
-               "a feature in 2^29 positions or more)";
+        return "problem beyond a fixed limit (allocation-free scratch: 2^20 features; CHAIN: 256 ids per example "
+               "unless the weights fit in shared memory; a feature in 2^29 positions or more)";
     default: return "unknown error";
     }
 }
@@ -566,7 +566,8 @@ int pdb_schedule_build(const pdb_conflicts *c, pdb_sched_mode mode, pdb_schedule
             cudaGetLastError();
             return PDB_ECUDA;
         }
-        const bool fits = c->h_info[INFO_MAX_ROW] <= chain_max_row();
+        const bool fits = c->h_info[INFO_MAX_ROW] <= chain_max_row() ||
+                          resident_smem(c->n_cols, c->h_info[INFO_MAX_ROW]) > 0;
         // AUTO: one chain dominates -> CHAIN; near occurrence pairs rare
         // (at most 1/8 of the positions) -> WINDOW; else READY
         if (mode == PDB_SCHED_AUTO)
@@ -607,10 +608,15 @@ int pdb_schedule_build(const pdb_conflicts *c, pdb_sched_mode mode, pdb_schedule
         rc = rc ? rc : alloc((void **)&h->prog, sizeof(unsigned) * h->prog_cap, s);
         rc = rc ? rc : alloc((void **)&h->wctl, sizeof(WindowCtl), s);
     } else if (mode == PDB_SCHED_CHAIN) {
-        rc = rc ? rc : materialize_chains(cm, s);
-        rc = rc ? rc : alloc((void **)&h->link, sizeof(uint32_t) * nnz, s);
-        rc = rc ? rc : ensure_row_of(cm, s);
-        rc = rc ? rc : chain_schedule(c->prev, c->next, c->row_of, c->row_ptr, nnz, h->link, c->status, s);
+        // rows longer than the forwarding engine takes: weights resident in
+        // shared memory (they fit, checked above), no link words
+        h->resident = c->h_info[INFO_MAX_ROW] > chain_max_row();
+        if (!h->resident) {
+            rc = rc ? rc : materialize_chains(cm, s);
+            rc = rc ? rc : alloc((void **)&h->link, sizeof(uint32_t) * nnz, s);
+            rc = rc ? rc : ensure_row_of(cm, s);
+            rc = rc ? rc : chain_schedule(c->prev, c->next, c->row_of, c->row_ptr, nnz, h->link, c->status, s);
+        }
     } else {
         rc = rc ? rc : materialize_chains(cm, s);
         rc = rc ? rc : ensure_row_of(cm, s);

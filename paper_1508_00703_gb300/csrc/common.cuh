@@ -31,6 +31,9 @@ int grid_1d(int64_t n);                               // blocks of 256 threads f
 
 // chain engine (chain.cu)
 int chain_max_row();
+int64_t resident_smem(int64_t n_cols, int64_t max_row);   // 0 when the weights do not fit in one block
+int resident_run(const pdb_csr *X, const float *y, float *w, int loss, float eta, int epochs, int max_row,
+                 int *status, cudaStream_t s);
 int chain_schedule(const int32_t *prev, const int32_t *next, const int32_t *row_of, const int64_t *row_ptr,
                    int64_t nnz, uint32_t *link, const int *status, cudaStream_t s);
 int chain_run(const pdb_csr *X, const float *y, const uint32_t *link, float *w, int loss, float eta, int epochs,
@@ -255,6 +258,7 @@ struct pdb_schedule {
     unsigned long long *rec;  // READY: per feature (weight bits | version << 32); WINDOW: near hand-offs
     unsigned *reads, *writes; // READY under pdb_ssp_epoch: reads / writes of each feature this epoch (first use)
     uint32_t *link;           // CHAIN: per position, receive flag and push target
+    bool resident;            // CHAIN: weights resident in shared memory (no link words)
     unsigned epochs_run;      // WINDOW: epochs run so far (epoch stamp of the record tags)
     unsigned *prog;           // WINDOW: progress word per worker warp
     int64_t prog_cap;

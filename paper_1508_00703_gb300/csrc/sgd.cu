@@ -414,7 +414,8 @@ int pdb_sgd_epoch(const pdb_csr *X, const float *y, const pdb_conflicts *c, cons
             cudaEventRecord(cm->ev_k1, s);
         } else if (h->mode == PDB_SCHED_CHAIN) {
             cudaEventRecord(cm->ev_k0, s);
-            rc = chain_run(X, y, h->link, w, lossi, eta, n_epochs, c->h_info[2], cm->status, s);
+            rc = h->resident ? resident_run(X, y, w, lossi, eta, n_epochs, c->h_info[2], cm->status, s)
+                             : chain_run(X, y, h->link, w, lossi, eta, n_epochs, c->h_info[2], cm->status, s);
             cudaEventRecord(cm->ev_k1, s);
         } else if (h->mode == PDB_SCHED_WINDOW) {
             cudaEventRecord(cm->ev_k0, s);

@@ -118,9 +118,14 @@ WORKLOADS = {
     "deep-chain": dict(n_rows=2_000_000, n_cols=50_000, k=200, ids="zipf", zipf_s=1.3,
                        vals="normal", labels="sign", wstar_std=1.0, loss="hinge", eta=0.01,
                        epochs=3, bsp_batch=4096),
+    # the dense linear-regression setting of the paper's Experiments 6.1/6.2:
+    # 960 numerical features, 5000 examples, full-batch gradient descent
+    # (BSP with one batch of all examples per iteration)
+    "dense-lr": dict(n_rows=5_000, n_cols=960, k=960, ids="dense", vals="normal", labels="linear",
+                     wstar_std=1.0, noise_std=0.1, loss="squared", eta=1e-4, epochs=20, bsp_batch=5_000),
 }
 
-_IDS = {"uniform": 0, "zipf": 1}
+_IDS = {"uniform": 0, "zipf": 1, "dense": 2}
 _VALS = {"normal": 0, "uniform": 1, "ones": 2}
 _LABELS = {"sign": 0, "bernoulli": 1, "linear": 2}
 

@@ -15,6 +15,8 @@
  * Feature-id distributions:
  *   uniform : ids uniform on [0, F), drawn with replacement, duplicates in a
  *             row rejected until k distinct ids are held.
+ *   dense   : every example holds features 0 .. k-1 (k <= F; k = F is a
+ *             dense matrix).
  *   zipf(s) : rank r in 1..F with probability r^-s / H(F,s), mapped to an id
  *             through one seeded Fisher-Yates permutation of [0, F); the
  *             inverse CDF is evaluated with a guide table (the cutpoint
@@ -31,7 +33,7 @@
 typedef struct {
     int64_t n_rows, n_cols;
     int32_t k, k_lo;       /* row length uniform in [k_lo, k]; k_lo == k gives fixed length */
-    int32_t id_dist;       /* 0 uniform, 1 zipf */
+    int32_t id_dist;       /* 0 uniform, 1 zipf, 2 dense */
     double zipf_s;
     int32_t val_dist;      /* 0 N(0,1), 1 U(-1,1), 2 all ones */
     int32_t label_kind;    /* 0 sign(w*.x) (sign(0)=+1), 1 Bernoulli(sigmoid(w*.x)) -> +-1, 2 w*.x + noise */
@@ -245,6 +247,11 @@ static void *row_worker(void *arg)
         int64_t draws = 0;
         while (n < len) {
             if (++draws > max_draws) { j->status = -3; free(set); return NULL; }
+            if (c->id_dist == 2) {      /* dense: the example holds features 0 .. len-1 */
+                ids[n] = n;
+                ++n;
+                continue;
+            }
             int32_t id = c->id_dist == 1 ? zipf_draw(j->z, &r) : (int32_t)rng_below(&r, (uint64_t)c->n_cols);
             uint64_t h = ((uint64_t)id * 0x9E3779B97F4A7C15ull) >> 20;
             int fresh = 1;

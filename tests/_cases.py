@@ -20,6 +20,11 @@ SMALL = {
     "wide-ids-4pass": ("low-conflict", dict(n_rows=3000, n_cols=20_000_000, k=50)),
     "ids-18bit": ("zipf-1m", dict(n_rows=20000, n_cols=200_000)),
     "ids-20bit": ("zipf-1m", dict(n_rows=20000, n_cols=1_000_000)),
+    # the paper's dense linear regression (Experiments 6.1/6.2): every example
+    # conflicts with every other; rows longer than CHAIN takes, and short
+    # enough for it
+    "dense-shape": ("dense-lr", dict(n_rows=800, n_cols=320, k=320, epochs=3, bsp_batch=800)),
+    "dense-narrow": ("dense-lr", dict(n_rows=1500, n_cols=200, k=200, epochs=2, bsp_batch=1500)),
 }
 
 FULL = {

@@ -113,13 +113,6 @@ def near(monkeypatch):
 @pytest.mark.parametrize("mode", list(MODES))
 @pytest.mark.parametrize("name", ALL)
 def test_sgd_weights(name, mode):
-    p = C.problem(name)
-    longest = int(np.max(np.diff(p.row_ptr))) if p.n_rows else 0
-    if mode == "chain" and longest > 256:
-        with pytest.raises(pdb.PdbError) as e:
-            _sgd(name, MODES[mode])
-        assert e.value.code == pdb.PDB_ETOOBIG
-        return
     got = _sgd(name, MODES[mode])
     ref = C.oracle_sgd(name)
     assert C.rel_err(got, ref) <= TOL
@@ -174,13 +167,32 @@ def test_auto_schedule_choice(name, expect):
     assert np.array_equal(w.cpu().numpy(), C.oracle_sgd(name))
 
 
+def test_chain_limits():
+    # CHAIN keeps the weights in shared memory when they fit (rows of any
+    # length); otherwise it forwards them between examples, for rows of at
+    # most 256 ids, and refuses longer ones
+    import synthdata
+    p = synthdata.generate("tiny", n_rows=300, n_cols=2_000_000, k=300, k_lo=260)
+    X = pdb.Csr.from_problem(p)
+    c = pdb.pdb_build_conflicts(X)
+    with pytest.raises(pdb.PdbError) as e:
+        pdb.pdb_schedule_build(c, pdb.PDB_SCHED_CHAIN)
+    assert e.value.code == pdb.PDB_ETOOBIG
+    s = pdb.pdb_schedule_build(c, pdb.PDB_SCHED_AUTO)       # AUTO falls back
+    assert pdb.pdb_get_stats(c, s)["sched_mode"] != pdb.PDB_SCHED_CHAIN
+
+
 @pytest.mark.parametrize("mode", ["chain", "window", "ready"])
 @pytest.mark.parametrize("shift", [1, 2, 3])
 def test_unaligned_input_arrays(mode, shift):
     # ids and values that do not start on a 16-byte boundary (views into
     # larger buffers): the engines that stage rows in 16-byte pieces must
     # fall back to element copies and give the same weights
-    name = "zipf-shape"
+    for name in ("zipf-shape", "ids-18bit"):    # resident weights, and forwarded ones
+        _unaligned_case(name, mode, shift)
+
+
+def _unaligned_case(name, mode, shift):
     p = C.problem(name)
     col_buf = torch.zeros(p.nnz + shift, dtype=torch.int32, device="cuda")
     val_buf = torch.zeros(p.nnz + shift, dtype=torch.float32, device="cuda")
@@ -212,7 +224,8 @@ def test_sgd_small_grid_and_repeat_calls():
 
 
 @pytest.mark.parametrize("batch", [1, 7, 64, 4096, 10**9])
-@pytest.mark.parametrize("name", ["tiny", "deepchain-shape", "ragged-empty-rows", "ctr-shape-binary"])
+@pytest.mark.parametrize("name", ["tiny", "deepchain-shape", "ragged-empty-rows", "ctr-shape-binary",
+                                  "dense-shape"])
 def test_bsp_weights(name, batch):
     import oracle
     p, X, y = _gpu(name)

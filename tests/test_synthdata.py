@@ -18,6 +18,7 @@ def test_philox_known_answer():
     ("ctr", dict(n_rows=20000, n_cols=200000)),
     ("low-conflict", dict(n_rows=20000, n_cols=1_000_000)),
     ("deep-chain", dict(n_rows=2000)),
+    ("dense-lr", {}),
 ])
 def test_workload_shape(name, kw):
     p = synthdata.generate(name, **kw)
@@ -60,3 +61,16 @@ def test_ragged_rows():
     lens = np.diff(p.row_ptr)
     assert lens.min() == 0 and lens.max() == 12
     assert abs(lens.mean() - 6) < 0.5
+
+
+def test_dense_rows_and_linear_labels():
+    # every example holds every feature; the labels are w*.x plus N(0, 0.1^2)
+    # noise, so a least-squares fit recovers w* and leaves residuals of
+    # standard deviation ~0.1
+    p = synthdata.generate("dense-lr", n_rows=3000, n_cols=200, k=200)
+    X = p.val.reshape(p.n_rows, 200).astype(np.float64)
+    assert np.array_equal(p.col.reshape(p.n_rows, 200), np.tile(np.arange(200), (p.n_rows, 1)))
+    coef, *_ = np.linalg.lstsq(X, p.y.astype(np.float64), rcond=None)
+    resid = p.y - X @ coef
+    assert 0.09 < np.std(resid) < 0.11
+    assert 0.8 < np.std(coef) < 1.2          # w* ~ N(0, 1)
