@@ -110,23 +110,57 @@ __global__ void k_slots(const uint32_t *__restrict__ skey, const int32_t *__rest
     const bool check_dup = *(volatile int *)(info + INFO_UNSORTED) != 0;
     int longest = 0, n_near = 0;
     bool dup = false, big = false;
-    for (int64_t s = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; s < nnz; s += (int64_t)gridDim.x * blockDim.x) {
-        const uint32_t j = skey[s];
-        const int32_t p = spos[s];
-        const bool last = s == nnz - 1 || skey[s + 1] != j;
-        const int64_t r = s - feat_ptr[j];
-        const bool near_prev = r > 0 && (int64_t)p - spos[s - 1] < near;
-        const bool near_next = !last && (int64_t)spos[s + 1] - p < near;
-        big |= r > (int64_t)GATE_RANK;
-        n_near += near_next;
-        const uint32_t g = ((uint32_t)r & GATE_RANK) | (near_next ? GATE_NEAR_NEXT : 0u) |
-                           (near_prev ? GATE_NEAR_PREV : 0u) | (last ? GATE_LAST : 0u);
-        if (gsort)
-            gsort[s] = g;
-        else
-            gate[p] = g;
-        if (last) longest = max(longest, (int)(r + 1));
-        if (check_dup && r > 0) dup |= find_row(row_ptr, n_rows, spos[s - 1]) == find_row(row_ptr, n_rows, p);
+    // four consecutive slots per thread and iteration (16-byte loads and
+    // stores; the buffers come from the pool, 256-byte aligned), with the
+    // neighbours on both sides
+    const int64_t groups = (nnz + 3) >> 2;
+    for (int64_t gi = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; gi < groups;
+         gi += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t s0 = gi << 2;
+        uint32_t kk[6];
+        int32_t pp[6];
+        if (s0 + 4 <= nnz) {
+            const uint4 k4 = __ldcs(reinterpret_cast<const uint4 *>(skey) + gi);
+            const int4 p4 = __ldcs(reinterpret_cast<const int4 *>(spos) + gi);
+            kk[1] = k4.x; kk[2] = k4.y; kk[3] = k4.z; kk[4] = k4.w;
+            pp[1] = p4.x; pp[2] = p4.y; pp[3] = p4.z; pp[4] = p4.w;
+        } else {
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                kk[e + 1] = s0 + e < nnz ? skey[s0 + e] : 0xffffffffu;
+                pp[e + 1] = s0 + e < nnz ? spos[s0 + e] : 0;
+            }
+        }
+        kk[0] = s0 > 0 ? skey[s0 - 1] : 0xffffffffu;
+        pp[0] = s0 > 0 ? spos[s0 - 1] : 0;
+        kk[5] = s0 + 4 < nnz ? skey[s0 + 4] : 0xffffffffu;
+        pp[5] = s0 + 4 < nnz ? spos[s0 + 4] : 0;
+        uint32_t g[4] = {0u, 0u, 0u, 0u};
+        int64_t r = 0;
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            const int64_t s = s0 + e;
+            if (s >= nnz) break;
+            const uint32_t j = kk[e + 1];
+            const int32_t p = pp[e + 1];
+            const bool last = s == nnz - 1 || kk[e + 2] != j;
+            r = (e > 0 && kk[e] == j) ? r + 1 : s - feat_ptr[j];
+            const bool near_prev = r > 0 && (int64_t)p - pp[e] < near;
+            const bool near_next = !last && (int64_t)pp[e + 2] - p < near;
+            big |= r > (int64_t)GATE_RANK;
+            n_near += near_next;
+            g[e] = ((uint32_t)r & GATE_RANK) | (near_next ? GATE_NEAR_NEXT : 0u) |
+                   (near_prev ? GATE_NEAR_PREV : 0u) | (last ? GATE_LAST : 0u);
+            if (!gsort) gate[p] = g[e];
+            if (last) longest = max(longest, (int)(r + 1));
+            if (check_dup && r > 0) dup |= find_row(row_ptr, n_rows, pp[e]) == find_row(row_ptr, n_rows, p);
+        }
+        if (gsort) {
+            if (s0 + 4 <= nnz)
+                __stcs(reinterpret_cast<uint4 *>(gsort) + gi, make_uint4(g[0], g[1], g[2], g[3]));
+            else
+                for (int e = 0; e < 4 && s0 + e < nnz; ++e) gsort[s0 + e] = g[e];
+        }
     }
     for (int off = 16; off >= 1; off >>= 1) {
         longest = max(longest, __shfl_xor_sync(FULL, longest, off));
@@ -467,7 +501,7 @@ int pdb_build_conflicts(const pdb_csr *X, pdb_conflicts **out, void *stream)
         // order (k_scatter_block)
         const int pbits = bits_for(nnz - 1);
         const bool partition = pbits > 22;
-        k_slots<<<grid_1d(nnz), 256, 0, s>>>(skey, c->csc_pos, nnz, c->feat_ptr, X->row_ptr, N, c->near, c->gate,
+        k_slots<<<grid_1d((nnz + 3) / 4), 256, 0, s>>>(skey, c->csc_pos, nnz, c->feat_ptr, X->row_ptr, N, c->near, c->gate,
                                              partition ? (uint32_t *)tval : nullptr, c->info);
         note_launch();
         if (partition) {

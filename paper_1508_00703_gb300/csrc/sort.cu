@@ -243,6 +243,7 @@ __global__ __launch_bounds__(RS_THREADS, 3) void k_rs_scatter(const uint32_t *__
     for (int d = tid; d < RADIX; d += RS_THREADS) s_base[d] = offs[(int64_t)blockIdx.x * RADIX + d];
     __syncthreads();
     const unsigned lt = lanemask_lt();
+    const bool full = ntile == RS_TILE;     // every tile but the last: no invalid lanes
     // 1. lanes holding the same digit, for all the thread's elements at once
     //    (one ballot per digit bit plus the valid bit, intersected; the
     //    ballots of different elements are independent, so they overlap):
@@ -253,7 +254,7 @@ __global__ __launch_bounds__(RS_THREADS, 3) void k_rs_scatter(const uint32_t *__
         const int idx = wbase + i * 32 + lane;
         const bool valid = idx < ntile;
         const unsigned d = valid ? ((key[i] >> shift) & MASK) : (unsigned)RADIX;
-        unsigned peers = __ballot_sync(FULL, valid);
+        unsigned peers = full ? FULL : __ballot_sync(FULL, valid);
         if (!valid) peers = ~peers;
 #pragma unroll
         for (int b = 0; b < D; ++b) {
@@ -423,17 +424,35 @@ int radix_sort_bits(const uint32_t *keys_in, const int32_t *vals_in, uint32_t *k
 }
 
 // ------------------------------------------------------------------ segment bounds
+// ptr[b] = first index whose key is >= b, for b in 0..n_bins (keys sorted);
+// four consecutive keys per thread and iteration
 __global__ void k_segment_bounds(const uint32_t *__restrict__ keys, int64_t n, int64_t n_bins, const int *n_bins_dev,
                                  int64_t *__restrict__ ptr, const int *status)
 {
     if (read_status(status)) return;
     const int64_t nb = n_bins_dev ? (int64_t)*n_bins_dev : n_bins;
-    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
-        int64_t k = keys[i];
-        int64_t kp = i == 0 ? -1 : (int64_t)keys[i - 1];
-        for (int64_t b = kp + 1; b <= k && b <= nb; ++b) ptr[b] = i;
-        if (i == n - 1)
-            for (int64_t b = k + 1; b <= nb; ++b) ptr[b] = n;
+    const bool vec = ((uintptr_t)keys & 15) == 0;
+    const int64_t groups = (n + 3) >> 2;
+    for (int64_t gi = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; gi < groups;
+         gi += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t i0 = gi << 2;
+        int64_t k[5];
+        k[0] = i0 == 0 ? -1 : (int64_t)keys[i0 - 1];
+        if (vec && i0 + 4 <= n) {
+            const uint4 k4 = __ldcs(reinterpret_cast<const uint4 *>(keys) + gi);
+            k[1] = k4.x; k[2] = k4.y; k[3] = k4.z; k[4] = k4.w;
+        } else {
+#pragma unroll
+            for (int e = 0; e < 4; ++e) k[e + 1] = i0 + e < n ? (int64_t)keys[i0 + e] : nb;
+        }
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            const int64_t i = i0 + e;
+            if (i >= n) break;
+            for (int64_t b = k[e] + 1; b <= k[e + 1] && b <= nb; ++b) ptr[b] = i;
+            if (i == n - 1)
+                for (int64_t b = k[e + 1] + 1; b <= nb; ++b) ptr[b] = n;
+        }
     }
 }
 
@@ -450,7 +469,7 @@ int segment_bounds(const uint32_t *sorted_keys, int64_t n, int64_t n_bins, const
     if (n == 0) {
         k_fill_i64<<<64, 256, 0, s>>>(ptr, n_bins, n_bins_dev, 0); note_launch();
     } else {
-        int64_t blocks = std::min<int64_t>((n + 255) / 256, 65536);
+        int64_t blocks = std::min<int64_t>((n + 1023) / 1024, 65536);
         k_segment_bounds<<<(unsigned)blocks, 256, 0, s>>>(sorted_keys, n, n_bins, n_bins_dev, ptr, status); note_launch();
     }
     return cudaPeekAtLastError() == cudaSuccess ? PDB_OK : PDB_ECUDA;
