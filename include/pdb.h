@@ -90,7 +90,10 @@ typedef enum { PDB_LOSS_LOGISTIC = 0, PDB_LOSS_SQUARED = 1, PDB_LOSS_HINGE = 2 }
  *           r reads w_j once the iteration number of j equals r and
  *           publishes r + 1 with its write (the read protocol of Section 5
  *           with the iteration number counted per feature); no barrier at
- *           all.  The number lives in the same 64-bit word as the weight.
+ *           all.  The number lives in the same 64-bit word as the weight,
+ *           with an epoch stamp: all epochs run in one pipelined launch,
+ *           each feature's next-epoch occurrences starting as soon as its
+ *           last occurrence of the epoch has written.
  *   CHAIN   for conflict graphs that are close to one chain (a feature in
  *           most examples): one thread block runs the examples strictly in
  *           data order (Algorithm 1 itself), prefetching ids, values and
@@ -206,8 +209,9 @@ int pdb_schedule_levels(const pdb_schedule *s, const int32_t **level, const int3
  * occurrence rank), bit 29 set when the next occurrence of its feature lies
  * within the build's `near` distance, bit 30 when the previous one does,
  * bit 31 on the last occurrence of its feature; and, READY only,
- * records[n_cols] (weight bits | version << 32, meaningful while
- * pdb_sgd_epoch runs; NULL under WINDOW).  PDB_ESTATE for LEVELS and CHAIN
+ * records[n_cols] (weight bits | version << 32, the version being the rank
+ * waited for in bits 0..28 and an epoch stamp 1..7 in bits 29..31;
+ * meaningful while pdb_sgd_epoch runs; NULL under WINDOW).  PDB_ESTATE for LEVELS and CHAIN
  * schedules. */
 int pdb_schedule_ready(const pdb_schedule *s, const uint32_t **gate, const uint64_t **records);
 

@@ -107,13 +107,20 @@ __global__ __launch_bounds__(THREADS) void k_sgd_levels(int32_t n_rows, const in
 // both checks the version and returns the weight written with it (Read
 // Constraint: the previous writer is done) -- and publishes the new weight
 // together with version r + 1 in one 64-bit store (Write Constraint: its own
-// read, the only read of that version, came first).  The last occurrence of
-// j in the epoch (GATE_LAST) writes version 0 for the next epoch.  Both
-// halves travel in one single-copy-atomic access, so no fence is needed.
-// Examples are taken in data order from a ticket counter, `chunk`
-// consecutive ones at a time and run in order by the warp that took them,
-// so the oldest unfinished example never waits on a younger one and the
-// kernel cannot deadlock whatever the number of resident warps.
+// read, the only read of that version, came first).  Both halves travel in
+// one single-copy-atomic access, so no fence is needed.
+// All epochs run in one launch, pipelined: a version carries the epoch's
+// stamp (1..7, bits 29-31 above the 29-bit rank), and the last occurrence
+// of j in an epoch (GATE_LAST) publishes version 0 with the next epoch's
+// stamp, so the next epoch's first occurrence of j starts as soon as that
+// write lands -- not at a kernel boundary (exact by Theorem 2: per feature
+// the order is still the data order, epoch after epoch).  A record only
+// ever holds a version of the current or the previous epoch of its
+// feature, so stamps that repeat every 7 epochs never match stale ones.
+// Examples are taken in data order (epoch-major) from a ticket counter,
+// `chunk` consecutive ones at a time and run in order by the warp that took
+// them, so the oldest unfinished example never waits on a younger one and
+// the kernel cannot deadlock whatever the number of resident warps.
 __device__ __forceinline__ unsigned long long ld_rec(const unsigned long long *p)
 {
     unsigned long long v;
@@ -168,8 +175,11 @@ __device__ __forceinline__ bool gather_ready(const unsigned long long *rec, cons
 }
 
 // one example under the ready protocol; false when a wait gave up
+__host__ __device__ __forceinline__ unsigned epoch_stamp(int64_t e) { return (1u + (unsigned)(e % 7)) << 29; }
+
 template <int R>
-__device__ __forceinline__ bool ready_example(int t, const int64_t *__restrict__ row_ptr,
+__device__ __forceinline__ bool ready_example(int t, unsigned stamp, unsigned next_stamp,
+                                              const int64_t *__restrict__ row_ptr,
                                               const int32_t *__restrict__ col, const float *__restrict__ val,
                                               const float *__restrict__ y, const uint32_t *__restrict__ gate,
                                               unsigned long long *rec, int loss, float eta, int *status,
@@ -189,8 +199,8 @@ __device__ __forceinline__ bool ready_example(int t, const int64_t *__restrict__
             j[r] = i < k ? col[b + i] : 0;
             x[r] = i < k ? (val ? val[b + i] : 1.0f) : 0.0f;
             uint32_t g = i < k ? gate[b + i] : 0u;
-            want[r] = g & GATE_RANK;
-            next[r] = (g & GATE_LAST) ? 0u : want[r] + 1u;
+            want[r] = (g & GATE_RANK) | stamp;
+            next[r] = (g & GATE_LAST) ? next_stamp : want[r] + 1u;
             wv[r] = 0.0f;
         }
         bool ok = gather_ready<R>(rec, j, want, wv, lane, k, status, timeout);
@@ -213,7 +223,7 @@ __device__ __forceinline__ bool ready_example(int t, const int64_t *__restrict__
     bool ok = true;
     for (int i = lane; i < k && ok; i += 32) {
         int j1[1] = {col[b + i]};
-        unsigned w1[1] = {gate[b + i] & GATE_RANK};
+        unsigned w1[1] = {(gate[b + i] & GATE_RANK) | stamp};
         float v1[1];
         ok = gather_ready<1>(rec, j1, w1, v1, 0, 1, status, timeout);
         if (ok) acc = __fmaf_rn(v1[0], val ? val[b + i] : 1.0f, acc);
@@ -226,7 +236,7 @@ __device__ __forceinline__ bool ready_example(int t, const int64_t *__restrict__
         const float xx = val ? val[b + i] : 1.0f;
         const uint32_t g = gate[b + i];
         const float wo = __uint_as_float((unsigned)ld_rec(rec + jj));
-        st_rec(rec + jj, __fsub_rn(wo, __fmul_rn(c, xx)), (g & GATE_LAST) ? 0u : (g & GATE_RANK) + 1u);
+        st_rec(rec + jj, __fsub_rn(wo, __fmul_rn(c, xx)), (g & GATE_LAST) ? next_stamp : ((g & GATE_RANK) + 1u) | stamp);
     }
     return true;
 }
@@ -235,29 +245,36 @@ template <int R>
 __global__ __launch_bounds__(THREADS) void k_sgd_ready(int32_t n_rows, const int64_t *__restrict__ row_ptr,
                                                        const int32_t *__restrict__ col, const float *__restrict__ val,
                                                        const float *__restrict__ y, const uint32_t *__restrict__ gate,
-                                                       unsigned long long *rec, int loss, float eta,
+                                                       unsigned long long *rec, int loss, float eta, int epochs,
                                                        unsigned long long *ticket, int chunk, int *status,
                                                        uint64_t timeout)
 {
     if (read_status(status)) return;
     const int lane = threadIdx.x & 31;
+    const int64_t total = (int64_t)epochs * n_rows;     // examples of all epochs, epoch-major
     for (;;) {
         unsigned long long tk = 0;
         if (lane == 0) tk = atomicAdd(ticket, (unsigned long long)chunk);
         tk = __shfl_sync(FULL, tk, 0);
-        if (tk >= (unsigned long long)n_rows) return;
-        const int t1 = (int)min64((int64_t)n_rows, (int64_t)tk + chunk);
-        for (int t = (int)tk; t < t1; ++t)
-            if (!ready_example<R>(t, row_ptr, col, val, y, gate, rec, loss, eta, status, timeout)) return;
+        if (tk >= (unsigned long long)total) return;
+        const int64_t t1 = min64(total, (int64_t)tk + chunk);
+        for (int64_t tg = (int64_t)tk; tg < t1; ++tg) {
+            const int64_t e = tg / n_rows;
+            if (!ready_example<R>((int)(tg - e * n_rows), epoch_stamp(e), epoch_stamp(e + 1), row_ptr, col, val, y,
+                                  gate, rec, loss, eta, status, timeout))
+                return;
+        }
     }
 }
 
-// rec[j] = (w_j, version 0) before the first epoch; w_j back after the last
+// rec[j] = (w_j, version 0 of the first epoch) before the first epoch; w_j
+// back after the last
 __global__ void k_pack(const float *__restrict__ w, int64_t n, unsigned long long *__restrict__ rec, const int *status)
 {
     if (read_status(status)) return;
+    const unsigned long long v0 = (unsigned long long)epoch_stamp(0) << 32;
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x)
-        rec[i] = (unsigned long long)__float_as_uint(w[i]);
+        rec[i] = (unsigned long long)__float_as_uint(w[i]) | v0;
 }
 
 __global__ void k_unpack(const unsigned long long *__restrict__ rec, int64_t n, float *__restrict__ w,
@@ -431,12 +448,10 @@ int pdb_sgd_epoch(const pdb_csr *X, const float *y, const pdb_conflicts *c, cons
             k_pack<<<grid_1d(F), 256, 0, s>>>(w, F, h->rec, cm->status);
             note_launch();
             cudaEventRecord(cm->ev_k0, s);
-            for (int ep = 0; ep < n_epochs; ++ep) {
-                cudaMemsetAsync(h->ticket, 0, sizeof(unsigned long long), s);
-                kern<<<grid, THREADS, 0, s>>>(n32, X->row_ptr, X->col, X->val, y, c->gate, h->rec, lossi, eta,
-                                              h->ticket, chunk, cm->status, tmo);
-                note_launch();
-            }
+            cudaMemsetAsync(h->ticket, 0, sizeof(unsigned long long), s);
+            kern<<<grid, THREADS, 0, s>>>(n32, X->row_ptr, X->col, X->val, y, c->gate, h->rec, lossi, eta, n_epochs,
+                                          h->ticket, chunk, cm->status, tmo);
+            note_launch();
             cudaEventRecord(cm->ev_k1, s);
             k_unpack<<<grid_1d(F), 256, 0, s>>>(h->rec, F, w, cm->status);
             note_launch();
@@ -623,12 +638,10 @@ extern "C" int pdb_sgd_epoch_ready_noalloc(const pdb_csr *X, const float *y, con
             k_pack<<<grid_1d(F), 256, 0, s>>>(w, F, rec, status);
             note_launch();
         }
-        for (int ep = 0; ep < n_epochs; ++ep) {
-            cudaMemsetAsync(ticket, 0, sizeof(unsigned long long), s);
-            k_sgd_ready<8><<<grid, THREADS, 0, s>>>(n32, X->row_ptr, X->col, X->val, y, gate, rec, (int)loss, eta,
-                                                    ticket, 2, status, tmo);
-            note_launch();
-        }
+        cudaMemsetAsync(ticket, 0, sizeof(unsigned long long), s);
+        k_sgd_ready<8><<<grid, THREADS, 0, s>>>(n32, X->row_ptr, X->col, X->val, y, gate, rec, (int)loss, eta,
+                                                n_epochs, ticket, 2, status, tmo);
+        note_launch();
         if (F > 0) {
             k_unpack<<<grid_1d(F), 256, 0, s>>>(rec, F, w, status);
             note_launch();
