@@ -18,6 +18,7 @@
  *   Theorem 2      RC + WC give the sequential result
  *   Theorem 3      BSP executions are a subset of RC/WC executions
  *   Section 5      read protocol: a per-chunk iteration number gates reads
+ *   Section 7      admissible delay: reads and writes within delta iterations
  *
  * Conventions for every call:
  *   - Pointers named as device pointers must be device memory of the current
