@@ -32,6 +32,9 @@ int grid_1d(int64_t n);                               // blocks of 256 threads f
 // chain engine (chain.cu)
 int chain_max_row();
 int64_t resident_smem(int64_t n_cols, int64_t max_row);   // 0 when the weights do not fit in one block
+int64_t block_ready_smem(int64_t n_cols, int64_t max_row);   // 0 when the records do not fit in one block
+int block_ready_run(const pdb_csr *X, const float *y, const uint32_t *gate, float *w, int loss, float eta,
+                    int epochs, int max_row, int *status, uint64_t timeout, cudaStream_t s);
 int resident_run(const pdb_csr *X, const float *y, float *w, int loss, float eta, int epochs, int max_row,
                  int *status, cudaStream_t s);
 int chain_schedule(const int32_t *prev, const int32_t *next, const int32_t *row_of, const int64_t *row_ptr,

@@ -443,6 +443,11 @@ int pdb_sgd_epoch(const pdb_csr *X, const float *y, const pdb_conflicts *c, cons
             rc = window_run(X, y, c->gate, w, h->rec, &hm->epochs_run, h->prog, h->prog_cap, h->wctl, c->near, lossi,
                             eta, n_epochs, width, opts, cm->status, tmo, s);
             cudaEventRecord(cm->ev_k1, s);
+        } else if (block_ready_smem(X->n_cols, c->h_info[2]) > 0 && (int64_t)n_epochs * X->n_rows < (1ll << 31)) {
+            // READY with every record in one block's shared memory (few features)
+            cudaEventRecord(cm->ev_k0, s);
+            rc = block_ready_run(X, y, c->gate, w, lossi, eta, n_epochs, c->h_info[2], cm->status, tmo, s);
+            cudaEventRecord(cm->ev_k1, s);
         } else {
             auto kern = width == 2 ? k_sgd_ready<2> : width == 4 ? k_sgd_ready<4> : k_sgd_ready<8>;
             int grid = persistent_grid((const void *)kern, opts);
