@@ -90,7 +90,7 @@ class pdb_csr(ctypes.Structure):
 
 class pdb_opts(ctypes.Structure):
     _fields_ = [("blocks_per_sm", ctypes.c_int32), ("ticket_chunk", ctypes.c_int32),
-                ("wait_timeout_s", ctypes.c_double)]
+                ("wait_timeout_s", ctypes.c_double), ("trace", ctypes.c_void_p)]
 
 
 class pdb_stats(ctypes.Structure):
@@ -252,7 +252,10 @@ def _opts(opts):
         return None
     if isinstance(opts, pdb_opts):
         return ctypes.byref(opts)
-    return ctypes.byref(pdb_opts(**opts))
+    kw = dict(opts)
+    if kw.get("trace") is not None and not isinstance(kw["trace"], int):
+        kw["trace"] = kw["trace"].data_ptr()     # a torch uint64/int64 tensor on the device
+    return ctypes.byref(pdb_opts(**kw))
 
 
 def pdb_sgd_epoch(X: Csr, y, c: Conflicts, s: Schedule, w, loss: int, eta: float, n_epochs: int, opts=None,

@@ -106,7 +106,7 @@ __global__ __launch_bounds__(BR_THREADS, 1) void k_sgd_block_ready(int32_t n_row
                                                                    const float *__restrict__ y,
                                                                    const uint32_t *__restrict__ gate, float *w,
                                                                    int loss, float eta, int epochs, int *status,
-                                                                   uint64_t timeout)
+                                                                   uint64_t timeout, uint64_t *trace)
 {
     extern __shared__ __align__(16) unsigned char smem_raw[];
     unsigned long long *rec = reinterpret_cast<unsigned long long *>(smem_raw);
@@ -173,12 +173,14 @@ __global__ __launch_bounds__(BR_THREADS, 1) void k_sgd_block_ready(int32_t n_row
             }
         }
         if (__any_sync(FULL, failed)) break;     // every warp still reaches the barrier below
+        trace_mark(trace, cur.tg, 0);
         float acc = 0.0f;
 #pragma unroll
         for (int r = 0; r < BR_R; ++r)
             if (r * 32 + lane < cur.k) acc = __fmaf_rn(wv[r], cur.x[r], acc);
         const float m = warp_combine(acc);
         const float c = __fmul_rn(eta, dev_grad(loss, m, cur.y));
+        trace_mark(trace, cur.tg, 1);   // before any write is visible
 #pragma unroll
         for (int r = 0; r < BR_R; ++r)
             if (r * 32 + lane < cur.k) {
@@ -211,7 +213,7 @@ int64_t block_ready_smem(int64_t n_cols, int64_t max_row)
 }
 
 int block_ready_run(const pdb_csr *X, const float *y, const uint32_t *gate, float *w, int loss, float eta,
-                    int epochs, int max_row, int *status, uint64_t timeout, cudaStream_t s)
+                    int epochs, int max_row, int *status, uint64_t timeout, uint64_t *trace, cudaStream_t s)
 {
     const int64_t smem = block_ready_smem(X->n_cols, max_row);
     if (smem == 0) return PDB_ETOOBIG;
@@ -219,7 +221,7 @@ int block_ready_run(const pdb_csr *X, const float *y, const uint32_t *gate, floa
         cudaSuccess)
         return PDB_ECUDA;
     k_sgd_block_ready<<<1, BR_THREADS, (size_t)smem, s>>>((int32_t)X->n_rows, X->n_cols, X->row_ptr, X->col,
-                                                          X->val, y, gate, w, loss, eta, epochs, status, timeout);
+                                                          X->val, y, gate, w, loss, eta, epochs, status, timeout, trace);
     note_launch();
     return cudaPeekAtLastError() == cudaSuccess ? PDB_OK : PDB_ECUDA;
 }

@@ -156,7 +156,8 @@ __global__ __launch_bounds__(CH_THREADS, 1) void k_sgd_chain(int32_t n_rows, con
                                                              const float *__restrict__ val,
                                                              const float *__restrict__ y,
                                                              const uint32_t *__restrict__ link, float *w, int loss,
-                                                             float eta, int epochs, bool vec, int *status)
+                                                             float eta, int epochs, bool vec, int *status,
+                                                             uint64_t *trace)
 {
     extern __shared__ __align__(16) unsigned char smem_raw[];
     ChainSmem &S = *reinterpret_cast<ChainSmem *>(smem_raw);
@@ -247,7 +248,9 @@ __global__ __launch_bounds__(CH_THREADS, 1) void k_sgd_chain(int32_t n_rows, con
                         }
                     }
                     const float m = combine_smem(acc, S.part);
+                    trace_mark(trace, (int64_t)ep * N + r, 0);
                     const float c = __fmul_rn(eta, dev_grad(loss, m, yr));
+                    trace_mark(trace, (int64_t)ep * N + r, 1);   // before any write is visible
 #pragma unroll
                     for (int q = 0; q < R; ++q) {
                         const int i = q * 32 + lane;
@@ -307,7 +310,7 @@ int chain_schedule(const int32_t *prev, const int32_t *next, const int32_t *row_
 }
 
 int chain_run(const pdb_csr *X, const float *y, const uint32_t *link, float *w, int loss, float eta, int epochs,
-              int max_row, int *status, cudaStream_t s)
+              int max_row, int *status, uint64_t *trace, cudaStream_t s)
 {
     // registers per lane for the longest example: 1, 2, 4 or 8 (32 to 256 ids)
     auto kern = max_row <= 32 ? k_sgd_chain<1> : max_row <= 64 ? k_sgd_chain<2>
@@ -325,7 +328,7 @@ int chain_run(const pdb_csr *X, const float *y, const uint32_t *link, float *w, 
     // 16-byte row copies need 16-byte aligned ids, values and link words
     const bool vec = ((uintptr_t)X->col & 15) == 0 && ((uintptr_t)X->val & 15) == 0 && ((uintptr_t)link & 15) == 0;
     kern<<<1, CH_THREADS, sizeof(ChainSmem), s>>>((int32_t)X->n_rows, X->row_ptr, X->col, X->val, y, link, w, loss,
-                                                  eta, epochs, vec, status);
+                                                  eta, epochs, vec, status, trace);
     note_launch();
     return cudaPeekAtLastError() == cudaSuccess ? PDB_OK : PDB_ECUDA;
 }

@@ -34,13 +34,13 @@ int chain_max_row();
 int64_t resident_smem(int64_t n_cols, int64_t max_row);   // 0 when the weights do not fit in one block
 int64_t block_ready_smem(int64_t n_cols, int64_t max_row);   // 0 when the records do not fit in one block
 int block_ready_run(const pdb_csr *X, const float *y, const uint32_t *gate, float *w, int loss, float eta,
-                    int epochs, int max_row, int *status, uint64_t timeout, cudaStream_t s);
+                    int epochs, int max_row, int *status, uint64_t timeout, uint64_t *trace, cudaStream_t s);
 int resident_run(const pdb_csr *X, const float *y, float *w, int loss, float eta, int epochs, int max_row,
-                 int *status, cudaStream_t s);
+                 int *status, uint64_t *trace, cudaStream_t s);
 int chain_schedule(const int32_t *prev, const int32_t *next, const int32_t *row_of, const int64_t *row_ptr,
                    int64_t nnz, uint32_t *link, const int *status, cudaStream_t s);
 int chain_run(const pdb_csr *X, const float *y, const uint32_t *link, float *w, int loss, float eta, int epochs,
-              int max_row, int *status, cudaStream_t s);
+              int max_row, int *status, uint64_t *trace, cudaStream_t s);
 void note_launch();                                   // count one kernel launch (pdb_launch_count)
 
 // Stable LSD radix sort of (key, value) pairs, 8-bit digits.  vals_in ==
@@ -175,6 +175,19 @@ __device__ __forceinline__ float dev_expf(float x)
     float s1 = __int_as_float((h + 127) << 23);
     float s2 = __int_as_float((k2 + 127) << 23);
     return __fmul_rn(__fmul_rn(p, s1), s2);
+}
+
+// execution trace (pdb_opts.trace): lane 0 stamps %globaltimer into
+// trace[2 * idx + which] (idx = epoch * n_rows + example), which = 0 once
+// every weight the example reads has been read, which = 1 once its update is
+// computed and before any of its writes is issued.  Called by the whole warp;
+// the __syncwarp keeps the other lanes' later writes after the stamp.
+__device__ __forceinline__ void trace_mark(uint64_t *trace, int64_t idx, int which)
+{
+    if (trace) {
+        if ((threadIdx.x & 31) == 0) trace[2 * idx + which] = globaltimer();
+        __syncwarp();
+    }
 }
 
 // derivative of the example's loss with respect to its margin m

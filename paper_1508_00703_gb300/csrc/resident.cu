@@ -121,7 +121,8 @@ __global__ __launch_bounds__(RZ_THREADS, 1) void k_sgd_resident(int32_t n_rows, 
                                                                 const int32_t *__restrict__ col,
                                                                 const float *__restrict__ val,
                                                                 const float *__restrict__ y, float *w, int loss,
-                                                                float eta, int epochs, bool vec, int *status)
+                                                                float eta, int epochs, bool vec, int *status,
+                                                                uint64_t *trace)
 {
     extern __shared__ __align__(16) unsigned char smem_raw[];
     if (read_status(status)) return;
@@ -188,7 +189,9 @@ __global__ __launch_bounds__(RZ_THREADS, 1) void k_sgd_resident(int32_t n_rows, 
                         }
                     }
                     const float m = combine_smem(acc, part);
+                    trace_mark(trace, rg, 0);
                     const float c = __fmul_rn(eta, dev_grad(loss, m, yr));
+                    trace_mark(trace, rg, 1);   // before any write is visible
 #pragma unroll
                     for (int q = 0; q < R; ++q)
                         if (q * 32 + lane < k) ws[j[q]] = __fsub_rn(wv[q], __fmul_rn(c, x[q]));
@@ -214,7 +217,9 @@ __global__ __launch_bounds__(RZ_THREADS, 1) void k_sgd_resident(int32_t n_rows, 
                             if (base + u * 32 + lane < k) acc = __fmaf_rn(wv[u], x[u], acc);
                     }
                     const float m = combine_smem(acc, part);
+                    trace_mark(trace, rg, 0);
                     const float c = __fmul_rn(eta, dev_grad(loss, m, yr));
+                    trace_mark(trace, rg, 1);   // before any write is visible
                     for (int base = 0; base < k; base += 32 * RZ_U) {
                         int j[RZ_U];
                         float x[RZ_U], wv[RZ_U];
@@ -264,7 +269,7 @@ int64_t resident_smem(int64_t n_cols, int64_t max_row)
 }
 
 int resident_run(const pdb_csr *X, const float *y, float *w, int loss, float eta, int epochs, int max_row,
-                 int *status, cudaStream_t s)
+                 int *status, uint64_t *trace, cudaStream_t s)
 {
     const int64_t smem = resident_smem(X->n_cols, max_row);
     if (smem == 0) return PDB_ETOOBIG;
@@ -274,7 +279,7 @@ int resident_run(const pdb_csr *X, const float *y, float *w, int loss, float eta
         return PDB_ECUDA;
     const bool vec = ((uintptr_t)X->col & 15) == 0 && ((uintptr_t)X->val & 15) == 0;
     kern<<<1, RZ_THREADS, (size_t)smem, s>>>((int32_t)X->n_rows, X->n_cols, kcap_for(max_row), X->row_ptr, X->col,
-                                             X->val, y, w, loss, eta, epochs, vec, status);
+                                             X->val, y, w, loss, eta, epochs, vec, status, trace);
     note_launch();
     return cudaPeekAtLastError() == cudaSuccess ? PDB_OK : PDB_ECUDA;
 }

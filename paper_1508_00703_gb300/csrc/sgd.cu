@@ -29,7 +29,7 @@ namespace {
 template <int R>
 __device__ __forceinline__ void sgd_example(int t, const int64_t *__restrict__ row_ptr, const int32_t *__restrict__ col,
                                             const float *__restrict__ val, const float *__restrict__ y, float *w,
-                                            int loss, float eta)
+                                            int loss, float eta, uint64_t *trace, int64_t idx)
 {
     const int lane = threadIdx.x & 31;
     const int64_t b = row_ptr[t];
@@ -51,21 +51,26 @@ __device__ __forceinline__ void sgd_example(int t, const int64_t *__restrict__ r
 #pragma unroll
         for (int r = 0; r < R; ++r)
             if (r * 32 + lane < k) acc = __fmaf_rn(wv[r], x[r], acc);
-        const float m = warp_combine(acc);
+        const float m = warp_combine(acc);       // every lane's loads have returned
+        trace_mark(trace, idx, 0);
         const float c = __fmul_rn(eta, dev_grad(loss, m, yt));
+        trace_mark(trace, idx, 1);   // before any write is visible
 #pragma unroll
         for (int r = 0; r < R; ++r)
             if (r * 32 + lane < k) __stcg(w + j[r], __fsub_rn(wv[r], __fmul_rn(c, x[r])));
     } else {
         for (int i = lane; i < k; i += 32) acc = __fmaf_rn(__ldcg(w + col[b + i]), val ? val[b + i] : 1.0f, acc);
         const float m = warp_combine(acc);
+        trace_mark(trace, idx, 0);
         const float c = __fmul_rn(eta, dev_grad(loss, m, yt));
+        trace_mark(trace, idx, 1);   // before any write is visible
         for (int i = lane; i < k; i += 32) {
             int jj = col[b + i];
             float xx = val ? val[b + i] : 1.0f;
             __stcg(w + jj, __fsub_rn(__ldcg(w + jj), __fmul_rn(c, xx)));
         }
     }
+    __syncwarp();
 }
 
 // ---------------------------------------------------------------- level-synchronous engine
@@ -78,7 +83,7 @@ __global__ __launch_bounds__(THREADS) void k_sgd_levels(int32_t n_rows, const in
                                                         const float *__restrict__ y, const int32_t *__restrict__ order,
                                                         const int64_t *__restrict__ level_ptr, const LevelCtl *ctl,
                                                         float *w, int loss, float eta, int epochs, GridBarrier *bar,
-                                                        int *status, uint64_t timeout)
+                                                        int *status, uint64_t timeout, uint64_t *trace)
 {
     if (read_status(status)) return;
     const int L = ctl->n_levels;
@@ -93,7 +98,7 @@ __global__ __launch_bounds__(THREADS) void k_sgd_levels(int32_t n_rows, const in
                     set_status(status, PDB_EFAULT);
                     continue;
                 }
-                sgd_example<R>(t, row_ptr, col, val, y, w, loss, eta);
+                sgd_example<R>(t, row_ptr, col, val, y, w, loss, eta, trace, (int64_t)ep * n_rows + t);
             }
             if (!grid_sync(bar, status, timeout)) return;
         }
@@ -186,7 +191,7 @@ __device__ __forceinline__ bool ready_example(int t, unsigned stamp, unsigned ne
                                               const int32_t *__restrict__ col, const float *__restrict__ val,
                                               const float *__restrict__ y, const uint32_t *__restrict__ gate,
                                               unsigned long long *rec, int loss, float eta, int *status,
-                                              uint64_t timeout)
+                                              uint64_t timeout, uint64_t *trace, int64_t idx)
 {
     const int lane = threadIdx.x & 31;
     const int64_t b = row_ptr[t];
@@ -208,12 +213,14 @@ __device__ __forceinline__ bool ready_example(int t, unsigned stamp, unsigned ne
         }
         bool ok = gather_ready<R>(rec, j, want, wv, lane, k, status, timeout);
         if (!__all_sync(FULL, ok)) return false;
+        trace_mark(trace, idx, 0);
         float acc = 0.0f;
 #pragma unroll
         for (int r = 0; r < R; ++r)
             if (r * 32 + lane < k) acc = __fmaf_rn(wv[r], x[r], acc);
         const float m = warp_combine(acc);
         const float c = __fmul_rn(eta, dev_grad(loss, m, yt));
+        trace_mark(trace, idx, 1);   // before any write is visible
 #pragma unroll
         for (int r = 0; r < R; ++r)
             if (r * 32 + lane < k) st_rec(rec + j[r], __fsub_rn(wv[r], __fmul_rn(c, x[r])), next[r]);
@@ -232,8 +239,10 @@ __device__ __forceinline__ bool ready_example(int t, unsigned stamp, unsigned ne
         if (ok) acc = __fmaf_rn(v1[0], val ? val[b + i] : 1.0f, acc);
     }
     if (!__all_sync(FULL, ok)) return false;
+    trace_mark(trace, idx, 0);
     const float m = warp_combine(acc);
     const float c = __fmul_rn(eta, dev_grad(loss, m, yt));
+    trace_mark(trace, idx, 1);   // before any write is visible
     for (int i = lane; i < k; i += 32) {
         const int jj = col[b + i];
         const float xx = val ? val[b + i] : 1.0f;
@@ -250,7 +259,7 @@ __global__ __launch_bounds__(THREADS) void k_sgd_ready(int32_t n_rows, const int
                                                        const float *__restrict__ y, const uint32_t *__restrict__ gate,
                                                        unsigned long long *rec, int loss, float eta, int epochs,
                                                        unsigned long long *ticket, int chunk, int *status,
-                                                       uint64_t timeout)
+                                                       uint64_t timeout, uint64_t *trace)
 {
     if (read_status(status)) return;
     const int lane = threadIdx.x & 31;
@@ -264,7 +273,7 @@ __global__ __launch_bounds__(THREADS) void k_sgd_ready(int32_t n_rows, const int
         for (int64_t tg = (int64_t)tk; tg < t1; ++tg) {
             const int64_t e = tg / n_rows;
             if (!ready_example<R>((int)(tg - e * n_rows), epoch_stamp(e), epoch_stamp(e + 1), row_ptr, col, val, y,
-                                  gate, rec, loss, eta, status, timeout))
+                                  gate, rec, loss, eta, status, timeout, trace, tg))
                 return;
         }
     }
@@ -414,6 +423,7 @@ int pdb_sgd_epoch(const pdb_csr *X, const float *y, const pdb_conflicts *c, cons
     cudaEventRecord(cm->ev_k0, s);
     cudaEventRecord(cm->ev_k1, s);
     const uint64_t tmo = timeout_ns(opts);
+    uint64_t *trace = opts ? opts->trace : nullptr;
     int32_t n32 = (int32_t)X->n_rows;
     int lossi = (int)loss;
     if (X->n_rows > 0 && n_epochs > 0) {
@@ -427,15 +437,15 @@ int pdb_sgd_epoch(const pdb_csr *X, const float *y, const pdb_conflicts *c, cons
             void *args[] = {(void *)&n32,      (void *)&rp,  (void *)&cl,       (void *)&vl,     (void *)&y,
                             (void *)&h->order, (void *)&h->level_ptr, (void *)&h->ctl, (void *)&w,
                             (void *)&lossi,    (void *)&eta, (void *)&n_epochs, (void *)&h->bar,
-                            (void *)&cm->status, (void *)&tmo};
+                            (void *)&cm->status, (void *)&tmo, (void *)&trace};
             cudaEventRecord(cm->ev_k0, s);
             if (cudaLaunchCooperativeKernel(kern, grid, THREADS, args, 0, s) != cudaSuccess) rc = PDB_ECUDA;
             note_launch();
             cudaEventRecord(cm->ev_k1, s);
         } else if (h->mode == PDB_SCHED_CHAIN) {
             cudaEventRecord(cm->ev_k0, s);
-            rc = h->resident ? resident_run(X, y, w, lossi, eta, n_epochs, c->h_info[2], cm->status, s)
-                             : chain_run(X, y, h->link, w, lossi, eta, n_epochs, c->h_info[2], cm->status, s);
+            rc = h->resident ? resident_run(X, y, w, lossi, eta, n_epochs, c->h_info[2], cm->status, trace, s)
+                             : chain_run(X, y, h->link, w, lossi, eta, n_epochs, c->h_info[2], cm->status, trace, s);
             cudaEventRecord(cm->ev_k1, s);
         } else if (h->mode == PDB_SCHED_WINDOW) {
             cudaEventRecord(cm->ev_k0, s);
@@ -446,7 +456,7 @@ int pdb_sgd_epoch(const pdb_csr *X, const float *y, const pdb_conflicts *c, cons
         } else if (block_ready_smem(X->n_cols, c->h_info[2]) > 0 && (int64_t)n_epochs * X->n_rows < (1ll << 31)) {
             // READY with every record in one block's shared memory (few features)
             cudaEventRecord(cm->ev_k0, s);
-            rc = block_ready_run(X, y, c->gate, w, lossi, eta, n_epochs, c->h_info[2], cm->status, tmo, s);
+            rc = block_ready_run(X, y, c->gate, w, lossi, eta, n_epochs, c->h_info[2], cm->status, tmo, trace, s);
             cudaEventRecord(cm->ev_k1, s);
         } else {
             auto kern = width == 2 ? k_sgd_ready<2> : width == 4 ? k_sgd_ready<4> : k_sgd_ready<8>;
@@ -458,7 +468,7 @@ int pdb_sgd_epoch(const pdb_csr *X, const float *y, const pdb_conflicts *c, cons
             cudaEventRecord(cm->ev_k0, s);
             cudaMemsetAsync(h->ticket, 0, sizeof(unsigned long long), s);
             kern<<<grid, THREADS, 0, s>>>(n32, X->row_ptr, X->col, X->val, y, c->gate, h->rec, lossi, eta, n_epochs,
-                                          h->ticket, chunk, cm->status, tmo);
+                                          h->ticket, chunk, cm->status, tmo, trace);
             note_launch();
             cudaEventRecord(cm->ev_k1, s);
             k_unpack<<<grid_1d(F), 256, 0, s>>>(h->rec, F, w, cm->status);
@@ -648,7 +658,7 @@ extern "C" int pdb_sgd_epoch_ready_noalloc(const pdb_csr *X, const float *y, con
         }
         cudaMemsetAsync(ticket, 0, sizeof(unsigned long long), s);
         k_sgd_ready<8><<<grid, THREADS, 0, s>>>(n32, X->row_ptr, X->col, X->val, y, gate, rec, (int)loss, eta,
-                                                n_epochs, ticket, 2, status, tmo);
+                                                n_epochs, ticket, 2, status, tmo, nullptr);
         note_launch();
         if (F > 0) {
             k_unpack<<<grid_1d(F), 256, 0, s>>>(rec, F, w, status);

@@ -94,7 +94,8 @@ __global__ __launch_bounds__(THREADS) void k_sgd_ssp(int32_t n_rows, const int64
                                                      const float *__restrict__ y, const uint32_t *__restrict__ gate,
                                                      float *w, unsigned *writes, unsigned *reads, long long delay,
                                                      float *coef, int loss, float eta, unsigned long long *ticket,
-                                                     int chunk, int *status, uint64_t timeout)
+                                                     int chunk, int *status, uint64_t timeout, uint64_t *trace,
+                                                     int64_t trace_base)
 {
     if (read_status(status)) return;
     const int lane = threadIdx.x & 31;
@@ -128,11 +129,13 @@ __global__ __launch_bounds__(THREADS) void k_sgd_ssp(int32_t n_rows, const int64
                         ok = read_admitted(w, writes, reads, j[r], rank[r] - delay, wv[r], status, timeout);
                     }
                 if (!__all_sync(FULL, ok)) return;
+                trace_mark(trace, trace_base + t, 0);
 #pragma unroll
                 for (int r = 0; r < R; ++r)
                     if (r * 32 + lane < k) acc = __fmaf_rn(wv[r], x[r], acc);
                 const float m = warp_combine(acc);
                 const float c = __fmul_rn(eta, dev_grad(loss, m, yt));
+                trace_mark(trace, trace_base + t, 1);   // before any write is visible
                 if (coef && lane == 0) coef[t] = c;
 #pragma unroll
                 for (int r = 0; r < R; ++r)
@@ -151,8 +154,10 @@ __global__ __launch_bounds__(THREADS) void k_sgd_ssp(int32_t n_rows, const int64
                 if (ok) acc = __fmaf_rn(v1, val ? val[b + i] : 1.0f, acc);
             }
             if (!__all_sync(FULL, ok)) return;
+            trace_mark(trace, trace_base + t, 0);
             const float m = warp_combine(acc);
             const float c = __fmul_rn(eta, dev_grad(loss, m, yt));
+            trace_mark(trace, trace_base + t, 1);   // before any write is visible
             if (coef && lane == 0) coef[t] = c;
             for (int i = lane; i < k && ok; i += 32)
                 ok = write_admitted(w, writes, reads, col[b + i], (long long)(gate[b + i] & GATE_RANK) - delay + 1,
@@ -181,7 +186,7 @@ int ssp_run(const pdb_csr *X, const float *y, const uint32_t *gate, float *w, un
         cudaMemsetAsync(ticket, 0, sizeof(unsigned long long), s);
         kern<<<grid, THREADS, 0, s>>>(n, X->row_ptr, X->col, X->val, y, gate, w, writes, reads, delay,
                                       coef ? coef + (int64_t)ep * n : nullptr, loss, eta, ticket, chunk, status,
-                                      timeout);
+                                      timeout, opts ? opts->trace : nullptr, (int64_t)ep * n);
         note_launch();
     }
     return cudaPeekAtLastError() == cudaSuccess ? PDB_OK : PDB_ECUDA;

@@ -180,7 +180,7 @@ __device__ __forceinline__ bool window_example(int t, int64_t floor_pos, const i
                                                float *w, unsigned long long *rec, unsigned stamp,
                                                const WindowCtl *ctl, int64_t near, int loss, float eta,
                                                long long &known, unsigned *slot, unsigned progress, int *status,
-                                               uint64_t timeout)
+                                               uint64_t timeout, uint64_t *trace, int64_t idx)
 {
     const int lane = threadIdx.x & 31;
     const int64_t b = row_ptr[t];
@@ -209,12 +209,14 @@ __device__ __forceinline__ bool window_example(int t, int64_t floor_pos, const i
         bool ok = !far || known >= need || wait_watermark(ctl, need, known, status, timeout);
         ok = ok && gather_window<R>(w, rec, j, g, stamp, wv, lane, k, status, timeout);
         if (!__all_sync(FULL, ok)) return false;
+        trace_mark(trace, idx, 0);
         float acc = 0.0f;
 #pragma unroll
         for (int r = 0; r < R; ++r)
             if (r * 32 + lane < k) acc = __fmaf_rn(wv[r], x[r], acc);
         const float m = warp_combine(acc);
         const float c = __fmul_rn(eta, dev_grad(loss, m, yt));
+        trace_mark(trace, idx, 1);   // before any write is visible
 #pragma unroll
         for (int r = 0; r < R; ++r)
             if (r * 32 + lane < k) publish(j[r], g[r], __fsub_rn(wv[r], __fmul_rn(c, x[r])), w, rec, stamp);
@@ -237,8 +239,10 @@ __device__ __forceinline__ bool window_example(int t, int64_t floor_pos, const i
         if (ok) acc = __fmaf_rn(v1[0], val ? val[b + i] : 1.0f, acc);
     }
     if (!__all_sync(FULL, ok)) return false;
+    trace_mark(trace, idx, 0);
     const float m = warp_combine(acc);
     const float c = __fmul_rn(eta, dev_grad(loss, m, yt));
+    trace_mark(trace, idx, 1);   // before any write is visible
     for (int i = lane; i < k; i += 32) {
         const int jj = col[b + i];
         const uint32_t gg = gate[b + i];
@@ -296,7 +300,8 @@ __global__ __launch_bounds__(THREADS) void k_sgd_window(int32_t n_rows, const in
                                                         const uint32_t *__restrict__ gate, float *w,
                                                         unsigned long long *rec, unsigned stamp, unsigned *prog,
                                                         WindowCtl *ctl, int64_t near, int loss, float eta, int chunk,
-                                                        int *status, uint64_t timeout)
+                                                        int *status, uint64_t timeout, uint64_t *trace,
+                                                        int64_t trace_base)
 {
     if (read_status(status)) return;
     const unsigned n_chunks = (unsigned)((n_rows + (int64_t)chunk - 1) / chunk);
@@ -320,7 +325,8 @@ __global__ __launch_bounds__(THREADS) void k_sgd_window(int32_t n_rows, const in
         const int64_t floor_pos = row_ptr[tk];
         for (int t = (int)tk; t < t1; ++t)
             if (!window_example<R>(t, floor_pos, row_ptr, col, val, y, gate, w, rec, stamp, ctl, near, loss, eta,
-                                   known, t == (int)tk ? slot : nullptr, (unsigned)(tk / chunk), status, timeout))
+                                   known, t == (int)tk ? slot : nullptr, (unsigned)(tk / chunk), status, timeout,
+                                   trace, trace_base + t))
                 return;
     }
 }
@@ -347,7 +353,8 @@ int window_run(const pdb_csr *X, const float *y, const uint32_t *gate, float *w,
         cudaMemsetAsync(prog, 0, sizeof(unsigned) * (size_t)(grid - 1) * WARPS, s);
         cudaMemsetAsync(ctl, 0, sizeof(WindowCtl), s);
         kern<<<grid, THREADS, 0, s>>>(n, X->row_ptr, X->col, X->val, y, gate, w, rec, stamp, prog, ctl, near, loss,
-                                      eta, chunk, status, timeout);
+                                      eta, chunk, status, timeout, opts ? opts->trace : nullptr,
+                                      (int64_t)ep * X->n_rows);
         note_launch();
     }
     return cudaPeekAtLastError() == cudaSuccess ? PDB_OK : PDB_ECUDA;
