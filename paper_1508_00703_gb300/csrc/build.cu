@@ -15,8 +15,10 @@
 // occurrence.  prev and next of a position follow from gate, feat_ptr and
 // csc_pos by gathers and are materialized only when a caller asks for them.
 #include <cuda_runtime.h>
+#include <nvtx3/nvToolsExt.h>
 
 #include <algorithm>
+#include <cstdio>
 #include <cstdlib>
 #include <cstring>
 #include <new>
@@ -397,6 +399,41 @@ int materialize_chains(pdb_conflicts *c, cudaStream_t s)
 }  // namespace
 
 // ------------------------------------------------------------------ C ABI
+namespace pdb {
+
+ApiScope::ApiScope(const char *name_, const pdb_conflicts *c_, const pdb_schedule *h_, pdb_conflicts *const *pc_,
+                   pdb_schedule *const *ph_, bool log_)
+    : name(name_), c(c_), h(h_), pc(pc_), ph(ph_), log(log_)
+{
+    nvtxRangePushA(name);
+}
+
+ApiScope::~ApiScope()
+{
+    nvtxRangePop();
+    const char *env = std::getenv("PDB_LOG");
+    if (!log || !env || !*env || std::strcmp(env, "0") == 0) return;
+    const pdb_conflicts *cc = pc ? *pc : c;
+    const pdb_schedule *hh = ph ? *ph : h;
+    if (!cc && hh) cc = hh->c;
+    pdb_stats st;
+    if (!cc || pdb_get_stats(cc, hh, &st) != PDB_OK) {
+        std::fprintf(stderr, "pdb %s: no handle\n", name);
+        return;
+    }
+    int status = 0;
+    cudaMemcpy(&status, cc->status, sizeof status, cudaMemcpyDeviceToHost);
+    std::fprintf(stderr,
+                 "pdb %s: n_rows=%lld n_cols=%lld nnz=%lld max_chain=%lld sched_mode=%lld n_levels=%lld "
+                 "max_level_width=%lld ms_build=%.3f ms_schedule=%.3f ms_sgd=%.3f ms_sgd_kernels=%.3f ms_bsp=%.3f "
+                 "status=%d launches=%lld\n",
+                 name, (long long)st.n_rows, (long long)st.n_cols, (long long)st.nnz, (long long)st.max_chain,
+                 (long long)st.sched_mode, (long long)st.n_levels, (long long)st.max_level_width, st.ms_build,
+                 st.ms_schedule, st.ms_sgd, st.ms_sgd_kernels, st.ms_bsp, status, (long long)pdb_launch_count());
+}
+
+}  // namespace pdb
+
 extern "C" {
 
 const char *pdb_strerror(int code)
@@ -431,6 +468,7 @@ void pdb_conflicts_free(pdb_conflicts *c)
 
 int pdb_build_conflicts(const pdb_csr *X, pdb_conflicts **out, void *stream)
 {
+    ApiScope scope("pdb_build_conflicts", nullptr, nullptr, out);
     if (!out) return PDB_EINVAL;
     *out = nullptr;
     int rc = check_csr(X);
@@ -590,6 +628,7 @@ void pdb_schedule_free(pdb_schedule *s)
 
 int pdb_schedule_build(const pdb_conflicts *c, pdb_sched_mode mode, pdb_schedule **out, void *stream)
 {
+    ApiScope scope("pdb_schedule_build", c, nullptr, nullptr, out);
     if (!c || !out || mode < PDB_SCHED_LEVELS || mode > PDB_SCHED_WINDOW) return PDB_EINVAL;
     *out = nullptr;
     cudaStream_t s = (cudaStream_t)stream;

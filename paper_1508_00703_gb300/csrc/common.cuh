@@ -284,3 +284,25 @@ struct pdb_schedule {
     cudaEvent_t ev0, ev1;
     bool timed;
 };
+
+namespace pdb {
+// Scope of one C-ABI call: an NVTX range named after the call (shown by
+// profilers, a no-op without one), and, when the environment variable
+// PDB_LOG is set to anything but "" or "0", one line of pdb_get_stats on
+// stderr after the call (pdb_get_stats synchronizes the device, so this is a
+// debugging aid).  pc / ph point at a handle the call creates, read when the
+// scope ends.
+struct ApiScope {
+    const char *name;
+    const pdb_conflicts *c;
+    const pdb_schedule *h;
+    pdb_conflicts *const *pc;
+    pdb_schedule *const *ph;
+    bool log;
+    ApiScope(const char *name_, const pdb_conflicts *c_, const pdb_schedule *h_ = nullptr,
+             pdb_conflicts *const *pc_ = nullptr, pdb_schedule *const *ph_ = nullptr, bool log_ = true);
+    ~ApiScope();
+    ApiScope(const ApiScope &) = delete;
+    ApiScope &operator=(const ApiScope &) = delete;
+};
+}  // namespace pdb

@@ -413,6 +413,7 @@ extern "C" {
 int pdb_sgd_epoch(const pdb_csr *X, const float *y, const pdb_conflicts *c, const pdb_schedule *h, float *w,
                   pdb_loss loss, float eta, int n_epochs, const pdb_opts *opts, void *stream)
 {
+    ApiScope scope("pdb_sgd_epoch", c, h);
     int rc = check_run(X, y, c, w, loss, n_epochs);
     if (rc != PDB_OK) return rc;
     if (!h || h->c != c) return PDB_EINVAL;
@@ -486,6 +487,7 @@ int pdb_ssp_epoch(const pdb_csr *X, const float *y, const pdb_conflicts *c, cons
                   pdb_loss loss, float eta, int n_epochs, int64_t delay, float *coef, const pdb_opts *opts,
                   void *stream)
 {
+    ApiScope scope("pdb_ssp_epoch", c, h);
     int rc = check_run(X, y, c, w, loss, n_epochs);
     if (rc != PDB_OK) return rc;
     if (!h || h->c != c || delay < 0) return PDB_EINVAL;
@@ -515,6 +517,7 @@ int pdb_ssp_epoch(const pdb_csr *X, const float *y, const pdb_conflicts *c, cons
 int pdb_bsp_epoch(const pdb_csr *X, const float *y, const pdb_conflicts *c, float *w, pdb_loss loss, float eta,
                   int64_t batch, int n_epochs, const pdb_opts *opts, void *stream)
 {
+    ApiScope scope("pdb_bsp_epoch", c);
     int rc = check_run(X, y, c, w, loss, n_epochs);
     if (rc != PDB_OK) return rc;
     if (batch < 1) return PDB_EINVAL;
@@ -633,6 +636,7 @@ unsigned long long *noalloc_scratch()
 extern "C" int pdb_sgd_epoch_ready_noalloc(const pdb_csr *X, const float *y, const uint32_t *gate, float *w,
                                            pdb_loss loss, float eta, int n_epochs, void *stream)
 {
+    ApiScope scope("pdb_sgd_epoch_ready_noalloc", nullptr, nullptr, nullptr, nullptr, false);  // no sync: may be captured
     if (!X || X->n_rows < 0 || X->n_cols < 0 || X->nnz < 0 || n_epochs < 0) return PDB_EINVAL;
     if (X->n_cols > NOALLOC_MAX_COLS) return PDB_ETOOBIG;
     if (X->n_rows >= (1ll << 31) - 1 || X->nnz >= (1ll << 31) - 1) return PDB_EINVAL;
