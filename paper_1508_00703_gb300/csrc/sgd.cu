@@ -310,16 +310,75 @@ __device__ __forceinline__ float margin(int t, const int64_t *__restrict__ row_p
     return warp_combine(acc);
 }
 
-// Algorithm 2a with B examples per step: reads (margins at the snapshot),
-// barrier, writes (ordered per-feature sums), barrier.  The batch's pairs
-// are pre-sorted by (batch, feature, example), so each feature's terms of a
-// batch are one contiguous run summed in ascending example order.
-__global__ __launch_bounds__(THREADS) void k_bsp(int32_t n_rows, int64_t batch, int64_t n_batches,
+// The next CH terms of feature j's run from q (the batch's sorted pairs end at
+// s1, its products start at s0), added to delta in ascending example order.
+// Loads first, then the dependent adds.  Returns whether the run continues
+// past the chunk (q then points after it).
+template <int CH>
+__device__ __forceinline__ bool run_chunk_prod(int32_t j, int64_t &q, int64_t s0, int64_t s1,
+                                               const int32_t *__restrict__ bcol, const float *prod, float &delta)
+{
+    int32_t jj[CH];
+    float pp[CH];
+#pragma unroll
+    for (int u = 0; u < CH; ++u) {
+        const bool in = q + u < s1;
+        jj[u] = in ? bcol[q + u] : -1;
+        pp[u] = in ? __ldcg(prod + (q + u - s0)) : 0.0f;
+    }
+    bool more = true;
+#pragma unroll
+    for (int u = 0; u < CH; ++u) {
+        more = more && jj[u] == j;
+        if (more) delta = __fadd_rn(delta, pp[u]);
+    }
+    q += CH;
+    return more;
+}
+
+// Runs longer than this many terms are summed by a whole warp.
+constexpr int BSP_LONG = 16;
+
+// Feature j's run from q, summed by the whole warp: 32 terms per load, the
+// adds in ascending order on every lane (each lane ends with the same delta).
+__device__ __forceinline__ float warp_run_sum(int32_t j, int64_t q, int64_t s0, int64_t s1,
+                                              const int32_t *__restrict__ bcol, const float *prod)
+{
+    const int lane = threadIdx.x & 31;
+    float delta = 0.0f;
+    int32_t jn = q + lane < s1 ? bcol[q + lane] : -1;
+    float pn = q + lane < s1 ? __ldcg(prod + (q + lane - s0)) : 0.0f;
+    for (;;) {
+        const float pc = pn;
+        const int n = __popc(__ballot_sync(FULL, jn == j));   // the run is a prefix of the 32
+        if (n == 32) {                                          // next 32 in flight during the adds
+            q += 32;
+            jn = q + lane < s1 ? bcol[q + lane] : -1;
+            pn = q + lane < s1 ? __ldcg(prod + (q + lane - s0)) : 0.0f;
+        }
+#pragma unroll
+        for (int u = 0; u < 32; ++u) {
+            const float v = __shfl_sync(FULL, pc, u);
+            if (u < n) delta = __fadd_rn(delta, v);
+        }
+        if (n < 32) return delta;
+    }
+}
+
+// Algorithm 2a with B examples per step: reads (the margins at the batch-start
+// weights), barrier; the products c_i * x_ij of the batch's pairs, which are
+// pre-sorted by (batch, feature, example), barrier; writes (each feature's
+// products summed in ascending example order, one run of the sorted pairs),
+// barrier.  A feature's run is summed by one thread, or by a whole warp when
+// it is longer than BSP_LONG terms.  Batches without such runs (has_long[b] =
+// 0) skip the products step: each thread forms its run's products itself.
+__global__ __launch_bounds__(THREADS, 8) void k_bsp(int32_t n_rows, int64_t batch, int64_t n_batches,
                                                  const int64_t *__restrict__ row_ptr, const int32_t *__restrict__ col,
                                                  const float *__restrict__ val, const float *__restrict__ y,
                                                  const int64_t *__restrict__ bptr, const int32_t *__restrict__ bcol,
                                                  const int32_t *__restrict__ brow, const float *__restrict__ bval,
-                                                 float *cbuf, float *w, int loss, float eta, int epochs,
+                                                 const uint8_t *__restrict__ has_long, float *cbuf, float *prod,
+                                                 float *w, int loss, float eta, int epochs,
                                                  GridBarrier *bar, int *status, uint64_t timeout)
 {
     if (read_status(status)) return;
@@ -336,22 +395,69 @@ __global__ __launch_bounds__(THREADS) void k_bsp(int32_t n_rows, int64_t batch, 
             }
             if (!grid_sync(bar, status, timeout)) return;
             const int64_t s0 = bptr[bi], s1 = bptr[bi + 1];
-            for (int64_t s = s0 + gtid; s < s1; s += nthr) {
-                const int32_t j = bcol[s];
-                if (s > s0 && bcol[s - 1] == j) continue;
-                float delta = 0.0f;
-                for (int64_t q = s; q < s1 && bcol[q] == j; ++q) {
-                    const int64_t i = brow[q] - r0;
-                    if (i < 0 || i >= r1 - r0) {     // cannot happen with a consistent batch sort
-                        set_status(status, PDB_EFAULT);
-                        break;
+            if (!has_long[bi]) {
+                // every run is short: one thread per run, term by term
+                for (int64_t s = s0 + gtid; s < s1; s += nthr) {
+                    const int32_t j = bcol[s];
+                    if (s > s0 && bcol[s - 1] == j) continue;
+                    float delta = 0.0f;
+                    for (int64_t q = s; q < s1 && bcol[q] == j; ++q) {
+                        const int64_t i = brow[q] - r0;
+                        if (i < 0 || i >= r1 - r0) {     // cannot happen with a consistent batch sort
+                            set_status(status, PDB_EFAULT);
+                            break;
+                        }
+                        delta = __fadd_rn(delta, __fmul_rn(__ldcg(cbuf + i), bval[q]));
                     }
-                    delta = __fadd_rn(delta, __fmul_rn(__ldcg(cbuf + i), bval[q]));
+                    __stcg(w + j, __fsub_rn(__ldcg(w + j), delta));
                 }
-                __stcg(w + j, __fsub_rn(__ldcg(w + j), delta));
+                if (!grid_sync(bar, status, timeout)) return;
+                continue;
+            }
+            for (int64_t s = s0 + gtid; s < s1; s += nthr) {
+                int64_t i = brow[s] - r0;
+                if (i < 0 || i >= r1 - r0) {     // cannot happen with a consistent batch sort
+                    set_status(status, PDB_EFAULT);
+                    i = 0;
+                }
+                __stcg(prod + (s - s0), __fmul_rn(__ldcg(cbuf + i), bval[s]));
+            }
+            if (!grid_sync(bar, status, timeout)) return;
+            for (int64_t base = s0 + (int64_t)gw * 32; base < s1; base += (int64_t)nw * 32) {
+                const int64_t s = base + lane;
+                const int32_t j = s < s1 ? bcol[s] : -1;
+                const bool start = s < s1 && (s == s0 || bcol[s - 1] != j);
+                const bool is_long = start && s + BSP_LONG < s1 && bcol[s + BSP_LONG] == j;
+                if (start && !is_long) {
+                    // at most BSP_LONG terms: a short first chunk (most runs hold one or two)
+                    float delta = 0.0f;
+                    int64_t q = s;
+                    if (run_chunk_prod<2>(j, q, s0, s1, bcol, prod, delta) &&
+                        run_chunk_prod<8>(j, q, s0, s1, bcol, prod, delta))
+                        run_chunk_prod<8>(j, q, s0, s1, bcol, prod, delta);
+                    __stcg(w + j, __fsub_rn(__ldcg(w + j), delta));
+                }
+                for (unsigned lm = __ballot_sync(FULL, is_long); lm; lm &= lm - 1) {
+                    const int src = __ffs(lm) - 1;
+                    const int64_t sr = __shfl_sync(FULL, s, src);
+                    const int32_t jr = __shfl_sync(FULL, j, src);
+                    const float delta = warp_run_sum(jr, sr, s0, s1, bcol, prod);
+                    if (lane == 0) __stcg(w + jr, __fsub_rn(__ldcg(w + jr), delta));
+                }
             }
             if (!grid_sync(bar, status, timeout)) return;
         }
+}
+
+// has_long[b] = 1 when batch b holds a feature run longer than BSP_LONG terms
+// (skey: batch of each pair in the (batch, feature, example) order)
+__global__ void k_bsp_long(const uint32_t *__restrict__ skey, const int32_t *__restrict__ bcol, int64_t nnz,
+                           uint8_t *__restrict__ has_long, const int *status)
+{
+    if (read_status(status)) return;
+    for (int64_t s = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; s + BSP_LONG < nnz;
+         s += (int64_t)gridDim.x * blockDim.x)
+        if (bcol[s + BSP_LONG] == bcol[s] && skey[s + BSP_LONG] == skey[s]) has_long[skey[s]] = 1;
 }
 
 __global__ void k_bsp_keys(const int32_t *__restrict__ csc_pos, const int32_t *__restrict__ row_of, int64_t nnz,
@@ -530,7 +636,8 @@ int pdb_bsp_epoch(const pdb_csr *X, const float *y, const pdb_conflicts *c, floa
         const int64_t n_batches = (N + batch - 1) / batch;
         uint32_t *key = nullptr, *skey = nullptr, *tkey = nullptr;
         int32_t *bpos = nullptr, *tval = nullptr, *bcol = nullptr, *brow = nullptr;
-        float *bval = nullptr, *cbuf = nullptr;
+        float *bval = nullptr, *cbuf = nullptr, *prod = nullptr;
+        uint8_t *has_long = nullptr;
         int64_t *bptr = nullptr;
         GridBarrier *bar = nullptr;
         rc = alloc((void **)&key, sizeof(uint32_t) * nnz, s);
@@ -542,6 +649,17 @@ int pdb_bsp_epoch(const pdb_csr *X, const float *y, const pdb_conflicts *c, floa
         rc = rc ? rc : alloc((void **)&brow, sizeof(int32_t) * nnz, s);
         rc = rc ? rc : alloc((void **)&bval, sizeof(float) * nnz, s);
         rc = rc ? rc : alloc((void **)&cbuf, sizeof(float) * batch, s);
+        // products of the largest batch: at most batch x (longest row) pairs
+        int64_t max_row = 0;
+        if (rc == PDB_OK) {
+            if (cudaEventSynchronize(c->ev1) != cudaSuccess) {
+                cudaGetLastError();
+                rc = PDB_ECUDA;
+            }
+            max_row = c->h_info[2];
+        }
+        rc = rc ? rc : alloc((void **)&has_long, (size_t)n_batches, s);
+        rc = rc ? rc : alloc((void **)&prod, sizeof(float) * std::max<int64_t>(1, std::min<int64_t>(nnz, batch * max_row)), s);
         rc = rc ? rc : alloc((void **)&bptr, sizeof(int64_t) * (n_batches + 1), s);
         rc = rc ? rc : alloc((void **)&bar, sizeof(GridBarrier), s);
         if (rc == PDB_OK) {
@@ -557,6 +675,13 @@ int pdb_bsp_epoch(const pdb_csr *X, const float *y, const pdb_conflicts *c, floa
             }
             if (rc == PDB_OK) rc = segment_bounds(skey, nnz, n_batches, nullptr, bptr, cm->status, s);
             if (rc == PDB_OK) {
+                cudaMemsetAsync(has_long, 0, (size_t)n_batches, s);
+                if (nnz > BSP_LONG) {
+                    k_bsp_long<<<grid_1d(nnz), 256, 0, s>>>(skey, bcol, nnz, has_long, cm->status);
+                    note_launch();
+                }
+            }
+            if (rc == PDB_OK) {
                 const void *kern = (const void *)k_bsp;
                 int grid = persistent_grid(kern, opts);
                 int32_t n32 = (int32_t)N;
@@ -566,13 +691,13 @@ int pdb_bsp_epoch(const pdb_csr *X, const float *y, const pdb_conflicts *c, floa
                 const int32_t *cl = X->col;
                 const float *vl = X->val;
                 void *args[] = {&n32,  &batch, (void *)&n_batches, (void *)&rp, (void *)&cl, (void *)&vl,
-                                (void *)&y, &bptr, &bcol, &brow, &bval, &cbuf, &w, &lossi, &eta, &n_epochs, &bar,
+                                (void *)&y, &bptr, &bcol, &brow, &bval, &has_long, &cbuf, &prod, &w, &lossi, &eta, &n_epochs, &bar,
                                 (void *)&cm->status, &tmo};
                 if (cudaLaunchCooperativeKernel(kern, grid, THREADS, args, 0, s) != cudaSuccess) rc = PDB_ECUDA; note_launch();
             }
         }
         for (void *p : {(void *)key, (void *)skey, (void *)tkey, (void *)bpos, (void *)tval, (void *)bcol, (void *)brow,
-                        (void *)bval, (void *)cbuf, (void *)bptr, (void *)bar})
+                        (void *)bval, (void *)cbuf, (void *)prod, (void *)has_long, (void *)bptr, (void *)bar})
             release(p, s);
     }
     cudaEventRecord(cm->ev_bsp1, s);
