@@ -361,6 +361,13 @@ def run_ours(args, rank, world, local_rank):
                 "peak_source": peak_kind,
                 "algorithmic_bytes_per_launch": sgd_bytes_per_launch, "launch_ms": round(sgd_launch_ms, 4),
                 "frac_of_8TBs": round(sgd_gbs / 8000.0, 4)}
+    if roofline["traffic"]:
+        # the DRAM bytes ncu counted per launch over this run's launch time: how busy
+        # HBM is, against the algorithmic fraction above (random 4-byte accesses move
+        # whole sectors)
+        dram_gbs = roofline["traffic"] / (sgd_launch_ms / 1e3) / 1e9
+        roofline["dram_gbs"] = round(dram_gbs, 1)
+        roofline["dram_frac"] = round(dram_gbs / peak, 4)
     result = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
