@@ -265,7 +265,8 @@ int pdb_ssp_epoch(const pdb_csr *X, const float *y, const pdb_conflicts *c, cons
  * dloss/dm at the weights of the batch start (read barrier), then each
  * feature j takes delta_j = sum over the batch's examples, ascending, of
  * c_i * x_ij and w_j = w_j - delta_j (write barrier).  batch = 1 equals
- * sequential SGD (Theorem 1).  Allocates per-call scratch stream-ordered. */
+ * sequential SGD (Theorem 1).  Allocates per-call scratch stream-ordered;
+ * sizing it waits (host) for the conflict build of c to finish. */
 int pdb_bsp_epoch(const pdb_csr *X, const float *y, const pdb_conflicts *c, float *w, pdb_loss loss, float eta,
                   int64_t batch, int n_epochs, const pdb_opts *opts, void *stream);
 
