@@ -15,8 +15,9 @@
 //                next D examples straight into that example's weight slot;
 //   warps 1-3, 5 prefetch one example of a step each with cp.async (ids,
 //                values, labels and link words 4 steps ahead; the weights
-//                nobody will push 2 steps ahead), lanes striding over the
-//                example's elements;
+//                nobody will push 2 steps ahead, together with the shared
+//                memory address each new weight goes to), lanes striding
+//                over the example's elements;
 //   warps 6, 7   write the new weights of the previous step that are not
 //                pushed through to global memory, and copy row bounds 7
 //                steps ahead;
@@ -59,18 +60,23 @@ static_assert(CH_SLOTS > (CH_DS + 2) * CH_G && CH_RP > (CH_L + 2) * CH_G + 1, "r
 static_assert(CH_D < 256 && CH_MAXK <= 65536, "link word fields");
 static_assert((CH_G & (CH_G - 1)) == 0, "examples per step must be a power of two");
 
-// ids, values and link words are copied in 16-byte pieces from the aligned
-// element before the example's first one: element i sits at index off + i,
-// off = (first position) mod 4 (0 when an input array is not 16-byte aligned)
+// ids and link words are copied in 16-byte pieces from the aligned element
+// before the example's first one: element i sits at index off + i, off =
+// (first position) mod 4 (0 when an input array is not 16-byte aligned).
+// Everything the compute warp reads is at element index i, so its loads need
+// no row bounds.
 constexpr int CH_ROW = CH_MAXK + 4;
 struct ChainSmem {
     int32_t col[CH_SLOTS][CH_ROW];
-    float val[CH_SLOTS][CH_ROW];
     uint32_t link[CH_SLOTS][CH_ROW];
+    float xa[CH_SLOTS][CH_MAXK];    // value of each element (1 without values)
+    uint32_t pa[CH_SLOTS][CH_MAXK]; // where the compute warp stores each element's new weight
     float wp[CH_SLOTS][CH_MAXK];    // weight each element reads (gathered or pushed)
     float out[CH_SLOTS][CH_MAXK];   // weight of the elements whose next occurrence is not pushed
     int64_t rp[CH_RP];
     float y[CH_SLOTS];
+    int kk[CH_SLOTS];               // length of each example
+    float dump[32];                 // store target of the lanes past an example's end
     __align__(16) float part[32];   // the compute warp's 32 partial sums
 };
 
@@ -207,19 +213,32 @@ __global__ __launch_bounds__(CH_THREADS, 1) void k_sgd_chain(int32_t n_rows, con
                         const int slot = r & (CH_SLOTS - 1);
                         cp_row(S.col[slot], col, b, k, off, vec, lane);
                         cp_row(S.link[slot], link, b, k, off, vec, lane);
-                        if (val) cp_row(S.val[slot], val, b, k, off, vec, lane);
+                        for (int i = lane; i < k; i += 32) {
+                            if (val)
+                                cp4(&S.xa[slot][i], val + b + i);
+                            else
+                                S.xa[slot][i] = 1.0f;
+                        }
                         if (lane == 0) cp4(&S.y[slot], y + r);
                     }
                 }
-                // stage B: weights of example g of step t + BS that no recent example pushes
+                // stage B: weights of example g of step t + BS that no recent example pushes,
+                // and where the compute warp stores each element's new weight: into the
+                // receiver's slot of wp when pushed, else into out (written through by 6, 7)
                 {
                     const int r = (t + CH_BS) * CH_G + gA;
                     int64_t b;
                     int k, off;
                     if (row_bounds(S, r, N, vec, b, k, off)) {
                         const int slot = r & (CH_SLOTS - 1);
-                        for (int i = lane; i < k; i += 32)
-                            if (!(S.link[slot][off + i] & LK_RECV)) cp4(&S.wp[slot][i], w + S.col[slot][off + i]);
+                        for (int i = lane; i < k; i += 32) {
+                            const uint32_t lk = S.link[slot][off + i];
+                            if (!(lk & LK_RECV)) cp4(&S.wp[slot][i], w + S.col[slot][off + i]);
+                            const unsigned tslot = ((unsigned)r + ((lk >> 16) & 0xffu)) & (CH_SLOTS - 1);
+                            S.pa[slot][i] = (lk & LK_PUSH) ? wp_base + 4u * (tslot * CH_MAXK + (lk & 0xffffu))
+                                                           : out_base + 4u * ((unsigned)slot * CH_MAXK + i);
+                        }
+                        if (lane == 0) S.kk[slot] = k;
                     }
                 }
             }
@@ -227,43 +246,47 @@ __global__ __launch_bounds__(CH_THREADS, 1) void k_sgd_chain(int32_t n_rows, con
                 cp_commit();
                 cp_wait_b();
             } else if (t >= 0 && t < steps) {
-                // compute the G examples of step t in data order
-                for (int r = t * CH_G; r < min(N, t * CH_G + CH_G); ++r) {
+                // compute the G examples of step t in data order; an example's length,
+                // label, values and store addresses are fetched while the one before
+                // finishes, its weights once that one's pushes are stored
+                const int r0 = t * CH_G, r1 = min(N, r0 + CH_G);
+                const unsigned dump = (unsigned)__cvta_generic_to_shared(&S.dump[lane]);
+                int k;
+                float yr, xv[R];
+                unsigned pa[R];
+                auto fetch = [&](int r) {
                     const int slot = r & (CH_SLOTS - 1);
-                    int64_t b;
-                    int k, off;
-                    row_bounds(S, r, N, vec, b, k, off);
-                    const float yr = S.y[slot];
-                    float xv[R], wv[R];
-                    uint32_t lk[R];
+                    k = S.kk[slot];
+                    yr = S.y[slot];
+#pragma unroll
+                    for (int q = 0; q < R; ++q) {
+                        xv[q] = S.xa[slot][q * 32 + lane];
+                        pa[q] = S.pa[slot][q * 32 + lane];
+                    }
+                };
+                fetch(r0);
+                for (int r = r0; r < r1; ++r) {
+                    const int slot = r & (CH_SLOTS - 1);
+                    float wv[R], xc[R];
+                    unsigned ac[R];
                     float acc = 0.0f;
 #pragma unroll
                     for (int q = 0; q < R; ++q) {
                         const int i = q * 32 + lane;
-                        if (i < k) {
-                            xv[q] = val ? S.val[slot][off + i] : 1.0f;
-                            wv[q] = S.wp[slot][i];
-                            lk[q] = S.link[slot][off + i];
-                            acc = __fmaf_rn(wv[q], xv[q], acc);
-                        }
+                        wv[q] = S.wp[slot][i];                  // past k: unused
+                        const float f = __fmaf_rn(wv[q], xv[q], acc);
+                        acc = i < k ? f : acc;
+                        xc[q] = xv[q];
+                        ac[q] = i < k ? pa[q] : dump;
                     }
+                    const float yc = yr;
+                    trace_mark(trace, (int64_t)ep * N + r, 0);    // every weight is read
                     const float m = combine_smem(acc, S.part);
-                    trace_mark(trace, (int64_t)ep * N + r, 0);
-                    const float c = __fmul_rn(eta, dev_grad(loss, m, yr));
+                    if (r + 1 < r1) fetch(r + 1);
+                    const float c = __fmul_rn(eta, dev_grad(loss, m, yc));
                     trace_mark(trace, (int64_t)ep * N + r, 1);   // before any write is visible
 #pragma unroll
-                    for (int q = 0; q < R; ++q) {
-                        const int i = q * 32 + lane;
-                        if (i < k) {
-                            // one store per element, no branch: into the receiver's slot of
-                            // wp when pushed, else into out (written through by warps 6, 7)
-                            const unsigned tslot = (r + ((lk[q] >> 16) & 0xffu)) & (CH_SLOTS - 1);
-                            const unsigned a_push = wp_base + 4u * (tslot * CH_MAXK + (lk[q] & 0xffffu));
-                            const unsigned a_out = out_base + 4u * (slot * CH_MAXK + i);
-                            st_shared((lk[q] & LK_PUSH) ? a_push : a_out,
-                                      __fsub_rn(wv[q], __fmul_rn(c, xv[q])));
-                        }
-                    }
+                    for (int q = 0; q < R; ++q) st_shared(ac[q], __fsub_rn(wv[q], __fmul_rn(c, xc[q])));
                     __syncwarp();
                 }
             }
