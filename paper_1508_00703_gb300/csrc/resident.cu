@@ -57,6 +57,10 @@ __device__ __forceinline__ void cp16(void *smem_dst, const void *gsrc)
 }
 __device__ __forceinline__ void cp_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
 __device__ __forceinline__ void cp_wait_1() { asm volatile("cp.async.wait_group 1;" ::: "memory"); }
+__device__ __forceinline__ void st_shared(unsigned addr, float v)
+{
+    asm volatile("st.shared.f32 [%0], %1;" ::"r"(addr), "f"(v) : "memory");
+}
 __device__ __forceinline__ void cp_wait_all() { asm volatile("cp.async.wait_group 0;" ::: "memory"); }
 
 // elements [b - off, b + k) of a 4-byte array into dst: 16-byte pieces from
@@ -111,7 +115,7 @@ __host__ __device__ __forceinline__ Layout layout(int64_t n_cols, int kcap)
     L.y = L.val + (int64_t)RZ_NS * kcap * 4;
     L.rp = L.y + RZ_NS * 4 + 16;
     L.part = L.rp + RZ_RP * 16;
-    L.total = L.part + 32 * 4;
+    L.total = L.part + 64 * 4;      // 32 partial sums, then 32 scratch words
     return L;
 }
 
@@ -133,6 +137,7 @@ __global__ __launch_bounds__(RZ_THREADS, 1) void k_sgd_resident(int32_t n_rows, 
     float *ys = reinterpret_cast<float *>(smem_raw + Lo.y);
     int64_t *rp = reinterpret_cast<int64_t *>(smem_raw + Lo.rp);    // [RZ_RP][2]: bounds of an example
     float *part = reinterpret_cast<float *>(smem_raw + Lo.part);
+    const unsigned dump = (unsigned)__cvta_generic_to_shared(part + 32 + (threadIdx.x & 31));
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
 
     for (int64_t f = tid; f < n_cols; f += RZ_THREADS) ws[f] = w[f];
@@ -176,25 +181,32 @@ __global__ __launch_bounds__(RZ_THREADS, 1) void k_sgd_resident(int32_t n_rows, 
                 const float yr = ys[slot];
                 float acc = 0.0f;
                 if (k <= 32 * R) {
+                    // the whole example in registers; no branches: lanes past the
+                    // example's end read w_0 and store into a scratch word
                     int j[R];
                     float x[R], wv[R];
 #pragma unroll
                     for (int q = 0; q < R; ++q) {
                         const int i = q * 32 + lane;
-                        if (i < k) {
-                            j[q] = ci[i];
-                            x[q] = val ? vi[i] : 1.0f;
-                            wv[q] = ws[j[q]];
-                            acc = __fmaf_rn(wv[q], x[q], acc);
-                        }
+                        j[q] = i < k ? ci[i] : 0;
+                        x[q] = i < k ? (val ? vi[i] : 1.0f) : 0.0f;
+                    }
+#pragma unroll
+                    for (int q = 0; q < R; ++q) wv[q] = ws[j[q]];
+#pragma unroll
+                    for (int q = 0; q < R; ++q) {
+                        const float f = __fmaf_rn(wv[q], x[q], acc);
+                        acc = q * 32 + lane < k ? f : acc;
                     }
                     const float m = combine_smem(acc, part);
                     trace_mark(trace, rg, 0);
                     const float c = __fmul_rn(eta, dev_grad(loss, m, yr));
                     trace_mark(trace, rg, 1);   // before any write is visible
+                    const unsigned ws_base = (unsigned)__cvta_generic_to_shared(ws);
 #pragma unroll
                     for (int q = 0; q < R; ++q)
-                        if (q * 32 + lane < k) ws[j[q]] = __fsub_rn(wv[q], __fmul_rn(c, x[q]));
+                        st_shared(q * 32 + lane < k ? ws_base + 4u * (unsigned)j[q] : dump,
+                                  __fsub_rn(wv[q], __fmul_rn(c, x[q])));
                 } else {
                     // long example, in pieces of RZ_U elements per lane (all their loads
                     // issued before the lane's fused multiply-adds, which keep element
@@ -273,8 +285,11 @@ int resident_run(const pdb_csr *X, const float *y, float *w, int loss, float eta
 {
     const int64_t smem = resident_smem(X->n_cols, max_row);
     if (smem == 0) return PDB_ETOOBIG;
+    // registers per lane for the longest example: 1 .. 32 (32 to 1024 ids); longer rows
+    // take the two-pass path of the 32-register variant
     auto kern = max_row <= 32 ? k_sgd_resident<1> : max_row <= 64 ? k_sgd_resident<2>
-              : max_row <= 128 ? k_sgd_resident<4> : k_sgd_resident<8>;
+              : max_row <= 128 ? k_sgd_resident<4> : max_row <= 256 ? k_sgd_resident<8>
+              : max_row <= 512 ? k_sgd_resident<16> : k_sgd_resident<32>;
     if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
         return PDB_ECUDA;
     const bool vec = ((uintptr_t)X->col & 15) == 0 && ((uintptr_t)X->val & 15) == 0;
