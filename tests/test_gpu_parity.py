@@ -69,6 +69,30 @@ def test_chains_bit_exact(name):
     assert st["max_chain"] == (counts.max() if counts.size else 0)
 
 
+@pytest.mark.parametrize("n_rows", [45_000, 52_429])
+def test_gate_words_past_the_l2_sized_path(n_rows):
+    # above 2^22 positions the gate words return to position order through a
+    # position sort and per-piece inversion; 52,429 x 100 ids leave a ragged
+    # last piece of 2^19 slots
+    import oracle
+    import synthdata
+    p = synthdata.generate("low-conflict", n_rows=n_rows, n_cols=2_000_000)
+    assert p.nnz > (1 << 22)
+    X = pdb.Csr.from_problem(p)
+    y = torch.from_numpy(p.y).cuda()
+    c = pdb.pdb_build_conflicts(X)
+    arrs = pdb.pdb_conflicts_arrays(c)
+    pdb.check_status(c)
+    ref = oracle.chains(p)
+    for key in ("prev", "next", "rank"):
+        assert np.array_equal(_arr(arrs[key], p.nnz, torch.int32), ref[key]), key
+    s = pdb.pdb_schedule_build(c, pdb.PDB_SCHED_WINDOW)
+    w = torch.zeros(p.n_cols, dtype=torch.float32, device="cuda")
+    pdb.pdb_sgd_epoch(X, y, c, s, w, p.loss, p.eta, 1)
+    pdb.check_status(c)
+    assert np.array_equal(w.cpu().numpy(), oracle.sgd(p, epochs=1))
+
+
 @pytest.mark.parametrize("name", ALL)
 def test_levels_bit_exact(name):
     p, X, y = _gpu(name)
