@@ -170,9 +170,10 @@ __global__ __launch_bounds__(CH_THREADS, 1) void k_sgd_chain(int32_t n_rows, con
     if (read_status(status)) return;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     // warp 0 computes; warps 1, 2, 3, 5 prefetch example g = 0..3 of a step
-    // (ids, values, link words, then weights); warps 6, 7 write the weights of
-    // the previous step through (two examples each) and copy row bounds; warp
-    // 4 only joins the barriers (it shares warp 0's scheduler)
+    // (ids, values, link words, then weights and store addresses); warps 6, 7
+    // write the weights of the previous step through (two examples each) and
+    // copy row bounds; warp 4 only joins the barriers (it shares warp 0's
+    // scheduler)
     const bool compute = warp == 0;
     const unsigned wp_base = (unsigned)__cvta_generic_to_shared(&S.wp[0][0]);
     const unsigned out_base = (unsigned)__cvta_generic_to_shared(&S.out[0][0]);
