@@ -188,8 +188,11 @@ int pdb_conflicts_arrays(const pdb_conflicts *c, const int32_t **csc_pos, const 
 /* Schedule for pdb_sgd_epoch.
  *   LEVELS: level[t] = 1 + max over features j of t with an earlier
  *     occurrence of level[row of that occurrence], 0 if none (longest
- *     conflict path), computed by a Kahn-style frontier sweep; order[N] lists
- *     the examples by level, ascending id inside a level; level_ptr[L+1]
+ *     conflict path), computed by dataflow (examples in data order, each
+ *     waiting, bounded, for its predecessors' levels) or, with the
+ *     environment variable PDB_LEVELS=kahn, by a Kahn-style frontier sweep
+ *     (one grid barrier per level); both give the same levels.  order[N]
+ *     lists the examples by level, ascending id inside a level; level_ptr[L+1]
  *     delimits the levels.
  *   READY: one 64-bit record per feature, bits(w_j) | version_j << 32,
  *     filled from w by pdb_sgd_epoch; each position waits for the version

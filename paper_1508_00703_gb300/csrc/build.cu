@@ -322,6 +322,88 @@ __global__ __launch_bounds__(THREADS) void k_levels_kahn(int32_t n_rows, const i
     }
 }
 
+// Theorem 3's levels by dataflow instead of frontiers: warps take examples
+// in data order from a ticket counter; example t waits (bounded) until the
+// example of every previous occurrence of its features has published its
+// level, then publishes 1 + their maximum (0 when there is none).  level[]
+// starts at -1 (unpublished).  An example waits only on smaller ones and the
+// smallest unfinished one on none, so there is no deadlock, and no grid
+// barrier: a chain of L levels costs L hand-offs through L2, not L barriers.
+__global__ __launch_bounds__(THREADS) void k_levels_flow(int32_t n_rows, const int64_t *__restrict__ row_ptr,
+                                                         const int32_t *__restrict__ prev,
+                                                         const int32_t *__restrict__ row_of, int32_t *level,
+                                                         unsigned long long *ticket, int chunk, int *status,
+                                                         uint64_t timeout)
+{
+    if (read_status(status)) return;
+    const int lane = threadIdx.x & 31;
+    for (;;) {
+        unsigned long long tk = 0;
+        if (lane == 0) tk = atomicAdd(ticket, (unsigned long long)chunk);
+        tk = __shfl_sync(FULL, tk, 0);
+        if (tk >= (unsigned long long)n_rows) return;
+        const int t1 = (int)min64(n_rows, (int64_t)tk + chunk);
+        for (int t = (int)tk; t < t1; ++t) {
+            const int64_t b = row_ptr[t], e = row_ptr[t + 1];
+            int best = -1;
+            bool ok = true;
+            for (int64_t p = b + lane; p < e && ok; p += 32) {
+                const int q = prev[p];
+                if (q < 0) continue;
+                const int u = row_of[q];
+                if (u < 0 || u >= t) {             // cannot happen with consistent chains
+                    set_status(status, PDB_EFAULT);
+                    ok = false;
+                    break;
+                }
+                int lv = ld_acquire_i(level + u);
+                if (lv < 0) {
+                    const uint64_t t0 = globaltimer();
+                    unsigned spins = 0, nap = 32;
+                    while ((lv = ld_acquire_i(level + u)) < 0) {
+                        __nanosleep(nap);
+                        nap = nap < 256 ? 2 * nap : 256;
+                        if ((++spins & 15u) != 0) continue;
+                        if (read_status(status)) {
+                            ok = false;
+                            break;
+                        }
+                        if (globaltimer() - t0 > timeout) {
+                            set_status(status, PDB_ETIMEOUT);
+                            ok = false;
+                            break;
+                        }
+                    }
+                }
+                best = max(best, lv);
+            }
+            if (!__all_sync(FULL, ok)) return;
+            for (int off = 16; off >= 1; off >>= 1) best = max(best, __shfl_xor_sync(FULL, best, off));
+            if (lane == 0) st_release(reinterpret_cast<unsigned *>(level + t), (unsigned)(best + 1));
+        }
+    }
+}
+
+// L = 1 + the largest level (the last of the sorted level keys)
+__global__ void k_level_count(const uint32_t *__restrict__ sorted_levels, int32_t n, LevelCtl *ctl,
+                              const int *status)
+{
+    if (read_status(status)) return;
+    if (threadIdx.x == 0) ctl->n_levels = n > 0 ? (int)sorted_levels[n - 1] + 1 : 0;
+}
+
+// the widest level, from the level boundaries
+__global__ void k_level_width(const int64_t *__restrict__ level_ptr, LevelCtl *ctl, const int *status)
+{
+    if (read_status(status)) return;
+    const int L = ctl->n_levels;
+    int widest = 0;
+    for (int l = blockIdx.x * blockDim.x + threadIdx.x; l < L; l += gridDim.x * blockDim.x)
+        widest = max(widest, (int)(level_ptr[l + 1] - level_ptr[l]));
+    for (int off = 16; off >= 1; off >>= 1) widest = max(widest, __shfl_xor_sync(FULL, widest, off));
+    if ((threadIdx.x & 31) == 0 && widest > 0) atomicMax(&ctl->max_width, widest);
+}
+
 __global__ void k_level_keys(const int32_t *__restrict__ level, uint32_t *__restrict__ key, int32_t n,
                              const int *status)
 {
@@ -691,9 +773,13 @@ int pdb_schedule_build(const pdb_conflicts *c, pdb_sched_mode mode, pdb_schedule
             rc = rc ? rc : chain_schedule(c->prev, c->next, c->row_of, c->row_ptr, nnz, h->link, c->status, s);
         }
     } else {
+        // Theorem 3's levels by dataflow (default) or by the Kahn frontier sweep
+        // (PDB_LEVELS=kahn: one grid barrier per level)
+        const char *lv_env = std::getenv("PDB_LEVELS");
+        const bool flow = !(lv_env && std::strcmp(lv_env, "kahn") == 0);
         rc = rc ? rc : materialize_chains(cm, s);
         rc = rc ? rc : ensure_row_of(cm, s);
-        if (rc == PDB_OK && !cm->npred) {
+        if (!flow && rc == PDB_OK && !cm->npred) {
             rc = alloc((void **)&cm->npred, sizeof(int32_t) * N, s);
             if (rc == PDB_OK && N > 0) {
                 k_npred<<<grid_1d(N * 32), 256, 0, s>>>(c->row_ptr, N, c->prev, cm->npred, c->status);
@@ -702,8 +788,10 @@ int pdb_schedule_build(const pdb_conflicts *c, pdb_sched_mode mode, pdb_schedule
         }
         rc = rc ? rc : alloc((void **)&h->level, sizeof(int32_t) * N, s);
         rc = rc ? rc : alloc((void **)&h->order, sizeof(int32_t) * N, s);
-        rc = rc ? rc : alloc((void **)&h->indeg, sizeof(int32_t) * N, s);
-        rc = rc ? rc : alloc((void **)&h->queue, sizeof(int32_t) * N, s);
+        if (!flow) {
+            rc = rc ? rc : alloc((void **)&h->indeg, sizeof(int32_t) * N, s);
+            rc = rc ? rc : alloc((void **)&h->queue, sizeof(int32_t) * N, s);
+        }
         rc = rc ? rc : alloc((void **)&h->level_ptr, sizeof(int64_t) * (N + 1), s);
         rc = rc ? rc : alloc((void **)&h->ctl, sizeof(LevelCtl), s);
         uint32_t *key = nullptr, *skey = nullptr, *tkey = nullptr;
@@ -715,21 +803,38 @@ int pdb_schedule_build(const pdb_conflicts *c, pdb_sched_mode mode, pdb_schedule
         if (rc == PDB_OK) {
             cudaMemsetAsync(h->ctl, 0, sizeof(LevelCtl), s);
             if (N > 0) {
-                const void *kern = (const void *)k_levels_kahn;
-                int grid = persistent_grid(kern, nullptr);
                 int32_t n32 = (int32_t)N;
                 uint64_t tmo = timeout_ns(nullptr);
-                void *args[] = {&n32,       (void *)&c->row_ptr, (void *)&c->next, (void *)&c->row_of,
-                                (void *)&c->npred, &h->indeg, &h->queue, &h->level,
-                                &h->ctl,    (void *)&c->status, &tmo};
-                if (cudaLaunchCooperativeKernel(kern, grid, THREADS, args, 0, s) != cudaSuccess) rc = PDB_ECUDA;
-                note_launch();
+                if (flow) {
+                    cudaMemsetAsync(h->level, 0xff, sizeof(int32_t) * N, s);
+                    cudaMemsetAsync(h->ticket, 0, sizeof(unsigned long long), s);
+                    const int grid = persistent_grid((const void *)k_levels_flow, nullptr);
+                    k_levels_flow<<<grid, THREADS, 0, s>>>(n32, c->row_ptr, c->prev, c->row_of, h->level, h->ticket, 4,
+                                                           c->status, tmo);
+                    note_launch();
+                } else {
+                    const void *kern = (const void *)k_levels_kahn;
+                    int grid = persistent_grid(kern, nullptr);
+                    void *args[] = {&n32,       (void *)&c->row_ptr, (void *)&c->next, (void *)&c->row_of,
+                                    (void *)&c->npred, &h->indeg, &h->queue, &h->level,
+                                    &h->ctl,    (void *)&c->status, &tmo};
+                    if (cudaLaunchCooperativeKernel(kern, grid, THREADS, args, 0, s) != cudaSuccess) rc = PDB_ECUDA;
+                    note_launch();
+                }
                 if (rc == PDB_OK) {
                     k_level_keys<<<grid_1d(N), 256, 0, s>>>(h->level, key, n32, c->status);
                     note_launch();
                     rc = radix_sort(key, nullptr, skey, h->order, tkey, tval, N, bits_for(N), c->status, s);
                 }
+                if (rc == PDB_OK && flow) {
+                    k_level_count<<<1, 32, 0, s>>>(skey, n32, h->ctl, c->status);
+                    note_launch();
+                }
                 if (rc == PDB_OK) rc = segment_bounds(skey, N, N, &h->ctl->n_levels, h->level_ptr, c->status, s);
+                if (rc == PDB_OK && flow) {
+                    k_level_width<<<grid_1d(N), 256, 0, s>>>(h->level_ptr, h->ctl, c->status);
+                    note_launch();
+                }
             } else {
                 cudaMemsetAsync(h->level_ptr, 0, sizeof(int64_t), s);
             }

@@ -72,8 +72,8 @@ def test_chains_bit_exact(name):
 @pytest.mark.parametrize("n_rows", [45_000, 52_429])
 def test_gate_words_past_the_l2_sized_path(n_rows):
     # above 2^22 positions the gate words return to position order through a
-    # position sort and per-piece inversion; 52,429 x 100 ids leave a ragged
-    # last piece of 2^19 slots
+    # position sort and per-block inversion; 52,429 x 100 ids leave a ragged
+    # last block (20 of 2^14 slots)
     import oracle
     import synthdata
     p = synthdata.generate("low-conflict", n_rows=n_rows, n_cols=2_000_000)
@@ -93,8 +93,11 @@ def test_gate_words_past_the_l2_sized_path(n_rows):
     assert np.array_equal(w.cpu().numpy(), oracle.sgd(p, epochs=1))
 
 
+@pytest.mark.parametrize("sweep", ["flow", "kahn"])
 @pytest.mark.parametrize("name", ALL)
-def test_levels_bit_exact(name):
+def test_levels_bit_exact(name, sweep, monkeypatch):
+    # the dataflow level builder (default) and the Kahn frontier sweep
+    monkeypatch.setenv("PDB_LEVELS", sweep)
     p, X, y = _gpu(name)
     c = pdb.pdb_build_conflicts(X)
     s = pdb.pdb_schedule_build(c, pdb.PDB_SCHED_LEVELS)
