@@ -25,6 +25,8 @@ SMALL = {
     # enough for it
     "dense-shape": ("dense-lr", dict(n_rows=800, n_cols=320, k=320, epochs=3, bsp_batch=800)),
     "dense-narrow": ("dense-lr", dict(n_rows=1500, n_cols=200, k=200, epochs=2, bsp_batch=1500)),
+    # the full 960-feature width (rows of 513..1024 ids: 32 registers per lane)
+    "dense-wide": ("dense-lr", dict(n_rows=300, epochs=2, bsp_batch=300)),
 }
 
 FULL = {
