@@ -170,6 +170,10 @@ typedef struct pdb_schedule pdb_schedule;   /* opaque, library-owned device arra
  * this call.  Any near >= 1 gives the same SGD result; it only decides which
  * positions wait on the watermark.
  * A feature occurring 2^29 times or more is reported as PDB_ETOOBIG.
+ * Above 2^22 positions the position-order gate array is built on first use
+ * (a READY, CHAIN or LEVELS schedule, or pdb_conflicts_arrays), enqueued on
+ * that call's stream; the WINDOW schedule needs only the near pairs' words,
+ * which the build writes directly.
  * *out receives a new handle (free with pdb_conflicts_free) even when the
  * device later reports a CSR error through pdb_status.  The handle keeps
  * referring to X's arrays (D is immutable, Definition 1): they must stay
@@ -218,7 +222,9 @@ int pdb_schedule_levels(const pdb_schedule *s, const int32_t **level, const int3
  * NULL): gate[nnz], per position bits 0..28 the version it waits for (its
  * occurrence rank), bit 29 set when the next occurrence of its feature lies
  * within the build's `near` distance, bit 30 when the previous one does,
- * bit 31 on the last occurrence of its feature; and, READY only,
+ * bit 31 on the last occurrence of its feature (under WINDOW with more than
+ * 2^22 positions: the WINDOW engine's copy, which holds only the words of
+ * positions with a near pair and 0 elsewhere); and, READY only,
  * records[n_cols] (weight bits | version << 32, the version being the rank
  * waited for in bits 0..28 and an epoch stamp 1..7 in bits 29..31;
  * meaningful while pdb_sgd_epoch runs; NULL under WINDOW).  PDB_ESTATE for LEVELS and CHAIN

@@ -105,8 +105,8 @@ __device__ __forceinline__ int64_t find_row(const int64_t *__restrict__ row_ptr,
 // (gsort[s]) for the partitioned scatter below.
 __global__ void k_slots(const uint32_t *__restrict__ skey, const int32_t *__restrict__ spos, int64_t nnz,
                         const int64_t *__restrict__ feat_ptr, const int64_t *__restrict__ row_ptr, int64_t n_rows,
-                        int64_t near,
-                        uint32_t *__restrict__ gate, uint32_t *__restrict__ gsort, int *info)
+                        int64_t near, uint32_t *__restrict__ gate, uint32_t *__restrict__ gsort,
+                        uint32_t *__restrict__ gwin, int *info)
 {
     if (read_status(info)) return;
     const bool check_dup = *(volatile int *)(info + INFO_UNSORTED) != 0;
@@ -154,6 +154,7 @@ __global__ void k_slots(const uint32_t *__restrict__ skey, const int32_t *__rest
             g[e] = ((uint32_t)r & GATE_RANK) | (near_next ? GATE_NEAR_NEXT : 0u) |
                    (near_prev ? GATE_NEAR_PREV : 0u) | (last ? GATE_LAST : 0u);
             if (!gsort) gate[p] = g[e];
+            if (gwin && (near_prev || near_next)) gwin[p] = g[e];
             if (last) longest = max(longest, (int)(r + 1));
             if (check_dup && r > 0) dup |= find_row(row_ptr, n_rows, pp[e]) == find_row(row_ptr, n_rows, p);
         }
@@ -452,10 +453,59 @@ int ensure_row_of(pdb_conflicts *c, cudaStream_t s)
 
 namespace {
 
+// The position-order gate array (idempotent; enqueued on s).  Above 2^22
+// positions the build keeps the gate words in csc_pos order only; here the
+// (position, gate) pairs are sorted on the position bits above SCATTER_SB
+// and k_scatter_block inverts each 2^SCATTER_SB-slot block in shared memory.
+int ensure_gate(pdb_conflicts *c, cudaStream_t s)
+{
+    if (c->gate) return PDB_OK;
+    const int64_t nnz = c->nnz;
+    uint32_t *gate = nullptr, *pk = nullptr, *tkey = nullptr;
+    int32_t *pv = nullptr, *tval = nullptr;
+    int rc = alloc((void **)&gate, sizeof(uint32_t) * nnz, s);
+    rc = rc ? rc : alloc((void **)&pk, sizeof(uint32_t) * nnz, s);
+    rc = rc ? rc : alloc((void **)&pv, sizeof(int32_t) * nnz, s);
+    rc = rc ? rc : alloc((void **)&tkey, sizeof(uint32_t) * nnz, s);
+    rc = rc ? rc : alloc((void **)&tval, sizeof(int32_t) * nnz, s);
+    if (rc == PDB_OK)
+        rc = radix_sort_bits((const uint32_t *)c->csc_pos, (const int32_t *)c->gate_sorted, pk, pv, tkey, tval, nnz,
+                             SCATTER_SB, bits_for(nnz - 1), c->info, s);
+    if (rc == PDB_OK) {
+        const size_t smem = sizeof(uint32_t) << SCATTER_SB;
+        static bool configured[64] = {};
+        if (c->device >= 0 && c->device < 64 && !configured[c->device]) {
+            if (cudaFuncSetAttribute(k_scatter_block, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) !=
+                cudaSuccess)
+                rc = PDB_ECUDA;
+            else
+                configured[c->device] = true;
+        }
+        if (rc == PDB_OK) {
+            const int64_t blocks = ((nnz - 1) >> SCATTER_SB) + 1;
+            k_scatter_block<<<(unsigned)blocks, SCATTER_THREADS, smem, s>>>(pk, (const uint32_t *)pv, nnz, gate,
+                                                                             c->info);
+            note_launch();
+        }
+    }
+    release(pk, s);
+    release(pv, s);
+    release(tkey, s);
+    release(tval, s);
+    if (rc != PDB_OK) {
+        release(gate, s);
+        return rc;
+    }
+    c->gate = gate;
+    return cudaPeekAtLastError() == cudaSuccess ? PDB_OK : PDB_ECUDA;
+}
+
 // prev/next/rank of every position (idempotent; enqueued on s)
 int materialize_chains(pdb_conflicts *c, cudaStream_t s)
 {
     if (c->prev) return PDB_OK;
+    const int rg = ensure_gate(c, s);
+    if (rg != PDB_OK) return rg;
     const int64_t nnz = c->nnz;
     int32_t *prev = nullptr, *next = nullptr, *rank = nullptr;
     int rc = alloc((void **)&prev, sizeof(int32_t) * nnz, s);
@@ -541,7 +591,8 @@ void pdb_conflicts_free(pdb_conflicts *c)
 {
     if (!c) return;
     cudaDeviceSynchronize();
-    free_ptrs({c->csc_pos, c->feat_ptr, c->gate, c->row_of, c->prev, c->next, c->rank, c->npred, c->info});
+    free_ptrs({c->csc_pos, c->feat_ptr, c->gate, c->gate_sorted, c->gate_window != c->gate ? c->gate_window : nullptr,
+               c->row_of, c->prev, c->next, c->rank, c->npred, c->info});
     if (c->h_info) cudaFreeHost(c->h_info);
     for (cudaEvent_t e : {c->ev0, c->ev1, c->ev_sgd0, c->ev_sgd1, c->ev_bsp0, c->ev_bsp1, c->ev_k0, c->ev_k1})
         if (e) cudaEventDestroy(e);
@@ -594,7 +645,19 @@ int pdb_build_conflicts(const pdb_csr *X, pdb_conflicts **out, void *stream)
     cudaEventRecord(c->ev0, s);
     rc = alloc((void **)&c->info, sizeof(int) * INFO_WORDS, s);
     rc = rc ? rc : alloc((void **)&c->csc_pos, sizeof(int32_t) * nnz, s);
-    rc = rc ? rc : alloc((void **)&c->gate, sizeof(uint32_t) * nnz, s);
+    // up to 2^22 slots the gate array (16 MB) stays in L2 and k_slots scatters
+    // it to position order directly; above, the build keeps it in slot order
+    // plus a WINDOW gate holding only the near pairs' words, and the full
+    // position-order array is built on first use (ensure_gate)
+    const bool partition = nnz > 0 && bits_for(nnz - 1) > 22;
+    if (!partition) {
+        rc = rc ? rc : alloc((void **)&c->gate, sizeof(uint32_t) * std::max<int64_t>(nnz, 1), s);
+        c->gate_window = c->gate;
+    } else {
+        rc = rc ? rc : alloc((void **)&c->gate_sorted, sizeof(uint32_t) * nnz, s);
+        rc = rc ? rc : alloc((void **)&c->gate_window, sizeof(uint32_t) * nnz, s);
+        if (rc == PDB_OK) cudaMemsetAsync(c->gate_window, 0, sizeof(uint32_t) * nnz, s);
+    }
     rc = rc ? rc : alloc((void **)&c->feat_ptr, sizeof(int64_t) * (F + 1), s);
     uint32_t *skey = nullptr, *tkey = nullptr;
     int32_t *tval = nullptr;
@@ -616,43 +679,10 @@ int pdb_build_conflicts(const pdb_csr *X, pdb_conflicts **out, void *stream)
     }
     if (rc == PDB_OK) rc = segment_bounds(skey, nnz, F, nullptr, c->feat_ptr, c->info, s);
     if (rc == PDB_OK && nnz > 0) {
-        // up to 2^22 slots the gate array (16 MB) stays in L2 and the direct
-        // scatter is cheapest; above, sort the gate words back to position
-        // order (k_scatter_block)
-        const int pbits = bits_for(nnz - 1);
-        const bool partition = pbits > 22;
-        k_slots<<<grid_1d((nnz + 3) / 4), 256, 0, s>>>(skey, c->csc_pos, nnz, c->feat_ptr, X->row_ptr, N, c->near, c->gate,
-                                             partition ? (uint32_t *)tval : nullptr, c->info);
+        k_slots<<<grid_1d((nnz + 3) / 4), 256, 0, s>>>(skey, c->csc_pos, nnz, c->feat_ptr, X->row_ptr, N, c->near,
+                                                        c->gate, c->gate_sorted, partition ? c->gate_window : nullptr,
+                                                        c->info);
         note_launch();
-        if (partition) {
-            // (position, gate) pairs sorted on the position bits above SCATTER_SB; skey is free after k_slots
-            uint32_t *pk = nullptr;
-            int32_t *pv = nullptr;
-            rc = alloc((void **)&pk, sizeof(uint32_t) * nnz, s);
-            rc = rc ? rc : alloc((void **)&pv, sizeof(int32_t) * nnz, s);
-            if (rc == PDB_OK)
-                rc = radix_sort_bits((const uint32_t *)c->csc_pos, tval, pk, pv, tkey, (int32_t *)skey, nnz,
-                                     SCATTER_SB, pbits, c->info, s);
-            if (rc == PDB_OK) {
-                const size_t smem = sizeof(uint32_t) << SCATTER_SB;
-                static bool configured[64] = {};
-                if (c->device >= 0 && c->device < 64 && !configured[c->device]) {
-                    if (cudaFuncSetAttribute(k_scatter_block, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) !=
-                        cudaSuccess)
-                        rc = PDB_ECUDA;
-                    else
-                        configured[c->device] = true;
-                }
-                if (rc == PDB_OK) {
-                    const int64_t blocks = ((nnz - 1) >> SCATTER_SB) + 1;
-                    k_scatter_block<<<(unsigned)blocks, SCATTER_THREADS, smem, s>>>(pk, (const uint32_t *)pv, nnz,
-                                                                                     c->gate, c->info);
-                    note_launch();
-                }
-            }
-            release(pk, s);
-            release(pv, s);
-        }
     }
     release(skey, s);
     release(tkey, s);
@@ -749,7 +779,9 @@ int pdb_schedule_build(const pdb_conflicts *c, pdb_sched_mode mode, pdb_schedule
         cudaMemsetAsync(h->ticket, 0, sizeof(unsigned long long), s);
     }
     if (mode == PDB_SCHED_READY) {
-        // one (weight, version) record per feature; filled from w by pdb_sgd_epoch
+        // one (weight, version) record per feature; filled from w by pdb_sgd_epoch;
+        // every position's gate word
+        rc = rc ? rc : ensure_gate(cm, s);
         rc = rc ? rc : alloc((void **)&h->rec, sizeof(unsigned long long) * F, s);
     } else if (mode == PDB_SCHED_WINDOW) {
         // near hand-off records (tag 0 = none: tags carry a nonzero epoch
@@ -878,7 +910,7 @@ int pdb_schedule_ready(const pdb_schedule *h, const uint32_t **gate, const uint6
 {
     if (!h) return PDB_EINVAL;
     if (h->mode != PDB_SCHED_READY && h->mode != PDB_SCHED_WINDOW) return PDB_ESTATE;
-    if (gate) *gate = h->c->gate;
+    if (gate) *gate = h->mode == PDB_SCHED_WINDOW ? h->c->gate_window : h->c->gate;
     if (records) *records = (const uint64_t *)h->rec;   // NULL under WINDOW
     return PDB_OK;
 }

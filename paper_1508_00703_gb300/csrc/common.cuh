@@ -244,7 +244,11 @@ struct pdb_conflicts {
     const float *val;
     int32_t *csc_pos;        // positions grouped by feature, data order inside a feature
     int64_t *feat_ptr;       // [F+1]
-    uint32_t *gate;          // per position: occurrence rank and flags (GATE_* below)
+    uint32_t *gate;          // per position: occurrence rank and flags (GATE_* below); above 2^22
+                             // positions built on first use (build.cu) from gate_sorted
+    uint32_t *gate_sorted;   // above 2^22 positions: the gate words in csc_pos order
+    uint32_t *gate_window;   // the WINDOW engine's gate: above 2^22 positions only the words of
+                             // positions with a near pair (0 elsewhere), else = gate
     int64_t near;            // distance (positions) under which an occurrence pair counts as near
     int32_t *row_of;         // example of each position (built on first use)
     int32_t *prev, *next, *rank;  // materialized from the above on first request

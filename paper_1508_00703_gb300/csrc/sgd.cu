@@ -557,7 +557,7 @@ int pdb_sgd_epoch(const pdb_csr *X, const float *y, const pdb_conflicts *c, cons
         } else if (h->mode == PDB_SCHED_WINDOW) {
             cudaEventRecord(cm->ev_k0, s);
             pdb_schedule *hm = const_cast<pdb_schedule *>(h);
-            rc = window_run(X, y, c->gate, w, h->rec, &hm->epochs_run, h->prog, h->prog_cap, h->wctl, c->near, lossi,
+            rc = window_run(X, y, c->gate_window, w, h->rec, &hm->epochs_run, h->prog, h->prog_cap, h->wctl, c->near, lossi,
                             eta, n_epochs, width, opts, cm->status, tmo, s);
             cudaEventRecord(cm->ev_k1, s);
         } else if (block_ready_smem(X->n_cols, c->h_info[2]) > 0 && (int64_t)n_epochs * X->n_rows < (1ll << 31)) {

@@ -157,8 +157,11 @@ __device__ __forceinline__ void publish(int j, uint32_t g, float nw, float *w, u
         __stcg(w + j, nw);
 }
 
-// a previous occurrence that is not near: read from w after the watermark
-__device__ __forceinline__ bool is_far(uint32_t g) { return (g & GATE_RANK) != 0 && !(g & GATE_NEAR_PREV); }
+// no near previous occurrence (far, or none at all): read from w after the
+// watermark; the gate of such a position may carry no rank (inputs above
+// 2^22 positions keep only the near pairs' words), and the watermark
+// condition holds for a first occurrence too
+__device__ __forceinline__ bool is_far(uint32_t g) { return !(g & GATE_NEAR_PREV); }
 
 // this warp's progress word: every chunk it took before `value` is finished
 // and its weights are visible (fence by every lane, then one release store)
