@@ -86,11 +86,21 @@ def test_gate_words_past_the_l2_sized_path(n_rows):
     ref = oracle.chains(p)
     for key in ("prev", "next", "rank"):
         assert np.array_equal(_arr(arrs[key], p.nnz, torch.int32), ref[key]), key
-    s = pdb.pdb_schedule_build(c, pdb.PDB_SCHED_WINDOW)
-    w = torch.zeros(p.n_cols, dtype=torch.float32, device="cuda")
-    pdb.pdb_sgd_epoch(X, y, c, s, w, p.loss, p.eta, 1)
-    pdb.check_status(c)
-    assert np.array_equal(w.cpu().numpy(), oracle.sgd(p, epochs=1))
+    ref_w = oracle.sgd(p, epochs=1)
+    # WINDOW reads the near pairs' gate words only; READY (and the admissible-delay
+    # engine on it) the full position-order gate, built on first use
+    for mode in (pdb.PDB_SCHED_WINDOW, pdb.PDB_SCHED_READY):
+        c = pdb.pdb_build_conflicts(X)
+        s = pdb.pdb_schedule_build(c, mode)
+        w = torch.zeros(p.n_cols, dtype=torch.float32, device="cuda")
+        pdb.pdb_sgd_epoch(X, y, c, s, w, p.loss, p.eta, 1)
+        pdb.check_status(c)
+        assert np.array_equal(w.cpu().numpy(), ref_w), mode
+        if mode == pdb.PDB_SCHED_READY:
+            w.zero_()
+            pdb.pdb_ssp_epoch(X, y, c, s, w, p.loss, p.eta, 1, 0)
+            pdb.check_status(c)
+            assert np.array_equal(w.cpu().numpy(), ref_w), "admissible delay 0"
 
 
 @pytest.mark.parametrize("sweep", ["flow", "kahn"])
