@@ -1,0 +1,73 @@
+"""The oracle's pins catch plausible mistakes.
+
+Each case copies oracle/pdb_oracle.c, plants one mistake in the copy (the
+committed file is never touched), builds it here on the CPU, points the
+oracle module at the planted build, and runs the pins that guard that
+routine: at least one of them must fail.  The pins compare against
+mathematics (fp64, exact sums, closed forms, brute force), so a mistake in
+the oracle cannot hide behind a matching mistake in its check."""
+import subprocess
+
+import pytest
+
+import oracle
+from tests import test_oracle_numerics as num
+from tests import test_oracle_schedule as sched
+from tests import test_oracle_sgd as sgd
+
+# name -> (text in pdb_oracle.c, planted text, pins that must catch it)
+PLANTS = {
+    "taylor-coefficient": (
+        "p = fmaf(p, r, (float)(1.0 / 120.0));", "p = fmaf(p, r, (float)(1.0 / 121.0));",
+        [num.test_expf_within_2ulp_dense_grid, num.test_expf_within_2ulp_random_and_small]),
+    "cody-waite-tail-dropped": (
+        "r = r - kf * ln2_lo;", "r = r;",
+        [num.test_expf_within_2ulp_dense_grid, num.test_expf_within_2ulp_random_and_small]),
+    "exp-argument-sign": (
+        "return -y / (1.0f + orc_expf(y * m));", "return -y / (1.0f + orc_expf(-y * m));",
+        [num.test_grad_logistic_closed_forms, num.test_grad_logistic_matches_fp64]),
+    "butterfly-stage-missing": (
+        "for (int off = 16; off >= 1; off >>= 1) {", "for (int off = 16; off >= 2; off >>= 1) {",
+        [num.test_dot_exact_on_small_integers, num.test_dot_uses_32_partial_sums]),
+    "sixteen-partial-sums": (
+        "a[i % 32] = fmaf(w[col[i]], val ? val[i] : 1.0f, a[i % 32]);",
+        "a[i % 16] = fmaf(w[col[i]], val ? val[i] : 1.0f, a[i % 16]);",
+        [num.test_dot_uses_32_partial_sums, num.test_dot_error_bound_random]),
+    "hinge-tie": (
+        "return (y * m < 1.0f) ? -y : 0.0f;", "return (y * m <= 1.0f) ? -y : 0.0f;",
+        [num.test_grad_squared_and_hinge]),
+    "update-sign": (
+        "w[col[b + i]] = w[col[b + i]] - c * x;", "w[col[b + i]] = w[col[b + i]] + c * x;",
+        [sgd.test_one_logistic_step_from_zero, sgd.test_squared_loss_geometric_closed_form]),
+    "chain-rank-off-by-one": (
+        "rank[p] = (int32_t)cnt[j];", "rank[p] = (int32_t)cnt[j] + 1;",
+        [lambda: sched.test_chains_brute_force(0), lambda: sched.test_chains_brute_force(1)]),
+    "level-first-position-ignored": (
+        "if (prev[p] >= 0 && level[row_of[prev[p]]] > lv)", "if (prev[p] > 0 && level[row_of[prev[p]]] > lv)",
+        [sched.test_levels_single_predecessor_chain] +
+        [lambda s=s: sched.test_levels_equal_brute_force(s) for s in range(16)]),
+    "bsp-sum-not-reset": (
+        "delta[col[p]] = 0.0f;", ";",
+        [lambda: sgd.test_bsp_batch_one_is_sequential(oracle.LOGISTIC), sgd.test_bsp_short_last_batch]),
+}
+
+
+@pytest.mark.parametrize("name", list(PLANTS))
+def test_planted_mistake_fails_a_pin(name, tmp_path, monkeypatch):
+    old, new, pins = PLANTS[name]
+    src = open(oracle._SRC).read()
+    assert src.count(old) == 1, "the planted text must name one place"
+    planted = tmp_path / "pdb_oracle.c"
+    planted.write_text(src.replace(old, new))
+    lib = tmp_path / "liboracle.so"
+    subprocess.run(["gcc", "-O2", "-std=c11", "-shared", "-fPIC", "-ffp-contract=off", "-fno-fast-math",
+                    "-o", str(lib), str(planted), "-lm"], check=True)
+    monkeypatch.setattr(oracle, "build", lambda: str(lib))
+    monkeypatch.setattr(oracle, "_lib", None)
+    caught = 0
+    for pin in pins:
+        try:
+            pin()
+        except AssertionError:
+            caught += 1
+    assert caught > 0, f"no pin caught the planted mistake {name!r}"

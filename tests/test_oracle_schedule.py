@@ -72,6 +72,17 @@ def test_levels_equal_brute_force(seed):
     assert L == (bf.max() + 1 if bf.size else 0)
 
 
+def test_levels_single_predecessor_chain():
+    # each example shares exactly one feature with the one before (the first
+    # link is position 0): the levels count the hops, 0, 1, 2, ...; an
+    # example that reuses no feature stays at level 0
+    p = synthdata.from_arrays([0, 1, 3, 5, 7, 8], [0, 0, 1, 1, 2, 2, 3, 9], None, np.ones(5), n_cols=10)
+    lv, L = oracle.levels(p)
+    assert lv.tolist() == [0, 1, 2, 3, 0]
+    assert L == 4
+    assert np.array_equal(lv, oracle.levels_bruteforce(p))
+
+
 def _check_level_invariants(p, lv):
     sets = [set(p.col[p.row_ptr[t]:p.row_ptr[t + 1]].tolist()) for t in range(p.n_rows)]
     by_level = {}
