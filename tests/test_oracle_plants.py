@@ -46,6 +46,26 @@ PLANTS = {
         "if (prev[p] >= 0 && level[row_of[prev[p]]] > lv)", "if (prev[p] > 0 && level[row_of[prev[p]]] > lv)",
         [sched.test_levels_single_predecessor_chain] +
         [lambda s=s: sched.test_levels_equal_brute_force(s) for s in range(16)]),
+    "squared-loss-sign": (
+        "if (loss == ORC_SQUARED) return m - y;", "if (loss == ORC_SQUARED) return y - m;",
+        [num.test_grad_squared_and_hinge, sgd.test_squared_loss_geometric_closed_form]),
+    "exp-scale-not-split": (
+        "int h = k / 2;", "int h = k;",
+        [num.test_expf_special_values, num.test_expf_subnormal_results_correctly_scaled,
+         num.test_expf_within_2ulp_dense_grid]),
+    "chain-next-not-linked": (
+        "if (last[j] >= 0) next[last[j]] = (int32_t)p;", ";",
+        [lambda: sched.test_chains_brute_force(0), lambda: sched.test_chains_brute_force(1)]),
+    "level-order-reversed-in-level": (
+        "for (int64_t t = 0; t < n_rows; ++t) order[fill[level[t]]++] = (int32_t)t;",
+        "for (int64_t t = n_rows - 1; t >= 0; --t) order[fill[level[t]]++] = (int32_t)t;",
+        [sched.test_level_order_is_stable_by_level_then_id]),
+    "bsp-batch-not-snapshot": (
+        "float m = orc_dot(w, col + b, val ? val + b : NULL, k);\n                c[t - b0] = eta * orc_grad(loss, m, y[t]);",
+        "float m = orc_dot(w, col + b, val ? val + b : NULL, k);\n                c[t - b0] = eta * orc_grad(loss, m, y[t]);\n"
+        "                for (int64_t p = b; p < b + k; ++p) w[col[p]] = w[col[p]] - c[t - b0] * (val ? val[p] : 1.0f);",
+        [lambda: sgd.test_bsp_full_batch_is_gradient_descent(oracle.LOGISTIC),
+         lambda: sgd.test_bsp_full_batch_is_gradient_descent(oracle.SQUARED)]),
     "bsp-sum-not-reset": (
         "delta[col[p]] = 0.0f;", ";",
         [lambda: sgd.test_bsp_batch_one_is_sequential(oracle.LOGISTIC), sgd.test_bsp_short_last_batch]),
