@@ -7,10 +7,13 @@ routine: at least one of them must fail.  The pins compare against
 mathematics (fp64, exact sums, closed forms, brute force), so a mistake in
 the oracle cannot hide behind a matching mistake in its check."""
 import subprocess
+from collections import defaultdict
 
 import pytest
 
 import oracle
+from oracle import history
+from tests import test_history as th
 from tests import test_oracle_numerics as num
 from tests import test_oracle_schedule as sched
 from tests import test_oracle_sgd as sgd
@@ -84,6 +87,69 @@ def test_planted_mistake_fails_a_pin(name, tmp_path, monkeypatch):
                     "-o", str(lib), str(planted), "-lm"], check=True)
     monkeypatch.setattr(oracle, "build", lambda: str(lib))
     monkeypatch.setattr(oracle, "_lib", None)
+    caught = 0
+    for pin in pins:
+        try:
+            pin()
+        except AssertionError:
+            caught += 1
+    assert caught > 0, f"no pin caught the planted mistake {name!r}"
+
+
+# ------------------------------------------------------------------ history
+# The checker of execution histories and traces (oracle/history.py) is
+# pinned the same way: a copy of one predicate with a mistake replaces it.
+
+
+def _rc_only(ops):
+    """The Read Constraint alone (a checker that forgot the Write Constraint)."""
+    pos_w = {}
+    for q, (kind, _, chunk, it) in enumerate(ops):
+        if kind == "w":
+            pos_w[(chunk, it)] = q
+    for q, (kind, _, chunk, it) in enumerate(ops):
+        if kind == "r" and it > 1:
+            wq = pos_w.get((chunk, it - 1))
+            if wq is None or wq > q:
+                return False
+    return True
+
+
+def _wc_only(ops):
+    """The Write Constraint alone (a checker that forgot the Read Constraint)."""
+    reads = defaultdict(list)
+    for q, (kind, _, chunk, it) in enumerate(ops):
+        if kind == "r":
+            reads[(chunk, it)].append(q)
+    for q, (kind, _, chunk, it) in enumerate(ops):
+        if kind == "w" and any(rq > q for rq in reads[(chunk, it)]):
+            return False
+    return True
+
+
+def _no_pair_breaks(row_ptr, col, n_epochs, trace):
+    v = _order_violations(row_ptr, col, n_epochs, trace)
+    v["rc"] = 0
+    return v
+
+
+_order_violations = history.trace_order_violations
+
+PY_PLANTS = {
+    "write-constraint-ignored": ("satisfies_rc_wc", _rc_only,
+                                 [lambda r=r: th.test_paper_histories(*r) for r in th._golden()]),
+    "read-constraint-ignored": ("satisfies_rc_wc", _wc_only,
+                                [th.test_theorem2_random_executions, th.test_trace_batch_with_conflicts_is_rejected]),
+    "trace-pairs-ignored": ("trace_order_violations", _no_pair_breaks,
+                            [th.test_trace_batch_with_conflicts_is_rejected] +
+                            [lambda s=s: th.test_trace_checkers_match_brute_force(s) for s in range(6)]),
+}
+
+
+@pytest.mark.parametrize("name", list(PY_PLANTS))
+def test_planted_checker_mistake_fails_a_pin(name, monkeypatch):
+    attr, fn, pins = PY_PLANTS[name]
+    monkeypatch.setattr(history, attr, fn)
     caught = 0
     for pin in pins:
         try:
