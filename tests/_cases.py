@@ -27,6 +27,8 @@ SMALL = {
     "dense-narrow": ("dense-lr", dict(n_rows=1500, n_cols=200, k=200, epochs=2, bsp_batch=1500)),
     # the full 960-feature width (rows of 513..1024 ids: 32 registers per lane)
     "dense-wide": ("dense-lr", dict(n_rows=300, epochs=2, bsp_batch=300)),
+    # rows longer than 1024 ids: the resident engine's two-pass path
+    "dense-xwide": ("dense-lr", dict(n_rows=120, n_cols=1500, k=1500, epochs=1, bsp_batch=120)),
 }
 
 FULL = {
