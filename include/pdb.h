@@ -36,6 +36,12 @@
  *   - Calls that share a handle must be ordered on one stream (the handles
  *     hold device-side counters that a concurrent call would clobber).
  *   - Limits: n_rows, n_cols and nnz below 2^31 (positions and ids are int32).
+ *   - Diagnostics: every call opens an NVTX range named after it (seen by
+ *     profilers); with the environment variable PDB_LOG set to anything but
+ *     "" or "0" each call (but pdb_sgd_epoch_ready_noalloc) prints one line
+ *     of pdb_get_stats on stderr afterwards, which synchronizes the device.
+ *     PDB_NEAR (pdb_build_conflicts) and PDB_LEVELS (pdb_schedule_build)
+ *     are described where they apply.
  */
 #ifndef PDB_H
 #define PDB_H
