@@ -1,5 +1,6 @@
 """Host logic of bench.py: the replica aggregation across ranks (gloo,
-world size 2, on CPU) and the JSON line of the reference arm."""
+world size 2, on CPU), the JSON line of the reference arm, the clock
+summary and the recorded-traffic check."""
 import json
 import os
 import socket
@@ -63,3 +64,44 @@ def test_reference_arm_other_ranks_exit_quietly():
     out = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference", "--workload", "tiny"],
                          capture_output=True, text=True, timeout=120, cwd=ROOT, env=env)
     assert out.returncode == 0 and out.stdout.strip() == ""
+
+
+def test_clock_summary_reads_samples_and_throttle_reasons(tmp_path):
+    # nvidia-smi --format=csv,noheader,nounits rows as the sampler records them
+    sys.path.insert(0, ROOT)
+    import bench
+    csv = tmp_path / "clocks.csv"
+    csv.write_text("0, 2070, 2070, 450.10, 0x0000000000000000, Not Active, Not Active, Not Active, Not Active\n"
+                   "0, 1995, 2070, 1399.70, 0x0000000000000004, Not Active, Not Active, Not Active, Active\n"
+                   "0, 2070, 2070, 600.00, 0x0000000000000000, Not Active, Not Active, Not Active, Not Active\n"
+                   "garbled line\n")
+
+    class _File:
+        name = str(csv)
+
+    smp = bench.ClockSampler.__new__(bench.ClockSampler)
+    smp.gpu, smp.proc, smp.file = "0", object(), _File()
+    s = smp.summary()
+    assert s["samples"] == 3 and s["sm_mhz"] == 2070.0 and s["sm_max_mhz"] == 2070.0
+    assert s["power_w_max"] == 1399.7 and s["reasons"] == ["sw_power_cap"]
+
+
+def test_recorded_traffic_only_while_the_sources_match(tmp_path, monkeypatch):
+    # the committed ncu traffic is reported only while the kernel's sources
+    # hash as they did when it was captured
+    sys.path.insert(0, ROOT)
+    import hashlib
+    import bench
+    csrc = tmp_path / "paper_1508_00703_gb300" / "csrc"
+    csrc.mkdir(parents=True)
+    (csrc / "window.cu").write_text("kernel A\n")
+    (csrc / "common.cuh").write_text("helpers\n")
+    (tmp_path / "profiles").mkdir()
+    h = hashlib.sha256(b"kernel A\n" + b"helpers\n").hexdigest()
+    (tmp_path / "profiles" / "k_sgd_window_low-conflict.md").write_text(
+        f"traffic_bytes_per_launch: 123456\nsource_sha256: {h}\n")
+    monkeypatch.setattr(bench, "ROOT", str(tmp_path))
+    assert bench.recorded_traffic("k_sgd_window", "low-conflict") == 123456.0
+    (csrc / "window.cu").write_text("kernel B\n")
+    assert bench.recorded_traffic("k_sgd_window", "low-conflict") is None
+    assert bench.recorded_traffic("k_sgd_window", "zipf-1m") is None
