@@ -1,0 +1,143 @@
+"""A model check of the WINDOW schedule's protocol, on the CPU.
+
+The WINDOW engine lets a position read its feature's weight in one of two
+ways: if the previous occurrence lies closer than `near` positions, from a
+hand-off record tagged with the reader's occurrence rank (and epoch); else
+(previous occurrence far, or none at all) from the plain weight array once
+the completion watermark -- the first position of the oldest unfinished
+chunk of examples -- has reached min(first position of the reader's chunk,
+end of the reader's example - near).  A position writes into the record when
+its next occurrence is near, else into the array.
+
+This test restates those rules as a state machine, runs it under random
+interleavings of workers that take chunks of examples in data order, with
+every read and every write of every position a separate step, and checks
+that each read observes exactly the write of the previous occurrence of its
+feature in data order (the Read Constraint of Section 4.4, which with one
+writer per occurrence gives the sequential result, Theorem 2), and that the
+workers never deadlock.  Occurrence chains come from the oracle.  The model
+uses the exact watermark; the engine's lags behind it (workers publish their
+progress late), which only makes reads wait longer."""
+import numpy as np
+import pytest
+
+import oracle
+import synthdata
+
+
+def _simulate(p, near, chunk, n_workers, epochs, rng, watermark_wait=True):
+    ch = oracle.chains(p)
+    prev, nxt, rank = ch["prev"], ch["next"], ch["rank"]
+    row_ptr, col = p.row_ptr, p.col
+    n = p.n_rows
+    row_of = np.repeat(np.arange(n), np.diff(row_ptr))
+    pos = np.arange(p.nnz)
+    near_prev = (prev >= 0) & (pos - prev < near)
+    near_next = (nxt >= 0) & (nxt - pos < near)
+    n_chunks = (n + chunk - 1) // chunk
+    w_src = {}            # feature -> (epoch, example) whose write sits in the array
+    rec = {}              # feature -> (tag, epoch, example) of the last record write
+    for ep in range(epochs):
+        chunk_done = np.zeros(n_chunks, bool)
+        next_ticket = 0
+        # worker state: [chunk, example index in chunk, phase, positions pending]
+        workers = [None] * n_workers
+        steps = 0
+        while not chunk_done.all():
+            steps += 1
+            assert steps < 100 * (p.nnz + n + 10), "no progress"
+            first_open = int(np.argmin(chunk_done)) if not chunk_done.all() else n_chunks
+            watermark = int(row_ptr[min(first_open * chunk, n)])
+            enabled = []
+            for wi, st in enumerate(workers):
+                if st is None:
+                    if next_ticket < n_chunks:
+                        enabled.append((wi, "take", None))
+                    continue
+                c, ti, phase, pending = st
+                t = c * chunk + ti
+                b, e = int(row_ptr[t]), int(row_ptr[t + 1])
+                for q in pending:
+                    if phase == "read":
+                        if near_prev[q]:
+                            r = rec.get(int(col[q]))
+                            ok = r is not None and r[0] == (int(rank[q]), ep)
+                        else:
+                            need = min(int(row_ptr[c * chunk]), e - near)
+                            ok = watermark >= need or not watermark_wait
+                    else:
+                        ok = True
+                    if ok:
+                        enabled.append((wi, phase, q))
+                if not pending:
+                    enabled.append((wi, "next", None))
+            assert enabled, "deadlock"
+            wi, kind, q = enabled[rng.integers(len(enabled))]
+            if kind == "take":
+                c = next_ticket
+                next_ticket += 1
+                t0 = c * chunk
+                if t0 >= n:
+                    chunk_done[c] = True
+                    continue
+                workers[wi] = [c, 0, "read", list(range(int(row_ptr[t0]), int(row_ptr[t0 + 1])))]
+                continue
+            c, ti, phase, pending = workers[wi]
+            t = c * chunk + ti
+            if kind == "read":
+                j = int(col[q])
+                seen = (rec[j][1], rec[j][2]) if near_prev[q] else w_src.get(j)
+                if prev[q] >= 0:
+                    want = (ep, int(row_of[prev[q]]))
+                else:                                   # first occurrence of the epoch
+                    last = ch["feat_ptr"][j + 1] - 1    # the feature's last position
+                    want = (ep - 1, int(row_of[ch["csc_pos"][last]])) if ep > 0 else None
+                assert seen == want, (ep, t, q, seen, want)
+                pending.remove(q)
+                if not pending:
+                    workers[wi] = [c, ti, "write", list(range(int(row_ptr[t]), int(row_ptr[t + 1])))]
+            elif kind == "write":
+                j = int(col[q])
+                if near_next[q]:
+                    rec[j] = ((int(rank[q]) + 1, ep), ep, t)
+                else:
+                    w_src[j] = (ep, t)
+                pending.remove(q)
+            else:                                       # the example is finished
+                ti += 1
+                t = c * chunk + ti
+                if ti < chunk and t < n:
+                    workers[wi] = [c, ti, "read", list(range(int(row_ptr[t]), int(row_ptr[t + 1])))]
+                else:
+                    chunk_done[c] = True
+                    workers[wi] = None
+    # after the last epoch every feature's array entry holds its last writer
+    for j in range(p.n_cols):
+        cnt = ch["feat_ptr"][j + 1] - ch["feat_ptr"][j]
+        if cnt:
+            last = ch["feat_ptr"][j + 1] - 1
+            assert w_src[j] == (epochs - 1, int(row_of[ch["csc_pos"][last]]))
+
+
+@pytest.mark.parametrize("seed", range(12))
+def test_window_protocol_reads_follow_data_order(seed):
+    rng = np.random.default_rng(seed)
+    p = synthdata.generate("tiny", seed=seed, n_rows=int(rng.integers(30, 90)), n_cols=int(rng.integers(6, 40)),
+                           k=int(rng.integers(1, 6)), k_lo=0, ids="zipf" if seed % 2 else "uniform", zipf_s=1.1)
+    near = int(rng.choice([1, 2, 5, 20, 10 ** 6]))     # all far .. all near
+    _simulate(p, near=near, chunk=int(rng.integers(1, 4)), n_workers=int(rng.integers(1, 7)),
+              epochs=int(rng.integers(1, 3)), rng=rng)
+
+
+def test_window_protocol_model_rejects_a_missing_wait():
+    # planted in the model: far reads skip the watermark; some interleaving
+    # then reads a weight before its previous occurrence has written it
+    rng = np.random.default_rng(7)
+    p = synthdata.generate("tiny", seed=3, n_rows=60, n_cols=6, k=3, k_lo=1)
+    failures = 0
+    for _ in range(20):
+        try:
+            _simulate(p, near=1, chunk=1, n_workers=6, epochs=1, rng=rng, watermark_wait=False)
+        except AssertionError:
+            failures += 1
+    assert failures > 0
