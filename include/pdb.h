@@ -263,8 +263,12 @@ int pdb_sgd_epoch(const pdb_csr *X, const float *y, const pdb_conflicts *c, cons
  * w_j (an atomic fp32 add of -(eta*g)*x_j, then the write is counted), so
  * every example's update is applied exactly once.  w is updated in place.
  *   delay = 0    the sequential result, bitwise equal to pdb_sgd_epoch
- *   delay > 0    reads may be up to `delay` occurrences stale; the result
- *                depends on timing and is not deterministic
+ *   delay > 0    a read sees at least r - delay of the writes of its
+ *                feature; the result depends on timing and is not
+ *                deterministic.  The write gate counts reads, so a slow
+ *                reader holds no writer back: its read may also see writes
+ *                of later occurrences (the paper's Write Protocol, which
+ *                waits for the slowest reader, would bound those too)
  *   delay >= the longest chain  no waits at all (Hogwild with atomic updates)
  *   coef         optional device array of n_epochs * n_rows floats (NULL for
  *                none): the step eta*g each example applied, epoch-major,

@@ -8,10 +8,17 @@
 //          r - delta writes of j are done (its view is at most delta
 //          occurrences stale);
 //   write  it may write once at least r - delta + 1 occurrences of j have
-//          read (no reader lags the writer by more than delta), and it
-//          applies its step to the current w_j with an atomic fp32 add of
-//          -(eta*g*x_j), then counts the write (release): no update is lost
-//          even when a later occurrence wrote first, and nothing retries.
+//          read, and it applies its step to the current w_j with an atomic
+//          fp32 add of -(eta*g*x_j), then counts the write (release): no
+//          update is lost even when a later occurrence wrote first, and
+//          nothing retries.
+//
+// Counts equal the paper's per-iteration conditions only while reads and
+// writes complete in rank order, which delta = 0 forces.  For delta >= 1 the
+// read gate still bounds staleness from below, but the write gate counts any
+// r - delta + 1 reads: a slow reader of low rank holds no writer back (the
+// paper's Write Protocol waits for the slowest reader), so its read may see
+// writes of occurrences delta or more ranks after it.
 //
 // delta = 0 is the sequential computation: the reader of rank r sees exactly
 // r writes, nobody else writes between its read and its write, and
