@@ -53,6 +53,8 @@ def parse_args(argv=None):
                     help="time pdb_bsp_epoch with this mini-batch instead of pdb_sgd_epoch (-1: the workload's own)")
     ap.add_argument("--delay", type=int, default=None,
                     help="time pdb_ssp_epoch (admissible delay, READY schedule) with this delay instead")
+    ap.add_argument("--ssp-gates", choices=["count", "prefix"], default="count",
+                    help="with --delay: counting gates, or prefix gates (a writer waits for the slowest reader)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=10.0, help="target length of the CPU oracle sample")
@@ -301,7 +303,9 @@ def run_ours(args, rank, world, local_rank):
             return c, None
         if args.delay is not None:
             s = pdb.pdb_schedule_build(c, pdb.PDB_SCHED_READY, stream)
-            pdb.pdb_ssp_epoch(X, y, c, s, w, p.loss, p.eta, E, args.delay, opts=opts, stream=stream)
+            gates = pdb.PDB_SSP_PREFIX if args.ssp_gates == "prefix" else pdb.PDB_SSP_COUNT
+            pdb.pdb_ssp_epoch(X, y, c, s, w, p.loss, p.eta, E, args.delay, opts=dict(opts, ssp_gates=gates),
+                              stream=stream)
             return c, s
         s = pdb.pdb_schedule_build(c, mode, stream)
         pdb.pdb_sgd_epoch(X, y, c, s, w, p.loss, p.eta, E, opts=opts, stream=stream)
@@ -394,6 +398,7 @@ def run_ours(args, rank, world, local_rank):
     if args.delay is not None:
         result["metric"] = METRIC.replace("serially-equivalent sparse SGD",
                                           f"admissible-delay ({args.delay}) sparse SGD")
+        result["config"]["ssp_gates"] = args.ssp_gates
         if args.delay > 0:
             result["config"]["note"] = "delay > 0: not serially equivalent, result depends on timing"
     if batch:

@@ -130,6 +130,15 @@ typedef enum {
     PDB_SCHED_WINDOW = 4
 } pdb_sched_mode;
 
+/* Gates of pdb_ssp_epoch (Section 7; iterations counted per feature, the
+ * occurrence of feature j with rank r being iteration r of j). */
+typedef enum {
+    PDB_SSP_COUNT = 1,  /* counters: rank r reads once r - delay writes of j are done and writes once
+                         * r - delay + 1 occurrences of j have read (the default) */
+    PDB_SSP_PREFIX = 2  /* prefixes: rank r reads once every rank <= r - 1 - delay has written and writes
+                         * once every rank <= r - delay has read (the Write Protocol's slowest reader) */
+} pdb_ssp_gates;
+
 /* Launch and wait options; a zeroed struct (or NULL) selects the defaults. */
 typedef struct {
     int32_t blocks_per_sm;     /* persistent grid = blocks_per_sm x #SM; 0 = occupancy maximum */
@@ -141,6 +150,7 @@ typedef struct {
                                 * and before any of its writes is issued, so a caller can check an
                                 * execution against the Read and Write Constraints (Section 4.4) or the
                                 * asynchronous ones (Section 7).  Costs two stores per example. */
+    int32_t ssp_gates;         /* pdb_ssp_epoch: a pdb_ssp_gates value; 0 = PDB_SSP_COUNT */
 } pdb_opts;
 
 /* Sizes and timings; timings are CUDA-event milliseconds of the last call of
@@ -265,16 +275,20 @@ int pdb_sgd_epoch(const pdb_csr *X, const float *y, const pdb_conflicts *c, cons
  *   delay = 0    the sequential result, bitwise equal to pdb_sgd_epoch
  *   delay > 0    a read sees at least r - delay of the writes of its
  *                feature; the result depends on timing and is not
- *                deterministic.  The write gate counts reads, so a slow
- *                reader holds no writer back: its read may also see writes
- *                of later occurrences (the paper's Write Protocol, which
- *                waits for the slowest reader, would bound those too)
+ *                deterministic.  Under PDB_SSP_COUNT the write gate counts
+ *                reads, so a slow reader holds no writer back: its read may
+ *                also see writes of later occurrences.  Under PDB_SSP_PREFIX
+ *                (the paper's Write Protocol: a writer waits for the slowest
+ *                reader) a read of rank r sees every write of rank
+ *                <= r - 1 - delay and none of rank >= r + delay; it keeps a
+ *                done-bitmap per direction (nnz / 4 bytes in all, allocated
+ *                on first use with the schedule)
  *   delay >= the longest chain  no waits at all (Hogwild with atomic updates)
  *   coef         optional device array of n_epochs * n_rows floats (NULL for
  *                none): the step eta*g each example applied, epoch-major,
  *                for auditing a delayed run
- * s must be a READY schedule of c (PDB_ESTATE otherwise); delay < 0 is
- * PDB_EINVAL.  Every wait is bounded (pdb_opts.wait_timeout_s). */
+ * s must be a READY schedule of c (PDB_ESTATE otherwise); delay < 0 or an
+ * unknown opts->ssp_gates is PDB_EINVAL.  Every wait is bounded (pdb_opts.wait_timeout_s). */
 int pdb_ssp_epoch(const pdb_csr *X, const float *y, const pdb_conflicts *c, const pdb_schedule *s, float *w,
                   pdb_loss loss, float eta, int n_epochs, int64_t delay, float *coef, const pdb_opts *opts,
                   void *stream);

@@ -30,6 +30,7 @@ PDB_ETOOBIG = -9
 NOALLOC_MAX_COLS = 1 << 20
 PDB_LOSS_LOGISTIC, PDB_LOSS_SQUARED, PDB_LOSS_HINGE = 0, 1, 2
 PDB_SCHED_LEVELS, PDB_SCHED_READY, PDB_SCHED_CHAIN, PDB_SCHED_AUTO, PDB_SCHED_WINDOW = 0, 1, 2, 3, 4
+PDB_SSP_COUNT, PDB_SSP_PREFIX = 1, 2
 
 _lock = threading.Lock()
 _lib = None
@@ -90,7 +91,7 @@ class pdb_csr(ctypes.Structure):
 
 class pdb_opts(ctypes.Structure):
     _fields_ = [("blocks_per_sm", ctypes.c_int32), ("ticket_chunk", ctypes.c_int32),
-                ("wait_timeout_s", ctypes.c_double), ("trace", ctypes.c_void_p)]
+                ("wait_timeout_s", ctypes.c_double), ("trace", ctypes.c_void_p), ("ssp_gates", ctypes.c_int32)]
 
 
 class pdb_stats(ctypes.Structure):

@@ -732,7 +732,7 @@ void pdb_schedule_free(pdb_schedule *s)
     if (!s) return;
     cudaDeviceSynchronize();
     free_ptrs({s->level, s->order, s->indeg, s->queue, s->level_ptr, s->ctl, s->rec, s->link, s->bar, s->ticket,
-               s->prog, s->wctl, s->reads, s->writes});
+               s->prog, s->wctl, s->reads, s->writes, s->rbits, s->wbits});
     if (s->ev0) cudaEventDestroy(s->ev0);
     if (s->ev1) cudaEventDestroy(s->ev1);
     delete s;

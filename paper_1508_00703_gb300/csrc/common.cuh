@@ -222,9 +222,12 @@ struct WindowCtl {
     long long wpos;             // every example starting below this position has finished
 };
 
+// admissible delay; rbits == nullptr selects the counting gates, else the
+// prefix gates on the done-bitmaps rbits / wbits (n_words words each)
 int ssp_run(const pdb_csr *X, const float *y, const uint32_t *gate, float *w, unsigned *writes, unsigned *reads,
             unsigned long long *ticket, long long delay, float *coef, int loss, float eta, int n_epochs, int width,
-            const pdb_opts *opts, int *status, uint64_t timeout, cudaStream_t s);
+            const pdb_opts *opts, int *status, uint64_t timeout, cudaStream_t s, const int64_t *feat_ptr,
+            unsigned *rbits, unsigned *wbits, int64_t n_words);
 
 int ensure_row_of(pdb_conflicts *c, cudaStream_t s);   // builds c->row_of on first use (stream-ordered)
 
@@ -276,7 +279,9 @@ struct pdb_schedule {
     int64_t *level_ptr;
     LevelCtl *ctl;            // device
     unsigned long long *rec;  // READY: per feature (weight bits | version << 32); WINDOW: near hand-offs
-    unsigned *reads, *writes; // READY under pdb_ssp_epoch: reads / writes of each feature this epoch (first use)
+    unsigned *reads, *writes; // READY under pdb_ssp_epoch: reads / writes of each feature this epoch (first use);
+                              // under prefix gates the known-done prefix of each feature's reads / writes
+    unsigned *rbits, *wbits;  // READY under pdb_ssp_epoch with prefix gates: done-bitmaps over the CSC slots
     uint32_t *link;           // CHAIN: per position, receive flag and push target
     bool resident;            // CHAIN: weights resident in shared memory (no link words)
     unsigned epochs_run;      // WINDOW: epochs run so far (epoch stamp of the record tags)

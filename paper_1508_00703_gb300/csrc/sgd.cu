@@ -598,6 +598,9 @@ int pdb_ssp_epoch(const pdb_csr *X, const float *y, const pdb_conflicts *c, cons
     if (rc != PDB_OK) return rc;
     if (!h || h->c != c || delay < 0) return PDB_EINVAL;
     if (h->mode != PDB_SCHED_READY) return PDB_ESTATE;
+    const int gates = opts ? opts->ssp_gates : 0;
+    if (gates < 0 || gates > PDB_SSP_PREFIX) return PDB_EINVAL;
+    const bool prefix = gates == PDB_SSP_PREFIX;
     cudaStream_t s = (cudaStream_t)stream;
     pdb_conflicts *cm = const_cast<pdb_conflicts *>(c);
     pdb_schedule *hm = const_cast<pdb_schedule *>(h);
@@ -607,11 +610,19 @@ int pdb_ssp_epoch(const pdb_csr *X, const float *y, const pdb_conflicts *c, cons
         rc = rc ? rc : alloc((void **)&hm->writes, sizeof(unsigned) * std::max<int64_t>(X->n_cols, 1), s);
         if (rc != PDB_OK) return rc;
     }
+    // one bit per CSC slot, two words of slack past the last slot's word
+    const int64_t n_words = X->nnz / 32 + 2;
+    if (prefix && !hm->rbits) {
+        rc = alloc((void **)&hm->rbits, sizeof(unsigned) * n_words, s);
+        rc = rc ? rc : alloc((void **)&hm->wbits, sizeof(unsigned) * n_words, s);
+        if (rc != PDB_OK) return rc;
+    }
     cudaEventRecord(cm->ev_sgd0, s);
     cudaEventRecord(cm->ev_k0, s);
     if (X->n_rows > 0 && n_epochs > 0)
         rc = ssp_run(X, y, c->gate, w, hm->writes, hm->reads, h->ticket, (long long)std::min<int64_t>(delay, 1ll << 40),
-                     coef, (int)loss, eta, n_epochs, width, opts, cm->status, timeout_ns(opts), s);
+                     coef, (int)loss, eta, n_epochs, width, opts, cm->status, timeout_ns(opts), s, c->feat_ptr,
+                     prefix ? hm->rbits : nullptr, prefix ? hm->wbits : nullptr, n_words);
     cudaEventRecord(cm->ev_k1, s);
     cudaEventRecord(cm->ev_sgd1, s);
     cm->timed_sgd = true;

@@ -6,7 +6,7 @@ cudaMalloc cannot be captured, or a process whose memory pool owns the whole
 device): its scratch is a fixed array inside the library.  Here it must give
 the same weights as pdb_sgd_epoch with a READY schedule, on two calls in a
 row (the second continues from the first's weights, so the shared scratch
-must be reset correctly between calls).  This file is collected last."""
+must be reset correctly between calls)."""
 import numpy as np
 import pytest
 
