@@ -6,7 +6,9 @@ oracle module at the planted build, and runs the pins that guard that
 routine: at least one of them must fail.  The pins compare against
 mathematics (fp64, exact sums, closed forms, brute force), so a mistake in
 the oracle cannot hide behind a matching mistake in its check."""
+import inspect
 import subprocess
+import textwrap
 from collections import defaultdict
 
 import pytest
@@ -152,6 +154,37 @@ def test_planted_checker_mistake_fails_a_pin(name, monkeypatch):
     monkeypatch.setattr(history, attr, fn)
     caught = 0
     for pin in pins:
+        try:
+            pin()
+        except AssertionError:
+            caught += 1
+    assert caught > 0, f"no pin caught the planted mistake {name!r}"
+
+
+# Mistakes planted by editing one line of a copy of a checker's source.
+PY_TEXT_PLANTS = {
+    "delay-need-off-by-one": (
+        "trace_delay_violations", "need = rank[(o[rd] - u.size)] - delay",
+        "need = rank[(o[rd] - u.size)] - delay - 1"),
+    "delay-group-first-write-dropped": (
+        "trace_delay_violations", "done = cw - (cw[base] - is_w[base])", "done = cw - cw[base]"),
+    "delay-ties-read-first": (
+        "trace_delay_violations", "o = np.lexsort((kind, times, keys))", "o = np.lexsort((-kind, times, keys))"),
+}
+_DELAY_PINS = ([lambda s=s: th.test_trace_checkers_match_brute_force(s) for s in range(6)] +
+               [th.test_trace_delay_fully_parallel_epoch, th.test_trace_sequential_and_level_traces_pass])
+
+
+@pytest.mark.parametrize("name", list(PY_TEXT_PLANTS))
+def test_planted_checker_line_fails_a_pin(name, monkeypatch):
+    attr, old, new = PY_TEXT_PLANTS[name]
+    src = textwrap.dedent(inspect.getsource(getattr(history, attr)))
+    assert src.count(old) == 1, "the planted text must name one place"
+    ns = dict(vars(history))
+    exec(compile(src.replace(old, new), f"<planted {name}>", "exec"), ns)
+    monkeypatch.setattr(history, attr, ns[attr])
+    caught = 0
+    for pin in _DELAY_PINS:
         try:
             pin()
         except AssertionError:
