@@ -605,16 +605,30 @@ int pdb_ssp_epoch(const pdb_csr *X, const float *y, const pdb_conflicts *c, cons
     pdb_conflicts *cm = const_cast<pdb_conflicts *>(c);
     pdb_schedule *hm = const_cast<pdb_schedule *>(h);
     const int width = register_width(cm);
-    if (!hm->reads) {
-        rc = alloc((void **)&hm->reads, sizeof(unsigned) * std::max<int64_t>(X->n_cols, 1), s);
-        rc = rc ? rc : alloc((void **)&hm->writes, sizeof(unsigned) * std::max<int64_t>(X->n_cols, 1), s);
-        if (rc != PDB_OK) return rc;
-    }
+    // scratch kept with the schedule, allocated in pairs on first use and
+    // attached only when both allocations succeeded
+    auto alloc_pair = [&](unsigned **a, unsigned **b, int64_t words) {
+        if (*a && *b) return PDB_OK;
+        unsigned *x = nullptr, *z = nullptr;
+        int r = alloc((void **)&x, sizeof(unsigned) * words, s);
+        r = r ? r : alloc((void **)&z, sizeof(unsigned) * words, s);
+        if (r != PDB_OK) {
+            release(x, s);
+            release(z, s);
+            return r;
+        }
+        release(*a, s);
+        release(*b, s);
+        *a = x;
+        *b = z;
+        return PDB_OK;
+    };
+    rc = alloc_pair(&hm->reads, &hm->writes, std::max<int64_t>(X->n_cols, 1));
+    if (rc != PDB_OK) return rc;
     // one bit per CSC slot, two words of slack past the last slot's word
     const int64_t n_words = X->nnz / 32 + 2;
-    if (prefix && !hm->rbits) {
-        rc = alloc((void **)&hm->rbits, sizeof(unsigned) * n_words, s);
-        rc = rc ? rc : alloc((void **)&hm->wbits, sizeof(unsigned) * n_words, s);
+    if (prefix) {
+        rc = alloc_pair(&hm->rbits, &hm->wbits, n_words);
         if (rc != PDB_OK) return rc;
     }
     cudaEventRecord(cm->ev_sgd0, s);
