@@ -9,11 +9,16 @@
 //
 // Layout: the (feature, position) pairs are stable-sorted by feature into
 // csc_pos (one slot per nonzero, feature-major, data order inside a
-// feature) delimited by feat_ptr.  The only position-indexed array written
-// by a scatter is gate: the occurrence rank of each position (the read
-// protocol's iteration number) with bit 31 marking the feature's last
-// occurrence.  prev and next of a position follow from gate, feat_ptr and
-// csc_pos by gathers and are materialized only when a caller asks for them.
+// feature) delimited by feat_ptr.  Each position has one gate word: its
+// occurrence rank (bits 0-28, the read protocol's iteration number), whether
+// the next (bit 29) and the previous (bit 30) occurrence of its feature lie
+// within `near` positions, and whether it is the feature's last occurrence
+// (bit 31).  Up to 2^22 positions k_slots scatters the gate words straight
+// to position order; above, the build keeps them in slot order (gate_sorted)
+// plus the near pairs' words in position order (gate_window, all WINDOW
+// needs), and ensure_gate builds the position-order array on first use.
+// prev and next of a position follow from gate, feat_ptr and csc_pos by
+// gathers and are materialized only when a caller asks for them.
 #include <cuda_runtime.h>
 #include <nvtx3/nvToolsExt.h>
 
