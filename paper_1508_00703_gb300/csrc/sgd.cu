@@ -1,7 +1,9 @@
-// Update engines: pdb_sgd_epoch (level-synchronous or ready-counter
-// dataflow) and pdb_bsp_epoch (the BSP mini-batch comparison).
+// Update engines: pdb_sgd_epoch's level-synchronous and ready-counter
+// dataflow engines and its dispatch to the others (window.cu, blockready.cu,
+// chain.cu, resident.cu); the host side of pdb_ssp_epoch (kernels in
+// ssp.cu); pdb_bsp_epoch (the BSP mini-batch comparison).
 //
-// One warp runs one example (one transaction, Definition 3): the lanes load
+// In the two engines here one warp runs one example (one transaction, Definition 3): the lanes load
 // the example's ids and values with coalesced loads, gather w through L2,
 // form the margin with per-lane fused multiply-adds and a xor-shuffle
 // combine, compute the scalar eta*g, and scatter w_j -= eta*g*x_j.  No
