@@ -3,12 +3,12 @@
 // chain.cu, resident.cu); the host side of pdb_ssp_epoch (kernels in
 // ssp.cu); pdb_bsp_epoch (the BSP mini-batch comparison).
 //
-// In the two engines here one warp runs one example (one transaction, Definition 3): the lanes load
-// the example's ids and values with coalesced loads, gather w through L2,
-// form the margin with per-lane fused multiply-adds and a xor-shuffle
-// combine, compute the scalar eta*g, and scatter w_j -= eta*g*x_j.  No
-// atomics touch w: the schedule guarantees that no other example holds any
-// of these features at the same time.
+// In the two engines here one warp runs one example (one transaction,
+// Definition 3): the lanes load the example's ids and values with coalesced
+// loads, gather w through L2, form the margin with per-lane fused
+// multiply-adds and a xor-shuffle combine, compute the scalar eta*g, and
+// scatter w_j -= eta*g*x_j.  No atomics touch w: the schedule guarantees
+// that no other example holds any of these features at the same time.
 #include <cuda_runtime.h>
 
 #include <algorithm>
