@@ -15,9 +15,14 @@ every read and every write of every position a separate step, and checks
 that each read observes exactly the write of the previous occurrence of its
 feature in data order (the Read Constraint of Section 4.4, which with one
 writer per occurrence gives the sequential result, Theorem 2), and that the
-workers never deadlock.  Occurrence chains come from the oracle.  The model
-uses the exact watermark; the engine's lags behind it (workers publish their
-progress late), which only makes reads wait longer."""
+workers never deadlock.  Occurrence chains come from the oracle.  The
+watermark is either the exact one (the first position of the oldest
+unfinished chunk) or the engine's: every worker publishes the chunk it has
+just taken before reading its first example (all chunks it took earlier are
+finished by then) and an infinite value once the tickets run out; a sweeper
+reads the workers' words one at a time (a snapshot spread over time, each
+read a step of its own), takes the minimum m and publishes the first position
+of chunk m as the watermark, raising it only."""
 import numpy as np
 import pytest
 
@@ -25,7 +30,10 @@ import oracle
 import synthdata
 
 
-def _simulate(p, near, chunk, n_workers, epochs, rng, watermark_wait=True):
+INF = 1 << 62
+
+
+def _simulate(p, near, chunk, n_workers, epochs, rng, watermark_wait=True, watermark="exact", sweep_ahead=0):
     ch = oracle.chains(p)
     prev, nxt, rank = ch["prev"], ch["next"], ch["rank"]
     row_ptr, col = p.row_ptr, p.col
@@ -42,19 +50,35 @@ def _simulate(p, near, chunk, n_workers, epochs, rng, watermark_wait=True):
         next_ticket = 0
         # worker state: [chunk, example index in chunk, phase, positions pending]
         workers = [None] * n_workers
+        prog = [0] * n_workers          # the engine's progress words (reset every epoch)
+        exited = [False] * n_workers
+        wpos = 0                        # the engine's published watermark
+        sweep_i, sweep_m = 0, INF       # the sweeper's position in its snapshot and its running minimum
         steps = 0
         while not chunk_done.all():
             steps += 1
-            assert steps < 100 * (p.nnz + n + 10), "no progress"
+            assert steps < 200 * (p.nnz + n + 10) + 50 * n_workers * (n + 10), "no progress"
             first_open = int(np.argmin(chunk_done)) if not chunk_done.all() else n_chunks
-            watermark = int(row_ptr[min(first_open * chunk, n)])
+            exact = int(row_ptr[min(first_open * chunk, n)])
+            if watermark == "exact":
+                wm_pos = exact
+            else:
+                assert wpos <= exact, "watermark ahead of the finished chunks"
+                wm_pos = wpos
             enabled = []
+            if watermark == "sweeper":
+                enabled.append((None, "sweep", None))
             for wi, st in enumerate(workers):
                 if st is None:
                     if next_ticket < n_chunks:
                         enabled.append((wi, "take", None))
+                    elif watermark == "sweeper" and not exited[wi]:
+                        enabled.append((wi, "exit", None))
                     continue
                 c, ti, phase, pending = st
+                if phase == "publish":
+                    enabled.append((wi, "publish", None))
+                    continue
                 t = c * chunk + ti
                 b, e = int(row_ptr[t]), int(row_ptr[t + 1])
                 for q in pending:
@@ -64,7 +88,7 @@ def _simulate(p, near, chunk, n_workers, epochs, rng, watermark_wait=True):
                             ok = r is not None and r[0] == (int(rank[q]), ep)
                         else:
                             need = min(int(row_ptr[c * chunk]), e - near)
-                            ok = watermark >= need or not watermark_wait
+                            ok = wm_pos >= need or not watermark_wait
                     else:
                         ok = True
                     if ok:
@@ -73,6 +97,23 @@ def _simulate(p, near, chunk, n_workers, epochs, rng, watermark_wait=True):
                     enabled.append((wi, "next", None))
             assert enabled, "deadlock"
             wi, kind, q = enabled[rng.integers(len(enabled))]
+            if kind == "sweep":
+                if sweep_i < n_workers:
+                    sweep_m = min(sweep_m, prog[sweep_i])
+                    sweep_i += 1
+                else:
+                    wm = min(sweep_m + sweep_ahead, n_chunks)
+                    wpos = max(wpos, int(row_ptr[min(n, wm * chunk)]))
+                    sweep_i, sweep_m = 0, INF
+                continue
+            if kind == "exit":
+                prog[wi] = INF
+                exited[wi] = True
+                continue
+            if kind == "publish":
+                prog[wi] = workers[wi][0]
+                workers[wi][2] = "read"
+                continue
             if kind == "take":
                 c = next_ticket
                 next_ticket += 1
@@ -80,7 +121,8 @@ def _simulate(p, near, chunk, n_workers, epochs, rng, watermark_wait=True):
                 if t0 >= n:
                     chunk_done[c] = True
                     continue
-                workers[wi] = [c, 0, "read", list(range(int(row_ptr[t0]), int(row_ptr[t0 + 1])))]
+                first = "publish" if watermark == "sweeper" else "read"
+                workers[wi] = [c, 0, first, list(range(int(row_ptr[t0]), int(row_ptr[t0 + 1])))]
                 continue
             c, ti, phase, pending = workers[wi]
             t = c * chunk + ti
@@ -119,14 +161,15 @@ def _simulate(p, near, chunk, n_workers, epochs, rng, watermark_wait=True):
             assert w_src[j] == (epochs - 1, int(row_of[ch["csc_pos"][last]]))
 
 
+@pytest.mark.parametrize("watermark", ["exact", "sweeper"])
 @pytest.mark.parametrize("seed", range(12))
-def test_window_protocol_reads_follow_data_order(seed):
+def test_window_protocol_reads_follow_data_order(seed, watermark):
     rng = np.random.default_rng(seed)
     p = synthdata.generate("tiny", seed=seed, n_rows=int(rng.integers(30, 90)), n_cols=int(rng.integers(6, 40)),
                            k=int(rng.integers(1, 6)), k_lo=0, ids="zipf" if seed % 2 else "uniform", zipf_s=1.1)
     near = int(rng.choice([1, 2, 5, 20, 10 ** 6]))     # all far .. all near
     _simulate(p, near=near, chunk=int(rng.integers(1, 4)), n_workers=int(rng.integers(1, 7)),
-              epochs=int(rng.integers(1, 3)), rng=rng)
+              epochs=int(rng.integers(1, 3)), rng=rng, watermark=watermark)
 
 
 def test_window_protocol_model_rejects_a_missing_wait():
@@ -138,6 +181,20 @@ def test_window_protocol_model_rejects_a_missing_wait():
     for _ in range(20):
         try:
             _simulate(p, near=1, chunk=1, n_workers=6, epochs=1, rng=rng, watermark_wait=False)
+        except AssertionError:
+            failures += 1
+    assert failures > 0
+
+
+def test_window_protocol_model_rejects_a_sweeper_one_chunk_ahead():
+    # planted in the model: the sweeper publishes the chunk after the minimum;
+    # some interleaving then lets a far read run before its writer finished
+    rng = np.random.default_rng(8)
+    p = synthdata.generate("tiny", seed=4, n_rows=60, n_cols=6, k=3, k_lo=1)
+    failures = 0
+    for _ in range(20):
+        try:
+            _simulate(p, near=1, chunk=1, n_workers=6, epochs=1, rng=rng, watermark="sweeper", sweep_ahead=1)
         except AssertionError:
             failures += 1
     assert failures > 0
