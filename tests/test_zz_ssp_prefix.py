@@ -8,7 +8,9 @@ over the CSC slots.  The protocol itself is model-checked on the CPU
 counting gates: the sequential result bit for bit at delay 0; every step
 applied exactly once and training that converges for delay > 0; the
 asynchronous Read Constraint on an execution trace; and argument checks and
-an out-of-range rank reported as errors.  This file is collected last."""
+an out-of-range rank reported as errors.  The degenerate inputs (no rows,
+only empty rows, one row, one feature, saturated exponentials) run here
+under both gate forms.  This file is collected last."""
 import numpy as np
 import pytest
 
@@ -111,3 +113,14 @@ def test_prefix_gates_report_a_rank_past_the_feature():
     pdb.pdb_ssp_epoch(X, y, c, s, w, p.loss, p.eta, 1, 4, opts=dict(PREFIX, wait_timeout_s=0.5))
     assert pdb.pdb_status(c) == pdb.PDB_EFAULT
     assert torch.arange(10, device="cuda").sum().item() == 45
+
+
+@pytest.mark.parametrize("gates", [1, 2])
+@pytest.mark.parametrize("name", C.EDGES)
+def test_edge_inputs_under_both_gate_forms(name, gates):
+    p, got, coef = ssp._run(name, 0, opts=dict(ssp_gates=gates))
+    assert np.array_equal(got, C.oracle_sgd(name))
+    p, got, coef = ssp._run(name, 3, opts=dict(ssp_gates=gates))
+    assert np.all(np.isfinite(got))
+    gap, allow = ssp._applied_gap(p, coef, got)
+    assert np.all(gap <= allow)
