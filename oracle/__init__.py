@@ -3,8 +3,9 @@
 Only ``tests/``, ``__graft_entry__.smoke()`` and the CPU-baseline leg of
 ``bench.py`` may import this package.  The product library never calls it and
 shares no code with it.  The arithmetic lives in ``pdb_oracle.c`` (plain C,
-single thread, no contraction); this module marshals numpy arrays, and adds
-the pure-Python brute-force levels and the history checker used on tiny cases.
+single thread, no contraction); this module marshals numpy arrays and adds
+the pure-Python brute-force levels used on tiny cases.  ``history.py`` holds
+the checker of execution histories and traces.
 
 Every routine follows one definition of the paper:
   validate      Definitions 1 and 3 (examples are sets of features)
@@ -12,9 +13,21 @@ Every routine follows one definition of the paper:
                 per-feature occurrence chain and rank)
   levels        Theorem 3 (a level is one barrier step over disjoint
                 transactions), longest conflict path
+  expf, dot,    the written numerics of the update (the paper fixes no
+  grad          summation order or exponential): Cody-Waite reduction and a
+                Taylor polynomial, 32 partial sums and a butterfly, the three
+                losses' derivatives
   sgd           Algorithm 1 / Definition 4, one iteration per example
   bsp           Algorithm 2a with B examples between barriers
   sgd_f64       fp64 drift reference (not a parity target)
+  history.*     Definition 4 and the Read and Write Constraints (Section
+                4.4) on histories; the asynchronous Read Constraint
+                (Section 7) on traces
+
+Admissible delay (Section 7) has no routine here: at delay 0 its result is
+``sgd``'s; for delay > 0 many results are correct (parity unpinned), and its
+runs are checked by properties instead (every step applied once, the
+asynchronous Read Constraint on a trace).
 """
 from __future__ import annotations
 
