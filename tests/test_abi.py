@@ -85,3 +85,26 @@ def test_struct_layouts_match_the_header(tmp_path):
         assert got[(name, "size")] == ctypes.sizeof(cls), name
         for field, _ in cls._fields_:
             assert got[(name, field)] == getattr(cls, field).offset, (name, field)
+
+
+def test_constants_match_the_header(tmp_path):
+    # every PDB_* value the header defines (error codes, enum members) as the
+    # C compiler sees it, against the binding's constant of the same name
+    text = open(os.path.join(ROOT, "include", "pdb.h")).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    names = set(re.findall(r"#define\s+(PDB_[A-Z_]+)\s+\(?-?\d+\)?", text))
+    for body in re.findall(r"typedef\s+enum\s*\{(.*?)\}", text, flags=re.S):
+        names |= set(re.findall(r"\b(PDB_[A-Z_]+)\s*=", body))
+    assert {"PDB_OK", "PDB_EDUP", "PDB_SCHED_WINDOW", "PDB_SSP_PREFIX", "PDB_LOSS_HINGE"} <= names
+    lines = ['#include <stdio.h>', '#include "pdb.h"', "int main(void) {"]
+    lines += [f'printf("{n} %lld\\n", (long long)({n}));' for n in sorted(names)]
+    lines += ["return 0;", "}"]
+    src = tmp_path / "consts.c"
+    src.write_text("\n".join(lines) + "\n")
+    exe = tmp_path / "consts"
+    subprocess.run(["gcc", "-std=c11", f"-I{os.path.join(ROOT, 'include')}", str(src), "-o", str(exe)], check=True)
+    out = subprocess.run([str(exe)], check=True, capture_output=True, text=True).stdout.split("\n")
+    got = {ln.split()[0]: int(ln.split()[1]) for ln in out if ln.strip()}
+    assert set(got) == names
+    for n, v in got.items():
+        assert getattr(pdb, n) == v, n
