@@ -266,29 +266,37 @@ int pdb_sgd_epoch(const pdb_csr *X, const float *y, const pdb_conflicts *c, cons
                   pdb_loss loss, float eta, int n_epochs, const pdb_opts *opts, void *stream);
 
 /* SGD with admissible delay (Section 7): like pdb_sgd_epoch under a READY
- * schedule, with the asynchronous Read and Write Constraints counted per
- * feature.  The occurrence of feature j with rank r reads w_j once at least
- * r - delay writes of j are done, and writes once at least r - delay + 1
- * occurrences of j have read; its write applies its step to the current
- * w_j (an atomic fp32 add of -(eta*g)*x_j, then the write is counted), so
- * every example's update is applied exactly once.  w is updated in place.
+ * schedule, with the asynchronous Read and Write Constraints per feature
+ * (iterations counted per feature: the occurrence of j with rank r is
+ * iteration r of j), in the form opts->ssp_gates selects:
+ *   PDB_SSP_COUNT   (default) rank r reads w_j once at least r - delay
+ *                   writes of j are done, and writes once at least
+ *                   r - delay + 1 occurrences of j have read;
+ *   PDB_SSP_PREFIX  rank r reads once every rank <= r - 1 - delay of j has
+ *                   written, and writes once every rank <= r - delay has
+ *                   read (the paper's Write Protocol: a writer waits for
+ *                   the slowest reader).  Keeps a done-bitmap per direction
+ *                   over the CSC slots: nnz / 4 bytes in all, allocated on
+ *                   first use and kept with the schedule.
+ * Either way a write applies its step to the current w_j (an atomic fp32
+ * add of -(eta*g)*x_j), so every example's update is applied exactly once;
+ * w is updated in place.
  *   delay = 0    the sequential result, bitwise equal to pdb_sgd_epoch
- *   delay > 0    a read sees at least r - delay of the writes of its
- *                feature; the result depends on timing and is not
- *                deterministic.  Under PDB_SSP_COUNT the write gate counts
- *                reads, so a slow reader holds no writer back: its read may
- *                also see writes of later occurrences.  Under PDB_SSP_PREFIX
- *                (the paper's Write Protocol: a writer waits for the slowest
- *                reader) a read of rank r sees every write of rank
- *                <= r - 1 - delay and none of rank >= r + delay; it keeps a
- *                done-bitmap per direction (nnz / 4 bytes in all, allocated
- *                on first use with the schedule)
+ *                (both forms)
+ *   delay > 0    the result depends on timing and is not deterministic.  A
+ *                read of rank r sees at least r - delay writes of its
+ *                feature.  Under PDB_SSP_PREFIX it sees every write of rank
+ *                <= r - 1 - delay and none of rank >= r + delay; under
+ *                PDB_SSP_COUNT a slow reader holds no writer back, so its
+ *                read may also see writes of later occurrences
  *   delay >= the longest chain  no waits at all (Hogwild with atomic updates)
  *   coef         optional device array of n_epochs * n_rows floats (NULL for
  *                none): the step eta*g each example applied, epoch-major,
  *                for auditing a delayed run
  * s must be a READY schedule of c (PDB_ESTATE otherwise); delay < 0 or an
- * unknown opts->ssp_gates is PDB_EINVAL.  Every wait is bounded (pdb_opts.wait_timeout_s). */
+ * unknown opts->ssp_gates is PDB_EINVAL; under PDB_SSP_PREFIX a gate word
+ * whose rank lies past its feature's occurrences is PDB_EFAULT (reported
+ * through pdb_status).  Every wait is bounded (pdb_opts.wait_timeout_s). */
 int pdb_ssp_epoch(const pdb_csr *X, const float *y, const pdb_conflicts *c, const pdb_schedule *s, float *w,
                   pdb_loss loss, float eta, int n_epochs, int64_t delay, float *coef, const pdb_opts *opts,
                   void *stream);
