@@ -90,6 +90,8 @@ class pdb_csr(ctypes.Structure):
 
 
 class pdb_opts(ctypes.Structure):
+    """Launch and wait options (zeroed = defaults).  The calls also take a dict of
+    the same fields; a torch tensor given as `trace` passes its device pointer."""
     _fields_ = [("blocks_per_sm", ctypes.c_int32), ("ticket_chunk", ctypes.c_int32),
                 ("wait_timeout_s", ctypes.c_double), ("trace", ctypes.c_void_p), ("ssp_gates", ctypes.c_int32)]
 
@@ -213,6 +215,8 @@ class Schedule:
 
 
 def pdb_build_conflicts(X: Csr, stream=None) -> Conflicts:
+    """Validate X and build its per-feature occurrence chains (Definitions 1-3,
+    Section 5); errors the device finds surface through pdb_status."""
     h = ctypes.c_void_p()
     _check(load().pdb_build_conflicts(ctypes.byref(X.struct), ctypes.byref(h), _stream(stream)),
            "pdb_build_conflicts")
@@ -228,12 +232,16 @@ def pdb_conflicts_arrays(c: Conflicts, stream=None) -> dict:
 
 
 def pdb_schedule_build(c: Conflicts, mode: int, stream=None) -> Schedule:
+    """Schedule for pdb_sgd_epoch: PDB_SCHED_LEVELS (Theorem 3), READY, WINDOW,
+    CHAIN or AUTO (include/pdb.h describes each)."""
     h = ctypes.c_void_p()
     _check(load().pdb_schedule_build(c.handle, int(mode), ctypes.byref(h), _stream(stream)), "pdb_schedule_build")
     return Schedule(h, c, mode)
 
 
 def pdb_schedule_levels(s: Schedule, stream=None) -> dict:
+    """Borrowed device pointers (ints) of a LEVELS schedule's level, order and
+    level_ptr arrays, and its number of levels (waits for the schedule)."""
     ptrs = [ctypes.c_void_p() for _ in range(3)]
     L = ctypes.c_int64()
     _check(load().pdb_schedule_levels(s.handle, *[ctypes.byref(p) for p in ptrs], ctypes.byref(L), _stream(stream)),
@@ -261,12 +269,17 @@ def _opts(opts):
 
 def pdb_sgd_epoch(X: Csr, y, c: Conflicts, s: Schedule, w, loss: int, eta: float, n_epochs: int, opts=None,
                   stream=None):
+    """n_epochs of SGD over X in data order, serially equivalent (Algorithm 1,
+    Theorem 2): w (float32, n_cols, on the device) is updated in place."""
     _check(load().pdb_sgd_epoch(ctypes.byref(X.struct), _ptr(y), c.handle, s.handle, _ptr(w), int(loss), float(eta),
                                 int(n_epochs), _opts(opts), _stream(stream)), "pdb_sgd_epoch")
 
 
 def pdb_ssp_epoch(X: Csr, y, c: Conflicts, s: Schedule, w, loss: int, eta: float, n_epochs: int, delay: int,
                   coef=None, opts=None, stream=None):
+    """SGD with admissible delay (Section 7) under a READY schedule; opts may set
+    ssp_gates to PDB_SSP_COUNT (default) or PDB_SSP_PREFIX.  delay = 0 is
+    pdb_sgd_epoch's result bit for bit."""
     _check(load().pdb_ssp_epoch(ctypes.byref(X.struct), _ptr(y), c.handle, s.handle, _ptr(w), int(loss), float(eta),
                                 int(n_epochs), int(delay), _ptr(coef), _opts(opts), _stream(stream)),
            "pdb_ssp_epoch")
@@ -274,6 +287,8 @@ def pdb_ssp_epoch(X: Csr, y, c: Conflicts, s: Schedule, w, loss: int, eta: float
 
 def pdb_bsp_epoch(X: Csr, y, c: Conflicts, w, loss: int, eta: float, batch: int, n_epochs: int, opts=None,
                   stream=None):
+    """The BSP comparison (Algorithm 2a): `batch` examples between barriers,
+    margins at the batch-start weights, ordered per-feature sums."""
     _check(load().pdb_bsp_epoch(ctypes.byref(X.struct), _ptr(y), c.handle, _ptr(w), int(loss), float(eta),
                                 int(batch), int(n_epochs), _opts(opts), _stream(stream)), "pdb_bsp_epoch")
 
@@ -290,25 +305,32 @@ def pdb_sgd_epoch_ready_noalloc(X: Csr, y, gate_ptr: int, w, loss: int, eta: flo
 
 
 def pdb_status(c: Conflicts, stream=None) -> int:
+    """Synchronize the stream and return the first error a kernel recorded in c
+    (PDB_OK when none)."""
     return int(load().pdb_status(c.handle, _stream(stream)))
 
 
 def pdb_get_stats(c: Conflicts, s: Schedule | None = None) -> dict:
+    """Sizes, level counts and CUDA-event timings of the last calls on c (and s)
+    as a dict; synchronizes the device."""
     st = pdb_stats()
     _check(load().pdb_get_stats(c.handle, None if s is None else s.handle, ctypes.byref(st)), "pdb_get_stats")
     return st.as_dict()
 
 
 def pdb_memcpy(dst_ptr: int, src_ptr: int, nbytes: int, stream=None):
+    """Stream-ordered copy between device or host pointers (ints)."""
     _check(load().pdb_memcpy(ctypes.c_void_p(dst_ptr), ctypes.c_void_p(src_ptr), int(nbytes), _stream(stream)),
            "pdb_memcpy")
 
 
 def pdb_eval_expf(x, out, stream=None):
+    """out = the library's device exponential of x (float32 tensors), for tests."""
     _check(load().pdb_eval_expf(_ptr(x), _ptr(out), x.numel(), _stream(stream)), "pdb_eval_expf")
 
 
 def pdb_launch_count() -> int:
+    """Kernels this process has launched through the library so far."""
     return int(load().pdb_launch_count())
 
 
