@@ -23,6 +23,7 @@
 #include <nvtx3/nvToolsExt.h>
 
 #include <algorithm>
+#include <atomic>
 #include <cstdio>
 #include <cstdlib>
 #include <cstring>
@@ -478,13 +479,15 @@ int ensure_gate(pdb_conflicts *c, cudaStream_t s)
                              SCATTER_SB, bits_for(nnz - 1), c->info, s);
     if (rc == PDB_OK) {
         const size_t smem = sizeof(uint32_t) << SCATTER_SB;
-        static bool configured[64] = {};
-        if (c->device >= 0 && c->device < 64 && !configured[c->device]) {
+        // set once per device (any device past the table: every call)
+        static std::atomic<bool> configured[64];
+        const bool known = c->device >= 0 && c->device < 64;
+        if (!known || !configured[c->device].load(std::memory_order_acquire)) {
             if (cudaFuncSetAttribute(k_scatter_block, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) !=
                 cudaSuccess)
                 rc = PDB_ECUDA;
-            else
-                configured[c->device] = true;
+            else if (known)
+                configured[c->device].store(true, std::memory_order_release);
         }
         if (rc == PDB_OK) {
             const int64_t blocks = ((nnz - 1) >> SCATTER_SB) + 1;

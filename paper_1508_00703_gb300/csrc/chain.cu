@@ -35,6 +35,8 @@
 // spin waits.
 #include <cuda_runtime.h>
 
+#include <atomic>
+
 #include "common.cuh"
 
 using namespace pdb;
@@ -340,14 +342,16 @@ int chain_run(const pdb_csr *X, const float *y, const uint32_t *link, float *w, 
     auto kern = max_row <= 32 ? k_sgd_chain<1> : max_row <= 64 ? k_sgd_chain<2>
               : max_row <= 128 ? k_sgd_chain<4> : k_sgd_chain<8>;
     const int variant = max_row <= 32 ? 0 : max_row <= 64 ? 1 : max_row <= 128 ? 2 : 3;
-    static bool configured[64][4] = {};
+    // set once per device and variant (any device past the table: every call)
+    static std::atomic<bool> configured[64][4];
     int dev = 0;
     cudaGetDevice(&dev);
-    if (dev >= 0 && dev < 64 && !configured[dev][variant]) {
+    const bool known = dev >= 0 && dev < 64;
+    if (!known || !configured[dev][variant].load(std::memory_order_acquire)) {
         if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sizeof(ChainSmem)) !=
             cudaSuccess)
             return PDB_ECUDA;
-        configured[dev][variant] = true;
+        if (known) configured[dev][variant].store(true, std::memory_order_release);
     }
     // 16-byte row copies need 16-byte aligned ids, values and link words
     const bool vec = ((uintptr_t)X->col & 15) == 0 && ((uintptr_t)X->val & 15) == 0 && ((uintptr_t)link & 15) == 0;

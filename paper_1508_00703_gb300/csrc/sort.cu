@@ -351,14 +351,16 @@ int radix_passes(const uint32_t *keys_in, const int32_t *vals_in, uint32_t *keys
 {
     constexpr int RADIX = 1 << D;
     const size_t smem = sizeof(uint32_t) * ((size_t)(WARPS + 2) * RADIX + 3 * RS_TILE);
-    static bool configured[64] = {};
+    // set once per device (any device past the table: every call)
+    static std::atomic<bool> configured[64];
     int dev = 0;
     cudaGetDevice(&dev);
-    if (dev >= 0 && dev < 64 && !configured[dev]) {
+    const bool known = dev >= 0 && dev < 64;
+    if (!known || !configured[dev].load(std::memory_order_acquire)) {
         if (cudaFuncSetAttribute(k_rs_scatter<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) !=
             cudaSuccess)
             return PDB_ECUDA;
-        configured[dev] = true;
+        if (known) configured[dev].store(true, std::memory_order_release);
     }
     const int64_t n_tiles = (n + RS_TILE - 1) / RS_TILE;
     const int64_t n_chunks = (n_tiles + RS_CHUNK - 1) / RS_CHUNK;
