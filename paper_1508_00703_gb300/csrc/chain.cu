@@ -61,6 +61,11 @@ static_assert((CH_SLOTS & (CH_SLOTS - 1)) == 0 && (CH_RP & (CH_RP - 1)) == 0, "r
 static_assert(CH_SLOTS > (CH_DS + 2) * CH_G && CH_RP > (CH_L + 2) * CH_G + 1, "rings too short");
 static_assert(CH_D < 256 && CH_MAXK <= 65536, "link word fields");
 static_assert((CH_G & (CH_G - 1)) == 0, "examples per step must be a power of two");
+// a weight is gathered (not pushed) when its last writer r' lies more than
+// CH_D examples back; r' stores it through at step r'/G + 1, the gather for r
+// runs at step r/G - CH_BS, and r/G - r'/G >= (CH_D + 1) / G: the store must
+// land at least one step (one __syncthreads) before the gather
+static_assert((CH_D + 1) / CH_G >= CH_BS + 2, "a gather may not meet its last writer's store in one step");
 
 // ids and link words are copied in 16-byte pieces from the aligned element
 // before the example's first one: element i sits at index off + i, off =
