@@ -63,8 +63,8 @@ def test_prefix_gates_still_train(name, delay):
     assert abs(delayed - exact) <= 0.05 * abs(start - exact) + 1e-6
 
 
-@pytest.mark.parametrize("delay", [0, 3])
-@pytest.mark.parametrize("name", ["tiny", "zipf-shape"])
+@pytest.mark.parametrize("delay", [0, 3, 64, 1024])
+@pytest.mark.parametrize("name", ["tiny", "zipf-shape", "long-rows"])
 def test_prefix_gates_trace_keeps_the_asynchronous_read_constraint(name, delay):
     p = C.problem(name)
     X = pdb.Csr.from_problem(p)
