@@ -39,6 +39,7 @@ int persistent_grid(const void *kernel, const pdb_opts *opts)
 uint64_t timeout_ns(const pdb_opts *opts)
 {
     double s = (opts && opts->wait_timeout_s > 0) ? opts->wait_timeout_s : 2.0;
+    if (s > 1e6) s = 1e6;   // keeps the nanosecond count inside uint64_t
     return (uint64_t)(s * 1e9);
 }
 
