@@ -155,3 +155,14 @@ def test_ready_protocol_model_needs_the_epoch_stamps():
         except AssertionError:
             failures += 1
     assert failures > 0
+
+
+@pytest.mark.parametrize("seed", range(3))
+def test_ready_protocol_past_the_stamp_wrap(seed):
+    # stamps repeat every 7 epochs: 16 epochs with a slow worker (and with
+    # chunks of several examples) must still read only the right epoch's
+    # records
+    rng = np.random.default_rng(400 + seed)
+    p = _problem(seed, rng)
+    _simulate(p, chunk=1, n_workers=5, epochs=16, rng=rng, slow_ticket=0)
+    _simulate(p, chunk=3, n_workers=4, epochs=16, rng=rng, slow_ticket=1)
