@@ -74,3 +74,37 @@ def test_dense_rows_and_linear_labels():
     resid = p.y - X @ coef
     assert 0.09 < np.std(resid) < 0.11
     assert 0.8 < np.std(coef) < 1.2          # w* ~ N(0, 1)
+
+
+def test_value_distributions():
+    # N(0, 1) values (tiny) and U(-1, 1) values (low-conflict): first moments
+    p = synthdata.generate("tiny")
+    assert abs(float(p.val.mean())) < 0.02 and abs(float(p.val.std()) - 1.0) < 0.02
+    q = synthdata.generate("low-conflict", n_rows=20000, n_cols=1_000_000)
+    assert abs(float(q.val.mean())) < 0.01 and abs(float(q.val.var()) - 1.0 / 3.0) < 0.005
+    # sign labels of a planted w* split about evenly
+    assert abs(float((p.y > 0).mean()) - 0.5) < 0.03
+
+
+def test_uniform_ids_are_flat():
+    # 100 distinct uniform ids per example over 10^6 features: per-feature
+    # counts are Poisson-like (variance / mean = 1)
+    q = synthdata.generate("low-conflict", n_rows=20000, n_cols=1_000_000)
+    c = np.bincount(q.col, minlength=q.n_cols).astype(np.float64)
+    assert 0.97 < c.var() / c.mean() < 1.03
+
+
+@pytest.mark.parametrize("name,kw,s", [
+    ("zipf-1m", dict(n_rows=100000), 1.0),
+    ("ctr", dict(n_rows=50000, n_cols=1_000_000), 1.1),
+    ("deep-chain", dict(n_rows=10000), 1.3),
+])
+def test_zipf_exponent(name, kw, s):
+    # rank-frequency slope on log-log axes over ranks 1000..10000, where a
+    # feature is rare enough per example that rejecting repeats inside an
+    # example does not bend the curve
+    p = synthdata.generate(name, **kw)
+    cnt = np.sort(np.bincount(p.col, minlength=p.n_cols))[::-1].astype(np.float64)
+    r = np.arange(1000, 10000)
+    slope = np.polyfit(np.log(r + 1.0), np.log(cnt[r]), 1)[0]
+    assert abs(-slope - s) < 0.05, -slope
