@@ -23,7 +23,7 @@ pdb = pytest.importorskip("paper_1508_00703_gb300")
 
 pytestmark = pytest.mark.gpu
 
-PREFIX = dict(ssp_gates=2)
+PREFIX = dict(ssp_gates=pdb.PDB_SSP_PREFIX)
 
 
 @pytest.fixture(scope="module", autouse=True)
@@ -31,7 +31,6 @@ def _cuda():
     if not torch.cuda.is_available():
         pytest.skip("no CUDA device")
     pdb.load()
-    assert pdb.PDB_SSP_PREFIX == PREFIX["ssp_gates"]
 
 
 @pytest.mark.parametrize("name", ["tiny", "zipf-shape", "deepchain-shape", "lowconflict-shape", "long-rows",
@@ -90,7 +89,7 @@ def test_prefix_gates_argument_checks():
     c = pdb.pdb_build_conflicts(X)
     s = pdb.pdb_schedule_build(c, pdb.PDB_SCHED_READY)
     w = torch.zeros(p.n_cols, dtype=torch.float32, device="cuda")
-    for bad in (-1, 3):
+    for bad in (-1, pdb.PDB_SSP_PREFIX + 1):
         with pytest.raises(pdb.PdbError) as e:
             pdb.pdb_ssp_epoch(X, y, c, s, w, p.loss, p.eta, 1, 0, opts=dict(ssp_gates=bad))
         assert e.value.code == pdb.PDB_EINVAL
@@ -115,7 +114,7 @@ def test_prefix_gates_report_a_rank_past_the_feature():
     assert torch.arange(10, device="cuda").sum().item() == 45
 
 
-@pytest.mark.parametrize("gates", [1, 2])
+@pytest.mark.parametrize("gates", [pdb.PDB_SSP_COUNT, pdb.PDB_SSP_PREFIX])
 @pytest.mark.parametrize("name", C.EDGES)
 def test_edge_inputs_under_both_gate_forms(name, gates):
     p, got, coef = ssp._run(name, 0, opts=dict(ssp_gates=gates))
