@@ -115,9 +115,12 @@ typedef enum { PDB_LOSS_LOGISTIC = 0, PDB_LOSS_SQUARED = 1, PDB_LOSS_HINGE = 2 }
  *           whose previous occurrence lies at least `near` positions back
  *           (a distance fixed by the build, >= 2^22) reads w_j once the
  *           completion watermark -- every example before it finished --
- *           has passed that occurrence; a nearer one waits for feature j's
- *           iteration number as under READY, kept in a separate word that
- *           only near writers release.
+ *           has passed that occurrence; a nearer one takes the weight from
+ *           its previous occurrence through feature j's 64-bit record,
+ *           bits(w_j) | tag << 32, written only by positions whose next
+ *           occurrence is near, the tag being the reader's occurrence rank
+ *           with an epoch stamp (the read protocol of Section 5 on the near
+ *           pairs only).
  *   AUTO    CHAIN when the longest per-feature chain exceeds n_rows / 20 and
  *           CHAIN takes the rows (see above); else WINDOW when at most 1/8
  *           of the positions have a near next occurrence; else READY (waits
@@ -205,25 +208,30 @@ int pdb_build_conflicts(const pdb_csr *X, pdb_conflicts **out, void *stream);
 int pdb_conflicts_arrays(const pdb_conflicts *c, const int32_t **csc_pos, const int64_t **feat_ptr,
                          const int32_t **prev, const int32_t **next, const int32_t **rank, void *stream);
 
-/* Schedule for pdb_sgd_epoch.
- *   LEVELS: level[t] = 1 + max over features j of t with an earlier
- *     occurrence of level[row of that occurrence], 0 if none (longest
- *     conflict path), computed by dataflow (examples in data order, each
+/* Schedule for pdb_sgd_epoch (each mode keeps the Read and Write
+ * Constraints of Section 4.4 per feature, so every mode gives the sequential
+ * result, Theorem 2).
+ *   LEVELS (Theorem 3): level[t] = 1 + max over features j of t with an
+ *     earlier occurrence of level[row of that occurrence], 0 if none
+ *     (longest conflict path), computed by dataflow (examples in data order, each
  *     waiting, bounded, for its predecessors' levels) or, with the
  *     environment variable PDB_LEVELS=kahn, by a Kahn-style frontier sweep
  *     (one grid barrier per level); both give the same levels.  order[N]
  *     lists the examples by level, ascending id inside a level; level_ptr[L+1]
  *     delimits the levels.
- *   READY: one 64-bit record per feature, bits(w_j) | version_j << 32,
- *     filled from w by pdb_sgd_epoch; each position waits for the version
- *     equal to its occurrence rank (the conflicts' gate array).
- *   CHAIN: per position, whether an example among the 16 before it writes
- *     its feature last (its weight is then forwarded on chip) and where the
- *     next occurrence sits if within the 16 examples after; nothing when the
+ *   READY (Section 5, read protocol): one 64-bit record per feature,
+ *     bits(w_j) | version_j << 32, filled from w by pdb_sgd_epoch; each
+ *     position waits for the version equal to its occurrence rank (the
+ *     conflicts' gate array).
+ *   CHAIN (Algorithm 1 in data order on one SM): per position, whether an
+ *     example among the 16 before it writes its feature last (its weight is
+ *     then forwarded on chip) and where the next occurrence sits if within
+ *     the 16 examples after; nothing when the
  *     longest example has more than 256 ids and the weights fit in shared
  *     memory (resident); PDB_ETOOBIG when they do not.
- *   WINDOW: per feature a 32-bit iteration number, per example a finished
- *     flag, and the watermark; the positions' near flags are in the gate.
+ *   WINDOW: per feature a 64-bit hand-off record for near pairs, one
+ *     progress word per worker warp, a ticket and the completion watermark;
+ *     the positions' near flags are in the gate.
  *   AUTO: CHAIN, WINDOW or READY (see pdb_sched_mode).
  * Allocates stream-ordered on `stream`. */
 int pdb_schedule_build(const pdb_conflicts *c, pdb_sched_mode mode, pdb_schedule **out, void *stream);
