@@ -200,8 +200,9 @@ typedef struct pdb_schedule pdb_schedule;   /* opaque, library-owned device arra
  * stream-ordered on `stream`. */
 int pdb_build_conflicts(const pdb_csr *X, pdb_conflicts **out, void *stream);
 
-/* Borrowed device pointers into the handle (valid until it is freed).  Any
- * output pointer may be NULL.  prev/next/rank are derived from the CSC
+/* Borrowed device pointers into the handle (valid until it is freed): the
+ * per-feature occurrence chains of Section 5's read protocol.  Any output
+ * pointer may be NULL.  prev/next/rank are derived from the CSC
  * order (rank = slot - feat_ptr[j], neighbours in the slot order) and are
  * materialized by a kernel enqueued on `stream` the first time one of them
  * is requested; read them after that work has completed. */
@@ -237,14 +238,14 @@ int pdb_conflicts_arrays(const pdb_conflicts *c, const int32_t **csc_pos, const 
 int pdb_schedule_build(const pdb_conflicts *c, pdb_sched_mode mode, pdb_schedule **out, void *stream);
 
 /* LEVELS schedule arrays (borrowed device pointers, any may be NULL) and the
- * level count.  SYNCHRONIZES `stream` to read L from the device.
+ * level count (Theorem 3's levels).  SYNCHRONIZES `stream` to read L from the device.
  * PDB_ESTATE for a READY schedule. */
 int pdb_schedule_levels(const pdb_schedule *s, const int32_t **level, const int32_t **order,
                         const int64_t **level_ptr, int64_t *n_levels, void *stream);
 
 /* READY and WINDOW schedule arrays (borrowed device pointers, any may be
- * NULL): gate[nnz], per position bits 0..28 the version it waits for (its
- * occurrence rank), bit 29 set when the next occurrence of its feature lies
+ * NULL; Section 5's read protocol per feature): gate[nnz], per position bits
+ * 0..28 the version it waits for (its occurrence rank), bit 29 set when the next occurrence of its feature lies
  * within the build's `near` distance, bit 30 when the previous one does,
  * bit 31 on the last occurrence of its feature (under WINDOW with more than
  * 2^22 positions: the WINDOW engine's copy, which holds only the words of
@@ -335,8 +336,9 @@ void pdb_schedule_free(pdb_schedule *s);
 /* Text of an error code. */
 const char *pdb_strerror(int code);
 
-/* Allocation-free variant of pdb_sgd_epoch with a READY schedule (the paper
- * has no counterpart; it exists for callers that must not allocate device
+/* Allocation-free variant of pdb_sgd_epoch with a READY schedule
+ * (Algorithm 1 under Section 5's read protocol; the paper has no counterpart
+ * of the allocation-free form; it exists for callers that must not allocate device
  * memory while they train: work recorded into a CUDA graph capture, where
  * cudaMalloc cannot be captured, or a process that has given all device
  * memory to its own pool).  It allocates nothing: its scratch (one 64-bit
@@ -371,7 +373,11 @@ int pdb_memcpy(void *dst, const void *src, size_t bytes, void *stream);
 int64_t pdb_launch_count(void);
 
 /* out[i] = the library's device exp of x[i] (device arrays of n floats), the
- * same function the logistic gradient uses. */
+ * same function the logistic gradient uses.  The paper fixes no exponential;
+ * this one is Cody-Waite range reduction (Cody and Waite 1980) with a
+ * degree-7 Taylor polynomial, within 2 ulp of exp on [-87, 88.5] and exact
+ * at 0, so the oracle can restate it bit for bit.  n < 0, or a NULL array
+ * with n > 0, is PDB_EINVAL. */
 int pdb_eval_expf(const float *x, float *out, int64_t n, void *stream);
 
 #ifdef __cplusplus
