@@ -108,3 +108,16 @@ def test_constants_match_the_header(tmp_path):
     assert set(got) == names
     for n, v in got.items():
         assert getattr(pdb, n) == v, n
+
+
+def test_every_compute_call_cites_its_passage():
+    # the comment above each compute call's declaration names the passage of
+    # the paper that defines the operation
+    text = open(os.path.join(ROOT, "include", "pdb.h")).read()
+    cite = re.compile(r"Section \d|Definitions? \d|Algorithm \d|Theorem \d")
+    found = {}
+    for m in re.finditer(r"(/\*(?:(?!\*/).)*\*/)\s*int\s+(pdb_\w+)\s*\(", text, flags=re.S):
+        found[m.group(2)] = bool(cite.search(m.group(1)))
+    compute = ["pdb_build_conflicts", "pdb_conflicts_arrays", "pdb_schedule_build", "pdb_schedule_levels",
+               "pdb_schedule_ready", "pdb_sgd_epoch", "pdb_ssp_epoch", "pdb_bsp_epoch", "pdb_sgd_epoch_ready_noalloc"]
+    assert all(found.get(n) for n in compute), {n: found.get(n) for n in compute}
