@@ -157,6 +157,9 @@ int orc_level_order(int64_t n_rows, int64_t n_levels, const int32_t *level, int3
 
 /* ------------------------------------------------------------------ numerics */
 
+/* expf_cw of the rule set above: the exponential of the logistic gradient.
+ * The paper fixes none; this one is written from Cody and Waite's range
+ * reduction and the Taylor series, so both sides can compute it alike. */
 float orc_expf(float x)
 {
     const float log2e = (float)1.4426950408889634074;
@@ -203,7 +206,8 @@ float orc_dot(const float *w, const int32_t *col, const float *val, int64_t k)
     return a[0];
 }
 
-/* derivative of the example's loss term f_t with respect to its margin */
+/* derivative of the example's loss term f_t with respect to its margin (the
+ * scalar of the gradient step of Section 2, per example) */
 float orc_grad(int loss, float m, float y)
 {
     if (loss == ORC_LOGISTIC) return -y / (1.0f + orc_expf(y * m));
