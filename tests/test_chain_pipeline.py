@@ -81,7 +81,7 @@ def _simulate(p, epochs, G, DS, BS, SLOTS, RP, D=None):
     for ep in range(epochs):
         ring = {}                         # rp ring: index -> example whose bound it holds
         slot_of = lambda r: r & (SLOTS - 1)
-        col, link_ok, wp, out, pa = {}, {}, {}, {}, {}
+        col, wp, out, pa = {}, {}, {}, {}
 
         def bounds(it, warp, r):
             if r < 0 or r >= N:
@@ -156,7 +156,8 @@ def _simulate(p, epochs, G, DS, BS, SLOTS, RP, D=None):
             if 0 <= t < steps:
                 local = {}
                 for r in range(t * G, min(N, t * G + G)):
-                    b, k = bounds(it, "C", r)
+                    # the compute warp takes the length from the slot, not the ring
+                    b, k = int(rp[r]), int(rp[r + 1] - rp[r])
                     s = slot_of(r)
                     it.r("C", ("kk", s))
                     it.r("C", ("y", s))
