@@ -58,8 +58,6 @@ def parse_args(argv=None):
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=10.0, help="target length of the CPU oracle sample")
-    ap.add_argument("--probe-random-rmw", action="store_true",
-                    help="print the random read-modify-write rate of a 1e8-float array and exit")
     return ap.parse_args(argv)
 
 
@@ -234,29 +232,6 @@ def recorded_traffic(kernel: str, workload: str):
         with open(os.path.join(ROOT, "paper_1508_00703_gb300", "csrc", f), "rb") as fh:
             h.update(fh.read())
     return float(m_b.group(1)) if h.hexdigest() == m_h.group(1) else None
-
-
-def probe_random_rmw(F: int = 100_000_000, n: int = 400_000_000, reps: int = 3):
-    """Random read-modify-write rate of a float array with library kernels
-    (torch gather + elementwise + scatter), the access pattern of one SGD
-    nonzero without any dependency tracking."""
-    import torch
-    g = torch.Generator(device="cuda")
-    g.manual_seed(1508)
-    idx = torch.randint(0, F, (n,), device="cuda", generator=g)
-    w = torch.zeros(F, device="cuda")
-    out = []
-    for r in range(reps + 1):
-        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        e0.record()
-        w.index_put_((idx,), w[idx] * 0.5 + 1.0)
-        e1.record()
-        torch.cuda.synchronize()
-        if r:
-            out.append(e0.elapsed_time(e1))
-    ms = statistics.median(out)
-    return {"probe": "random read-modify-write of 4-byte words (torch gather+scatter)", "n_cols": F,
-            "updates": n, "ms": ms, "updates_per_s": n / (ms / 1e3)}
 
 
 def workload_config(name, problem, mode):
@@ -510,10 +485,6 @@ def run_reference(args, rank, world):
 def main(argv=None):
     args = parse_args(argv)
     rank, world, local_rank = dist_env()
-    if args.probe_random_rmw:
-        if rank == 0:
-            print(json.dumps(probe_random_rmw()), flush=True)
-        return 0
     if args.impl == "reference":
         if rank != 0:
             return 0

@@ -36,6 +36,11 @@
  *   - Calls that share a handle must be ordered on one stream (the handles
  *     hold device-side counters that a concurrent call would clobber).
  *   - Limits: n_rows, n_cols and nnz below 2^31 (positions and ids are int32).
+ *   - Memory: handles allocate stream-ordered from a memory pool the library
+ *     creates for each device on first use.  That pool keeps freed blocks for
+ *     reuse (its release threshold is raised) until the process exits; the
+ *     device's default pool and every other process-wide CUDA setting are left
+ *     as they are.
  *   - Diagnostics: every call opens an NVTX range named after it (seen by
  *     profilers); with the environment variable PDB_LOG set to anything but
  *     "" or "0" each call (but pdb_sgd_epoch_ready_noalloc) prints one line
@@ -337,14 +342,16 @@ void pdb_schedule_free(pdb_schedule *s);
 const char *pdb_strerror(int code);
 
 /* Allocation-free variant of pdb_sgd_epoch with a READY schedule
- * (Algorithm 1 under Section 5's read protocol; the paper has no counterpart
- * of the allocation-free form; it exists for callers that must not allocate device
- * memory while they train: work recorded into a CUDA graph capture, where
- * cudaMalloc cannot be captured, or a process that has given all device
- * memory to its own pool).  It allocates nothing: its scratch (one 64-bit
- * (weight, version) record per feature, a ticket counter and a status word)
- * is one fixed array inside the library of 2^20 records, about 8 MiB, that
- * every GPU loading the library holds until the process exits.
+ * (Algorithm 1 under Section 5's read protocol).  The paper has no
+ * counterpart of the allocation-free form.  It is for callers that cannot
+ * let a library allocate device memory while they train: a server that has
+ * handed all device memory to its own pool and must not see it grow or
+ * fragment, or a host runtime that accounts for every device allocation
+ * itself.  It calls no cudaMalloc, cudaFree or allocating library routine:
+ * its scratch (one 64-bit (weight, version) record per feature, a ticket
+ * counter and a status word) is one fixed array inside the library of 2^20
+ * records, about 8 MiB, that every GPU loading the library holds until the
+ * process exits.
  *   X, y, w     as for pdb_sgd_epoch; X->n_cols must be <= 2^20, else
  *               PDB_ETOOBIG and nothing runs.
  *   gate[nnz]   per position, the gate word (occurrence rank of its feature
@@ -352,13 +359,15 @@ const char *pdb_strerror(int code);
  *               bits 29-30 ignored here) -- the array that
  *               pdb_schedule_ready returns for a READY schedule of X (device,
  *               caller-owned here).
- * Same arithmetic and result as pdb_sgd_epoch.  The first call on each
- * device looks up the array's device address (cudaGetSymbolAddress); make
- * that first call before any stream capture.  All calls on a device share
- * the array (each clears what must start at zero): calls whose GPU work
- * overlaps race, so order them on one stream.  SYNCHRONIZES `stream` and
- * returns PDB_OK, a kernel-recorded error (PDB_ETIMEOUT, PDB_EFAULT), or a
- * host error. */
+ * Same arithmetic and result as pdb_sgd_epoch.  Set-up: the first call on
+ * each device (and again after that device's context is reset) looks up
+ * the array's device address with cudaGetSymbolAddress; make that first
+ * call before any stream capture.  All calls on a device share the array,
+ * which keeps the last call's contents (each call clears what must start at
+ * zero): calls whose GPU work overlaps race, so order them on one stream.
+ * SYNCHRONIZES `stream` (the status word is copied to the host) and returns
+ * PDB_OK, a kernel-recorded error (PDB_ETIMEOUT, PDB_EFAULT), or a host
+ * error. */
 int pdb_sgd_epoch_ready_noalloc(const pdb_csr *X, const float *y, const uint32_t *gate, float *w, pdb_loss loss,
                                 float eta, int n_epochs, void *stream);
 

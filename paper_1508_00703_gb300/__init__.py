@@ -297,9 +297,9 @@ def pdb_sgd_epoch_ready_noalloc(X: Csr, y, gate_ptr: int, w, loss: int, eta: flo
                                 stream=None) -> int:
     """READY-schedule SGD epochs that allocate no device memory (scratch is a
     fixed array inside the library, up to NOALLOC_MAX_COLS features).  For
-    callers that cannot allocate while training, e.g. inside a CUDA graph
-    capture or under a memory pool that owns the whole device.  Synchronizes
-    and returns the status code (PDB_OK on success)."""
+    callers that cannot let a library allocate while they train, e.g. a
+    server whose own memory pool owns the whole device.  Synchronizes the
+    stream and returns the status code (PDB_OK on success)."""
     return int(load().pdb_sgd_epoch_ready_noalloc(ctypes.byref(X.struct), _ptr(y), ctypes.c_void_p(gate_ptr), _ptr(w),
                                                   int(loss), float(eta), int(n_epochs), _stream(stream)))
 

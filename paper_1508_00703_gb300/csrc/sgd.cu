@@ -9,6 +9,7 @@
 // multiply-adds and a xor-shuffle combine, compute the scalar eta*g, and
 // scatter w_j -= eta*g*x_j.  No atomics touch w: the schedule guarantees
 // that no other example holds any of these features at the same time.
+#include <cuda.h>
 #include <cuda_runtime.h>
 
 #include <algorithm>
@@ -745,17 +746,17 @@ int pdb_eval_expf(const float *x, float *out, int64_t n, void *stream)
 }  // extern "C"
 
 // ---------------------------------------------------------------- allocation-free READY epoch
-// Some callers cannot allocate device memory while they train: code that
-// runs between the two halves of a CUDA graph capture (cudaMalloc is not a
-// capturable operation), a server that has handed all device memory to its
-// own pool and must not grow or fragment it, or an embedding runtime that
-// forbids the library from owning memory.  For them the READY epoch below
-// keeps its per-feature (weight, version) records, its ticket counter and
-// its status word in one fixed array compiled into the library instead of
-// in a schedule handle.  Every GPU that loads libpdb holds this array
-// (NOALLOC_MAX_COLS * 8 bytes + 256 bytes, about 8 MiB) until the process
-// exits.  All calls on a device share it: two calls whose work overlaps on
-// the GPU corrupt each other, so order them on one stream.
+// Some callers cannot let a library allocate device memory while they
+// train: a server that has handed all device memory to its own pool and
+// must not see it grow or fragment, or a host runtime that accounts for
+// every device allocation itself and forbids libraries to make their own.
+// For them the READY epoch below keeps its per-feature (weight, version)
+// records, its ticket counter and its status word in one fixed array
+// compiled into the library instead of in a schedule handle.  Every GPU that
+// loads libpdb holds this array (NOALLOC_MAX_COLS * 8 bytes + 256 bytes,
+// about 8 MiB) until the process exits.  All calls on a device share it:
+// two calls whose work overlaps on the GPU corrupt each other, so order them
+// on one stream.
 constexpr int64_t NOALLOC_MAX_COLS = 1 << 20;
 constexpr int64_t NOALLOC_WORDS = NOALLOC_MAX_COLS + 32;   // records, then ticket and status
 static __device__ __align__(256) unsigned long long g_noalloc_scratch[NOALLOC_WORDS];
@@ -763,24 +764,56 @@ static __device__ __align__(256) unsigned long long g_noalloc_scratch[NOALLOC_WO
 namespace {
 
 std::mutex g_noalloc_lock;
-unsigned long long *g_noalloc_ptr[64];
+struct NoallocSlot {
+    void *ctx;                  // context the address was looked up in
+    unsigned long long *ptr;
+};
+NoallocSlot g_noalloc_slot[64];
 
-// Device address of the scratch array for the current device, looked up
-// once per device (host code only sees a stand-in symbol, not the address).
+// The driver's current context (nullptr when none is current or the driver
+// entry point is unavailable).  A device's module, and with it the scratch
+// array, is loaded once per context: after cudaDeviceReset the array may sit
+// elsewhere, so the cached address is keyed by context as well as device.
+void *current_context()
+{
+    typedef CUresult (*GetCurrent)(CUcontext *);
+    static GetCurrent fn = [] {
+        void *f = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &f, 12000, cudaEnableDefault, &q) != cudaSuccess ||
+            q != cudaDriverEntryPointSuccess) {
+            cudaGetLastError();
+            return (GetCurrent) nullptr;
+        }
+        return (GetCurrent)f;
+    }();
+    CUcontext c = nullptr;
+    if (!fn || fn(&c) != CUDA_SUCCESS) return nullptr;
+    return (void *)c;
+}
+
+// Device address of the scratch array for the current device and context.
+// Host code only sees a stand-in symbol, not the address, so the address is
+// looked up (cudaGetSymbolAddress, with that device current) on the first
+// call in each device context and reused afterwards.
 unsigned long long *noalloc_scratch()
 {
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
     std::lock_guard<std::mutex> guard(g_noalloc_lock);
-    if (!g_noalloc_ptr[dev]) {
+    NoallocSlot &slot = g_noalloc_slot[dev];
+    void *ctx = current_context();
+    if (!slot.ptr || !ctx || ctx != slot.ctx) {
         void *p = nullptr;
         if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess) {
             cudaGetLastError();
+            slot.ptr = nullptr;
             return nullptr;
         }
-        g_noalloc_ptr[dev] = (unsigned long long *)p;
+        slot.ptr = (unsigned long long *)p;
+        slot.ctx = current_context();   // the lookup makes the device's primary context current
     }
-    return g_noalloc_ptr[dev];
+    return slot.ptr;
 }
 
 }  // namespace
@@ -788,7 +821,7 @@ unsigned long long *noalloc_scratch()
 extern "C" int pdb_sgd_epoch_ready_noalloc(const pdb_csr *X, const float *y, const uint32_t *gate, float *w,
                                            pdb_loss loss, float eta, int n_epochs, void *stream)
 {
-    ApiScope scope("pdb_sgd_epoch_ready_noalloc", nullptr, nullptr, nullptr, nullptr, false);  // no sync: may be captured
+    ApiScope scope("pdb_sgd_epoch_ready_noalloc", nullptr, nullptr, nullptr, nullptr, false);  // no handle to log
     if (!X || X->n_rows < 0 || X->n_cols < 0 || X->nnz < 0 || n_epochs < 0) return PDB_EINVAL;
     if (X->n_cols > NOALLOC_MAX_COLS) return PDB_ETOOBIG;
     if (X->n_rows >= (1ll << 31) - 1 || X->nnz >= (1ll << 31) - 1) return PDB_EINVAL;

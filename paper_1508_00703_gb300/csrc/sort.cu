@@ -6,6 +6,7 @@
 
 #include <algorithm>
 #include <atomic>
+#include <mutex>
 
 #include "common.cuh"
 
@@ -43,19 +44,34 @@ uint64_t timeout_ns(const pdb_opts *opts)
     return (uint64_t)(s * 1e9);
 }
 
-// Keep freed stream-ordered allocations in the device's default pool instead
-// of returning them to the driver at every synchronization (done once per
-// device; affects only cudaMallocAsync users of that pool).
-static void keep_pool(int device)
+// The library's device memory comes from a stream-ordered memory pool of
+// its own, one per device, created on first use.  Its release threshold is
+// raised so that freed blocks stay in the pool for the next build or
+// schedule instead of going back to the driver at every synchronization.
+// The device's default pool, which other code in the process may use, is
+// left as it is.
+static std::mutex g_pool_lock;
+static cudaMemPool_t g_pool[64];
+
+static cudaMemPool_t library_pool(int device)
 {
-    static bool done[64] = {};
-    if (device < 0 || device >= 64 || done[device]) return;
-    cudaMemPool_t pool;
-    if (cudaDeviceGetDefaultMemPool(&pool, device) == cudaSuccess) {
+    if (device < 0 || device >= 64) return nullptr;
+    std::lock_guard<std::mutex> guard(g_pool_lock);
+    if (!g_pool[device]) {
+        cudaMemPoolProps props = {};
+        props.allocType = cudaMemAllocationTypePinned;
+        props.location.type = cudaMemLocationTypeDevice;
+        props.location.id = device;
+        cudaMemPool_t pool = nullptr;
+        if (cudaMemPoolCreate(&pool, &props) != cudaSuccess) {
+            cudaGetLastError();
+            return nullptr;
+        }
         uint64_t keep = UINT64_MAX;
         cudaMemPoolSetAttribute(pool, cudaMemPoolAttrReleaseThreshold, &keep);
+        g_pool[device] = pool;
     }
-    done[device] = true;
+    return g_pool[device];
 }
 
 int alloc(void **p, size_t bytes, cudaStream_t s)
@@ -63,10 +79,11 @@ int alloc(void **p, size_t bytes, cudaStream_t s)
     *p = nullptr;
     int dev = 0;
     cudaGetDevice(&dev);
-    keep_pool(dev);
+    cudaMemPool_t pool = library_pool(dev);
+    if (!pool) return PDB_ENOMEM;
     if (bytes == 0) bytes = 256;
     bytes = (bytes + 255) & ~(size_t)255;
-    if (cudaMallocAsync(p, bytes, s) != cudaSuccess) {
+    if (cudaMallocFromPoolAsync(p, bytes, pool, s) != cudaSuccess) {
         cudaGetLastError();
         *p = nullptr;
         return PDB_ENOMEM;
