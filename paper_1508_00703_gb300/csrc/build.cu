@@ -35,44 +35,44 @@ using namespace pdb;
 
 namespace {
 
-enum { INFO_STATUS = 0, INFO_MAX_CHAIN = 1, INFO_MAX_ROW = 2, INFO_UNSORTED = 3, INFO_NEAR = 4, INFO_WORDS = 5 };
+// device info words of a conflicts handle: status, longest chain, longest row,
+// near occurrence pairs, and two descent counts (every position p >= 1 with
+// col[p-1] >= col[p], and those where p starts a row: a row whose ids do not
+// increase strictly is one with more of the first than of the second)
+enum {
+    INFO_STATUS = 0, INFO_MAX_CHAIN = 1, INFO_MAX_ROW = 2, INFO_DESC_ALL = 3, INFO_NEAR = 4, INFO_DESC_ROWS = 5,
+    INFO_WORDS = 6
+};
 
-// row_ptr[0] = 0, row_ptr[N] = nnz, nondecreasing (Definition 1: D is a list of examples)
-__global__ void k_validate_rows(const int64_t *__restrict__ row_ptr, int64_t n_rows, int64_t nnz, int *info)
+// row_ptr[0] = 0, row_ptr[N] = nnz, nondecreasing (Definition 1: D is a list
+// of examples); also the longest row and, for every row that is not empty and
+// does not start the data, whether its first id is <= the id before it (the
+// descents the feature sort counts over all positions, minus these, are the
+// ones inside rows: only rows with one can repeat an id)
+__global__ void k_validate_rows(const int64_t *__restrict__ row_ptr, const int32_t *__restrict__ col,
+                                int64_t n_rows, int64_t nnz, int *info)
 {
+    int longest = 0, desc = 0;
     for (int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; t <= n_rows;
          t += (int64_t)gridDim.x * blockDim.x) {
-        int64_t a = row_ptr[t];
-        bool bad = (t == 0 && a != 0) || (t == n_rows && a != nnz) || (t < n_rows && row_ptr[t + 1] < a) ||
-                   a < 0 || a > nnz;
-        if (bad) set_status(info, PDB_EINVAL);
-    }
-}
-
-// One warp per example: ids in [0, n_cols) (else ERANGE), the longest row,
-// and whether the row's ids are strictly increasing (a row that is cannot
-// hold a repeated id; only unsorted rows need the slot check).
-__global__ void k_rows_scan(const int64_t *__restrict__ row_ptr, const int32_t *__restrict__ col, int64_t n_rows,
-                            int64_t n_cols, int *info)
-{
-    if (read_status(info)) return;
-    const int lane = threadIdx.x & 31;
-    const int64_t gw = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-    const int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
-    bool bad = false, unsorted = false;
-    int longest = 0;
-    for (int64_t t = gw; t < n_rows; t += nw) {
-        const int64_t b = row_ptr[t], e = row_ptr[t + 1];
-        longest = max(longest, (int)(e - b));
-        for (int64_t p = b + lane; p < e; p += 32) {
-            int32_t j = col[p];
-            bad |= j < 0 || (int64_t)j >= n_cols;
-            unsorted |= p > b && col[p - 1] >= j;
+        const int64_t a = row_ptr[t];
+        const int64_t e = t < n_rows ? row_ptr[t + 1] : a;
+        const bool bad = (t == 0 && a != 0) || (t == n_rows && a != nnz) || e < a || a < 0 || a > nnz;
+        if (bad) {
+            set_status(info, PDB_EINVAL);
+        } else if (t < n_rows && e <= nnz) {
+            longest = max(longest, (int)(e - a));
+            if (a > 0 && a < e) desc += col[a - 1] >= col[a] ? 1 : 0;
         }
     }
-    if (__any_sync(FULL, bad) && lane == 0) set_status(info, PDB_ERANGE);
-    if (__any_sync(FULL, unsorted) && lane == 0) atomicExch(info + INFO_UNSORTED, 1);
-    if (lane == 0 && longest > 0) atomicMax(info + INFO_MAX_ROW, longest);
+    for (int off = 16; off >= 1; off >>= 1) {
+        longest = max(longest, __shfl_xor_sync(FULL, longest, off));
+        desc += __shfl_xor_sync(FULL, desc, off);
+    }
+    if ((threadIdx.x & 31) == 0) {
+        if (longest > 0) atomicMax(info + INFO_MAX_ROW, longest);
+        if (desc > 0) atomicAdd(info + INFO_DESC_ROWS, desc);
+    }
 }
 
 // example of each position (built on first use: LEVELS, CHAIN, BSP)
@@ -115,7 +115,7 @@ __global__ void k_slots(const uint32_t *__restrict__ skey, const int32_t *__rest
                         uint32_t *__restrict__ gwin, int *info)
 {
     if (read_status(info)) return;
-    const bool check_dup = *(volatile int *)(info + INFO_UNSORTED) != 0;
+    const bool check_dup = *(volatile int *)(info + INFO_DESC_ALL) > *(volatile int *)(info + INFO_DESC_ROWS);
     int longest = 0, n_near = 0;
     bool dup = false, big = false;
     // four consecutive slots per thread and iteration (16-byte loads and
@@ -675,15 +675,13 @@ int pdb_build_conflicts(const pdb_csr *X, pdb_conflicts **out, void *stream)
     c->status = c->info;
     if (rc == PDB_OK) {
         cudaMemsetAsync(c->info, 0, sizeof(int) * INFO_WORDS, s);
-        k_validate_rows<<<grid_1d(N + 1), 256, 0, s>>>(X->row_ptr, N, nnz, c->info);
+        k_validate_rows<<<grid_1d(N + 1), 256, 0, s>>>(X->row_ptr, X->col, N, nnz, c->info);
         note_launch();
-        if (N > 0) {
-            k_rows_scan<<<grid_1d(N * 32), 256, 0, s>>>(X->row_ptr, X->col, N, F, c->info);
-            note_launch();
-        }
-        // (feature, position) pairs sorted by feature, stable: positions stay in data order
+        // (feature, position) pairs sorted by feature, stable: positions stay in data order.
+        // The sort's first read of the ids also checks that they lie in [0, n_cols)
+        // (PDB_ERANGE) and counts the descents.
         rc = radix_sort((const uint32_t *)X->col, nullptr, skey, c->csc_pos, tkey, tval, nnz,
-                        bits_for(F > 0 ? F - 1 : 0), c->info, s);
+                        bits_for(F > 0 ? F - 1 : 0), c->info, s, (uint32_t)F, c->info + INFO_DESC_ALL);
     }
     if (rc == PDB_OK) rc = segment_bounds(skey, nnz, F, nullptr, c->feat_ptr, c->info, s);
     if (rc == PDB_OK && nnz > 0) {
@@ -793,14 +791,14 @@ int pdb_schedule_build(const pdb_conflicts *c, pdb_sched_mode mode, pdb_schedule
         rc = rc ? rc : alloc((void **)&h->rec, sizeof(unsigned long long) * F, s);
     } else if (mode == PDB_SCHED_WINDOW) {
         // near hand-off records (tag 0 = none: tags carry a nonzero epoch
-        // stamp), one progress word per warp the device can hold resident,
-        // the watermark (progress and watermark reset every epoch)
-        int sms = 0;
-        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, c->device);
-        h->prog_cap = (int64_t)std::max(sms, 1) * 64;
+        // stamp), a done flag per chunk of examples (zeroed once: flags
+        // carry the epoch's tag), the ticket and the watermark (reset every
+        // epoch)
+        h->prog_cap = (std::max<int64_t>(N, 1) + 3) & ~(int64_t)3;   // the sweeper reads four flags at a time
         rc = rc ? rc : alloc((void **)&h->rec, sizeof(unsigned long long) * std::max<int64_t>(F, 1), s);
         if (rc == PDB_OK) cudaMemsetAsync(h->rec, 0, sizeof(unsigned long long) * std::max<int64_t>(F, 1), s);
         rc = rc ? rc : alloc((void **)&h->prog, sizeof(unsigned) * h->prog_cap, s);
+        if (rc == PDB_OK) cudaMemsetAsync(h->prog, 0, sizeof(unsigned) * h->prog_cap, s);
         rc = rc ? rc : alloc((void **)&h->wctl, sizeof(WindowCtl), s);
     } else if (mode == PDB_SCHED_CHAIN) {
         // rows longer than the forwarding engine takes: weights resident in

@@ -43,13 +43,16 @@ int chain_run(const pdb_csr *X, const float *y, const uint32_t *link, float *w, 
               int max_row, int *status, uint64_t *trace, cudaStream_t s);
 void note_launch();                                   // count one kernel launch (pdb_launch_count)
 
-// Stable LSD radix sort of (key, value) pairs, 8-bit digits.  vals_in ==
-// nullptr means value = index.  Sorted pairs land in keys_out/vals_out;
-// keys_tmp/vals_tmp are scratch of n elements each.  Kernels return early
-// when *status != 0.
+// Stable LSD radix sort of (key, value) pairs, digits of 8 to 10 bits.
+// vals_in == nullptr means value = index.  Sorted pairs land in
+// keys_out/vals_out; keys_tmp/vals_tmp are scratch of n elements each.
+// Kernels return early when *status != 0.  With range != 0 every key must be
+// below it (else PDB_ERANGE in *status); with descents != nullptr the device
+// counter gains the number of i >= 1 with (int32) key[i-1] >= (int32) key[i]
+// (both counted during the first read of the keys).
 int radix_sort(const uint32_t *keys_in, const int32_t *vals_in, uint32_t *keys_out, int32_t *vals_out,
                uint32_t *keys_tmp, int32_t *vals_tmp, int64_t n, int key_bits, const int *status,
-               cudaStream_t s);
+               cudaStream_t s, uint32_t range = 0, int *descents = nullptr);
 // stable sort on key bits [lo_bit, hi_bit) only (the bits below stay in input order)
 int radix_sort_bits(const uint32_t *keys_in, const int32_t *vals_in, uint32_t *keys_out, int32_t *vals_out,
                     uint32_t *keys_tmp, int32_t *vals_tmp, int64_t n, int lo_bit, int hi_bit, const int *status,
@@ -220,6 +223,8 @@ constexpr uint32_t GATE_LAST = 1u << 31;
 struct WindowCtl {
     unsigned long long ticket;  // next example to hand out
     long long wpos;             // every example starting below this position has finished
+    unsigned arrive;            // blocks started so far (the first one sweeps)
+    unsigned pad;
 };
 
 // admissible delay; rbits == nullptr selects the counting gates, else the
@@ -232,7 +237,7 @@ int ssp_run(const pdb_csr *X, const float *y, const uint32_t *gate, float *w, un
 int ensure_row_of(pdb_conflicts *c, cudaStream_t s);   // builds c->row_of on first use (stream-ordered)
 
 int window_run(const pdb_csr *X, const float *y, const uint32_t *gate, float *w, unsigned long long *rec,
-               unsigned *epoch_count, unsigned *prog, int64_t prog_cap, WindowCtl *ctl, int64_t near, int loss,
+               unsigned *epoch_count, unsigned *done, int64_t done_cap, WindowCtl *ctl, int64_t near, int loss,
                float eta, int n_epochs, int width, const pdb_opts *opts, int *status, uint64_t timeout,
                cudaStream_t s);
 
@@ -284,14 +289,26 @@ struct pdb_schedule {
     unsigned *rbits, *wbits;  // READY under pdb_ssp_epoch with prefix gates: done-bitmaps over the CSC slots
     uint32_t *link;           // CHAIN: per position, receive flag and push target
     bool resident;            // CHAIN: weights resident in shared memory (no link words)
-    unsigned epochs_run;      // WINDOW: epochs run so far (epoch stamp of the record tags)
-    unsigned *prog;           // WINDOW: progress word per worker warp
-    int64_t prog_cap;
+    unsigned epochs_run;      // WINDOW: epochs run so far (epoch stamp of the record tags, done-flag tag)
+    unsigned *prog;           // WINDOW: done flag per chunk of examples (zeroed once)
+    int64_t prog_cap;         // WINDOW: flags allocated (one per example: chunks of one example or more)
     pdb::WindowCtl *wctl;     // WINDOW: ticket and watermark
     pdb::GridBarrier *bar;    // barrier for the level-synchronous engine
     unsigned long long *ticket;
     cudaEvent_t ev0, ev1;
     bool timed;
+};
+
+// BSP batches for the data-parallel split (pdb_bsp_plan_build): every pair of
+// the data sorted by (batch, feature, example), with its feature, example and
+// value, and where each batch's pairs start (device and host copies)
+struct pdb_bsp_plan {
+    const pdb_conflicts *c;
+    int64_t batch, n_batches;
+    int64_t *bptr;            // [n_batches + 1] device
+    int64_t *h_bptr;          // [n_batches + 1] host
+    int32_t *bcol, *brow;
+    float *bval;
 };
 
 namespace pdb {

@@ -114,7 +114,8 @@ int bits_for(int64_t max_key)
 
 // ------------------------------------------------------------------ radix sort
 // Stable LSD radix sort, reduce-then-scan per pass (no inter-tile waiting):
-//   1. k_rs_hist:  digit counts of every 4096-pair tile, written tile-major;
+//   1. k_rs_hist:  digit counts of every 4096-pair tile, written tile-major
+//      (in the conflict build's first pass also the id checks);
 //   2. k_rs_chunk_sum / k_rs_chunk_scan / k_rs_chunk_down: the counts in
 //      digit-major order become the global output offset of each (tile,
 //      digit), computed hierarchically over chunks of 256 tiles;
@@ -128,9 +129,14 @@ constexpr int RS_IPT = 16;
 constexpr int RS_TILE = RS_THREADS * RS_IPT;   // pairs per tile
 constexpr int RS_CHUNK = 256;                  // tiles per scan chunk
 
+// Per-tile digit counts.  In the first pass of the conflict build the same
+// read of the ids also checks them: each must be below `range` (else
+// PDB_ERANGE; range = 0: no check), and `descents` (when not null) gains the
+// number of positions i >= 1 with (int32) key[i-1] >= (int32) key[i].
 template <int D>
 __global__ __launch_bounds__(RS_THREADS) void k_rs_hist(const uint32_t *__restrict__ keys, int64_t n, int shift,
-                                                         uint32_t *__restrict__ hist, const int *status)
+                                                         uint32_t *__restrict__ hist, uint32_t range, int *descents,
+                                                         int *status)
 {
     constexpr int RADIX = 1 << D;
     __shared__ uint32_t h[WARPS][RADIX];
@@ -144,6 +150,18 @@ __global__ __launch_bounds__(RS_THREADS) void k_rs_hist(const uint32_t *__restri
         const int idx = i * RS_THREADS + threadIdx.x;
         k[i] = idx < ntile ? __ldcs(keys + tile0 + idx) : 0u;
     }
+    bool bad = false;
+    int desc = 0;
+    if (range || descents) {
+#pragma unroll
+        for (int i = 0; i < RS_IPT; ++i) {
+            const int idx = i * RS_THREADS + threadIdx.x;
+            if (idx < ntile) {
+                bad |= range && k[i] >= range;
+                if (descents && tile0 + idx > 0) desc += (int32_t)keys[tile0 + idx - 1] >= (int32_t)k[i] ? 1 : 0;
+            }
+        }
+    }
     __syncthreads();
     const int warp = threadIdx.x >> 5;
 #pragma unroll
@@ -155,6 +173,11 @@ __global__ __launch_bounds__(RS_THREADS) void k_rs_hist(const uint32_t *__restri
 #pragma unroll
         for (int w = 0; w < WARPS; ++w) sum += h[w][d];
         hist[(int64_t)blockIdx.x * RADIX + d] = sum;
+    }
+    if (range || descents) {
+        for (int off = 16; off >= 1; off >>= 1) desc += __shfl_xor_sync(FULL, desc, off);
+        if ((threadIdx.x & 31) == 0 && desc) atomicAdd(descents, desc);
+        if (__any_sync(FULL, bad) && (threadIdx.x & 31) == 0) set_status(status, PDB_ERANGE);
     }
 }
 
@@ -365,7 +388,7 @@ __global__ __launch_bounds__(RS_THREADS, 3) void k_rs_scatter(const uint32_t *__
 template <int D>
 int radix_passes(const uint32_t *keys_in, const int32_t *vals_in, uint32_t *keys_out, int32_t *vals_out,
                  uint32_t *keys_tmp, int32_t *vals_tmp, int64_t n, int passes, int shift0, const int *status,
-                 cudaStream_t s)
+                 cudaStream_t s, uint32_t range = 0, int *descents = nullptr)
 {
     constexpr int RADIX = 1 << D;
     const size_t smem = sizeof(uint32_t) * ((size_t)(WARPS + 2) * RADIX + 3 * RS_TILE);
@@ -394,7 +417,8 @@ int radix_passes(const uint32_t *keys_in, const int32_t *vals_in, uint32_t *keys
             uint32_t *ko = to_out ? keys_out : keys_tmp;
             int32_t *vo = to_out ? vals_out : vals_tmp;
             const int shift = shift0 + D * p;
-            k_rs_hist<D><<<(unsigned)n_tiles, RS_THREADS, 0, s>>>(kin, n, shift, hist, status);
+            k_rs_hist<D><<<(unsigned)n_tiles, RS_THREADS, 0, s>>>(kin, n, shift, hist, p == 0 ? range : 0u,
+                                                                  p == 0 ? descents : nullptr, const_cast<int *>(status));
             note_launch();
             k_rs_chunk_sum<<<(unsigned)n_chunks, RADIX, 0, s>>>(hist, n_tiles, RADIX, csum, status);
             note_launch();
@@ -416,16 +440,22 @@ int radix_passes(const uint32_t *keys_in, const int32_t *vals_in, uint32_t *keys
 }
 
 int radix_sort(const uint32_t *keys_in, const int32_t *vals_in, uint32_t *keys_out, int32_t *vals_out,
-               uint32_t *keys_tmp, int32_t *vals_tmp, int64_t n, int key_bits, const int *status, cudaStream_t s)
+               uint32_t *keys_tmp, int32_t *vals_tmp, int64_t n, int key_bits, const int *status, cudaStream_t s,
+               uint32_t range, int *descents)
 {
     if (n <= 0) return PDB_OK;
     // equal digit widths of 8..10 bits: 27-bit ids take 3 passes of 9
     const int kb = std::max(1, std::min(key_bits, 32));
     const int passes = (kb + 9) / 10;
     const int d = std::max(8, (kb + passes - 1) / passes);
-    if (d == 8) return radix_passes<8>(keys_in, vals_in, keys_out, vals_out, keys_tmp, vals_tmp, n, passes, 0, status, s);
-    if (d == 9) return radix_passes<9>(keys_in, vals_in, keys_out, vals_out, keys_tmp, vals_tmp, n, passes, 0, status, s);
-    return radix_passes<10>(keys_in, vals_in, keys_out, vals_out, keys_tmp, vals_tmp, n, passes, 0, status, s);
+    if (d == 8)
+        return radix_passes<8>(keys_in, vals_in, keys_out, vals_out, keys_tmp, vals_tmp, n, passes, 0, status, s,
+                               range, descents);
+    if (d == 9)
+        return radix_passes<9>(keys_in, vals_in, keys_out, vals_out, keys_tmp, vals_tmp, n, passes, 0, status, s,
+                               range, descents);
+    return radix_passes<10>(keys_in, vals_in, keys_out, vals_out, keys_tmp, vals_tmp, n, passes, 0, status, s,
+                            range, descents);
 }
 
 int radix_sort_bits(const uint32_t *keys_in, const int32_t *vals_in, uint32_t *keys_out, int32_t *vals_out,

@@ -17,12 +17,19 @@ feature in data order (the Read Constraint of Section 4.4, which with one
 writer per occurrence gives the sequential result, Theorem 2), and that the
 workers never deadlock.  Occurrence chains come from the oracle.  The
 watermark is either the exact one (the first position of the oldest
-unfinished chunk) or the engine's: every worker publishes the chunk it has
-just taken before reading its first example (all chunks it took earlier are
-finished by then) and an infinite value once the tickets run out; a sweeper
-reads the workers' words one at a time (a snapshot spread over time, each
-read a step of its own), takes the minimum m and publishes the first position
-of chunk m as the watermark, raising it only."""
+unfinished chunk) or the engine's: a worker that has finished chunk c sets
+done[c] when it has taken its next chunk, before that chunk's first read
+(or when the tickets run out); a sweeper reads the flags one at a time from
+its current chunk (each read a step of its own), and when it meets an unset
+flag (or has read a span of them) it publishes the first position of the
+first chunk it has not seen set, raising the watermark only.
+
+Some workers may start late: they take no step until a started worker has
+exited, as thread blocks the device has not made resident start only when a
+running block finishes.  The engine's watermark must not wait for them.  The
+rule the engine used before, a progress word per worker that starts at 0
+and that the sweeper takes the minimum of, is kept as a planted variant: a
+late worker's word pins the watermark and the model reports no progress."""
 import numpy as np
 import pytest
 
@@ -33,7 +40,11 @@ import synthdata
 INF = 1 << 62
 
 
-def _simulate(p, near, chunk, n_workers, epochs, rng, watermark_wait=True, watermark="exact", sweep_ahead=0):
+SPAN = 3     # flags the model's sweeper reads before it publishes
+
+
+def _simulate(p, near, chunk, n_workers, epochs, rng, watermark_wait=True, watermark="exact", sweep_ahead=0,
+              n_late=0):
     ch = oracle.chains(p)
     prev, nxt, rank = ch["prev"], ch["next"], ch["rank"]
     row_ptr, col = p.row_ptr, p.col
@@ -45,15 +56,19 @@ def _simulate(p, near, chunk, n_workers, epochs, rng, watermark_wait=True, water
     n_chunks = (n + chunk - 1) // chunk
     w_src = {}            # feature -> (epoch, example) whose write sits in the array
     rec = {}              # feature -> (tag, epoch, example) of the last record write
+    swept = watermark in ("flags", "words")
     for ep in range(epochs):
         chunk_done = np.zeros(n_chunks, bool)
+        flag = np.zeros(n_chunks, bool)  # the engine's done flags (a fresh tag every epoch)
         next_ticket = 0
         # worker state: [chunk, example index in chunk, phase, positions pending]
         workers = [None] * n_workers
-        prog = [0] * n_workers          # the engine's progress words (reset every epoch)
+        owed = [None] * n_workers        # chunk a worker has finished and not flagged yet
+        prog = [0] * n_workers           # the previous engine's progress words
         exited = [False] * n_workers
-        wpos = 0                        # the engine's published watermark
-        sweep_i, sweep_m = 0, INF       # the sweeper's position in its snapshot and its running minimum
+        started = [wi < n_workers - n_late for wi in range(n_workers)]
+        wpos = 0                         # the engine's published watermark
+        sweep_c, sweep_i, sweep_m = 0, 0, INF
         steps = 0
         while not chunk_done.all():
             steps += 1
@@ -66,13 +81,19 @@ def _simulate(p, near, chunk, n_workers, epochs, rng, watermark_wait=True, water
                 assert wpos <= exact, "watermark ahead of the finished chunks"
                 wm_pos = wpos
             enabled = []
-            if watermark == "sweeper":
+            if swept:
                 enabled.append((None, "sweep", None))
             for wi, st in enumerate(workers):
+                if not started[wi]:
+                    if any(exited[v] for v in range(n_workers) if v != wi):
+                        enabled.append((wi, "start", None))
+                    continue
                 if st is None:
                     if next_ticket < n_chunks:
                         enabled.append((wi, "take", None))
-                    elif watermark == "sweeper" and not exited[wi]:
+                    elif swept and not exited[wi]:
+                        enabled.append((wi, "exit", None))
+                    elif not exited[wi]:
                         enabled.append((wi, "exit", None))
                     continue
                 c, ti, phase, pending = st
@@ -98,30 +119,46 @@ def _simulate(p, near, chunk, n_workers, epochs, rng, watermark_wait=True, water
             assert enabled, "deadlock"
             wi, kind, q = enabled[rng.integers(len(enabled))]
             if kind == "sweep":
-                if sweep_i < n_workers:
-                    sweep_m = min(sweep_m, prog[sweep_i])
+                if watermark == "words":
+                    if sweep_i < n_workers:
+                        sweep_m = min(sweep_m, prog[sweep_i])
+                        sweep_i += 1
+                    else:
+                        wm = min(sweep_m + sweep_ahead, n_chunks)
+                        wpos = max(wpos, int(row_ptr[min(n, wm * chunk)]))
+                        sweep_i, sweep_m = 0, INF
+                    continue
+                c = sweep_c + sweep_i
+                if c < n_chunks and flag[c] and sweep_i < SPAN:
                     sweep_i += 1
                 else:
-                    wm = min(sweep_m + sweep_ahead, n_chunks)
-                    wpos = max(wpos, int(row_ptr[min(n, wm * chunk)]))
-                    sweep_i, sweep_m = 0, INF
+                    sweep_c = min(sweep_c + sweep_i + sweep_ahead, n_chunks)
+                    wpos = max(wpos, int(row_ptr[min(n, sweep_c * chunk)]))
+                    sweep_i = 0
+                continue
+            if kind == "start":
+                started[wi] = True
                 continue
             if kind == "exit":
                 prog[wi] = INF
+                if owed[wi] is not None:
+                    flag[owed[wi]] = True
+                    owed[wi] = None
                 exited[wi] = True
                 continue
             if kind == "publish":
-                prog[wi] = workers[wi][0]
+                if watermark == "words":
+                    prog[wi] = workers[wi][0]
+                elif owed[wi] is not None:
+                    flag[owed[wi]] = True
+                    owed[wi] = None
                 workers[wi][2] = "read"
                 continue
             if kind == "take":
                 c = next_ticket
                 next_ticket += 1
                 t0 = c * chunk
-                if t0 >= n:
-                    chunk_done[c] = True
-                    continue
-                first = "publish" if watermark == "sweeper" else "read"
+                first = "publish" if swept else "read"
                 workers[wi] = [c, 0, first, list(range(int(row_ptr[t0]), int(row_ptr[t0 + 1])))]
                 continue
             c, ti, phase, pending = workers[wi]
@@ -152,6 +189,7 @@ def _simulate(p, near, chunk, n_workers, epochs, rng, watermark_wait=True, water
                     workers[wi] = [c, ti, "read", list(range(int(row_ptr[t]), int(row_ptr[t + 1])))]
                 else:
                     chunk_done[c] = True
+                    owed[wi] = c
                     workers[wi] = None
     # after the last epoch every feature's array entry holds its last writer
     for j in range(p.n_cols):
@@ -161,15 +199,45 @@ def _simulate(p, near, chunk, n_workers, epochs, rng, watermark_wait=True, water
             assert w_src[j] == (epochs - 1, int(row_of[ch["csc_pos"][last]]))
 
 
-@pytest.mark.parametrize("watermark", ["exact", "sweeper"])
+@pytest.mark.parametrize("watermark", ["exact", "flags"])
 @pytest.mark.parametrize("seed", range(12))
 def test_window_protocol_reads_follow_data_order(seed, watermark):
     rng = np.random.default_rng(seed)
     p = synthdata.generate("tiny", seed=seed, n_rows=int(rng.integers(30, 90)), n_cols=int(rng.integers(6, 40)),
                            k=int(rng.integers(1, 6)), k_lo=0, ids="zipf" if seed % 2 else "uniform", zipf_s=1.1)
     near = int(rng.choice([1, 2, 5, 20, 10 ** 6]))     # all far .. all near
-    _simulate(p, near=near, chunk=int(rng.integers(1, 4)), n_workers=int(rng.integers(1, 7)),
-              epochs=int(rng.integers(1, 3)), rng=rng, watermark=watermark)
+    n_workers = int(rng.integers(1, 7))
+    _simulate(p, near=near, chunk=int(rng.integers(1, 4)), n_workers=n_workers,
+              epochs=int(rng.integers(1, 3)), rng=rng, watermark=watermark,
+              n_late=int(rng.integers(0, n_workers)) if watermark == "flags" else 0)
+
+
+@pytest.mark.parametrize("seed", range(6))
+def test_window_protocol_with_most_workers_starting_late(seed):
+    # all far (every read with a predecessor waits on the watermark), one or
+    # two workers running, the rest only after one of them has exited
+    rng = np.random.default_rng(100 + seed)
+    p = synthdata.generate("tiny", seed=seed, n_rows=50, n_cols=12, k=3, k_lo=1)
+    n_workers = 6
+    _simulate(p, near=1, chunk=int(rng.integers(1, 3)), n_workers=n_workers, epochs=2, rng=rng,
+              watermark="flags", n_late=n_workers - 1 - seed % 2)
+
+
+def test_window_protocol_model_rejects_progress_words_with_late_workers():
+    # planted: the previous rule (per-worker progress words starting at 0,
+    # minimum over all workers) with workers that start late pins the
+    # watermark at chunk 0, and the running workers' far reads never pass
+    rng = np.random.default_rng(9)
+    p = synthdata.generate("tiny", seed=5, n_rows=40, n_cols=8, k=3, k_lo=1)
+    with pytest.raises(AssertionError):
+        _simulate(p, near=1, chunk=1, n_workers=4, epochs=1, rng=rng, watermark="words", n_late=2)
+
+
+def test_window_protocol_words_pass_when_every_worker_is_resident():
+    # the same planted rule is sound when every worker runs from the start
+    rng = np.random.default_rng(10)
+    p = synthdata.generate("tiny", seed=5, n_rows=40, n_cols=8, k=3, k_lo=1)
+    _simulate(p, near=1, chunk=1, n_workers=4, epochs=1, rng=rng, watermark="words", n_late=0)
 
 
 def test_window_protocol_model_rejects_a_missing_wait():
@@ -187,14 +255,15 @@ def test_window_protocol_model_rejects_a_missing_wait():
 
 
 def test_window_protocol_model_rejects_a_sweeper_one_chunk_ahead():
-    # planted in the model: the sweeper publishes the chunk after the minimum;
-    # some interleaving then lets a far read run before its writer finished
+    # planted in the model: the sweeper publishes one chunk past the first
+    # unset flag; some interleaving then lets a far read run before its
+    # writer finished
     rng = np.random.default_rng(8)
     p = synthdata.generate("tiny", seed=4, n_rows=60, n_cols=6, k=3, k_lo=1)
     failures = 0
     for _ in range(20):
         try:
-            _simulate(p, near=1, chunk=1, n_workers=6, epochs=1, rng=rng, watermark="sweeper", sweep_ahead=1)
+            _simulate(p, near=1, chunk=1, n_workers=6, epochs=1, rng=rng, watermark="flags", sweep_ahead=1)
         except AssertionError:
             failures += 1
     assert failures > 0
