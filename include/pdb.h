@@ -175,6 +175,7 @@ typedef struct {
 
 typedef struct pdb_conflicts pdb_conflicts; /* opaque, library-owned device arrays */
 typedef struct pdb_schedule pdb_schedule;   /* opaque, library-owned device arrays */
+typedef struct pdb_bsp_plan pdb_bsp_plan;   /* opaque, library-owned device arrays */
 
 /* ---------------------------------------------------------------- calls */
 
@@ -324,6 +325,38 @@ int pdb_ssp_epoch(const pdb_csr *X, const float *y, const pdb_conflicts *c, cons
  * sizing it waits (host) for the conflict build of c to finish. */
 int pdb_bsp_epoch(const pdb_csr *X, const float *y, const pdb_conflicts *c, float *w, pdb_loss loss, float eta,
                   int64_t batch, int n_epochs, const pdb_opts *opts, void *stream);
+
+/* Algorithm 2a split over data-parallel ranks.  Every rank holds the whole
+ * data and a replica of w.  Per batch b (rows [b*B, min((b+1)*B, N))) each
+ * rank computes the coefficients c_i = eta * dloss/dm of its slice of the
+ * batch's rows at the batch-start weights (the reads), the ranks gather the
+ * batch's coefficients in row order (a collective of the caller's choice),
+ * and every rank applies delta_j = sum over the batch's examples, ascending,
+ * of c_i * x_ij, w_j = w_j - delta_j (the writes).  The arithmetic and its
+ * order are pdb_bsp_epoch's, so any split gives that call's result bit for
+ * bit.
+ *
+ * pdb_bsp_plan_build: sorts c's pairs by (batch, feature, example) once for
+ *   batch size `batch` (>= 1; above N it is N) into a plan handle (device
+ *   arrays, library-owned; the plan borrows c, which must outlive it).
+ *   SYNCHRONIZES `stream` (the batch bounds are copied to the host).
+ *   PDB_EINVAL for a NULL argument or batch < 1.
+ * pdb_bsp_plan_batches: number of batches, or -1 for NULL.
+ * pdb_bsp_coef: coef[i - row_begin] = c_i for rows [row_begin, row_end),
+ *   which must lie inside one batch (PDB_EINVAL otherwise); w = the batch's
+ *   start weights (device, n_cols floats); coef device, caller-owned.
+ *   X, y, loss as for pdb_sgd_epoch.  Asynchronous.
+ * pdb_bsp_apply: the write half of batch `batch_index` with coef = all of
+ *   the batch's coefficients in row order (device, rows of the batch
+ *   floats); w updated in place.  Asynchronous.  An inconsistent plan is
+ *   PDB_EFAULT in c's status word.
+ * pdb_bsp_plan_free: waits for the device, frees the plan's arrays. */
+int pdb_bsp_plan_build(const pdb_conflicts *c, int64_t batch, pdb_bsp_plan **out, void *stream);
+int64_t pdb_bsp_plan_batches(const pdb_bsp_plan *p);
+int pdb_bsp_coef(const pdb_bsp_plan *p, const pdb_csr *X, const float *y, const float *w, pdb_loss loss, float eta,
+                 int64_t row_begin, int64_t row_end, float *coef, void *stream);
+int pdb_bsp_apply(const pdb_bsp_plan *p, float *w, int64_t batch_index, const float *coef, void *stream);
+void pdb_bsp_plan_free(pdb_bsp_plan *p);
 
 /* SYNCHRONIZES `stream` and returns the device status of handle c: PDB_OK
  * or the first error a kernel recorded (PDB_EINVAL, PDB_ERANGE, PDB_EDUP,

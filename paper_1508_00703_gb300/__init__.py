@@ -110,7 +110,8 @@ EXPORTS = ["pdb_build_conflicts", "pdb_conflicts_arrays", "pdb_schedule_build", 
            "pdb_schedule_ready",
            "pdb_sgd_epoch", "pdb_bsp_epoch", "pdb_status", "pdb_get_stats", "pdb_conflicts_free",
            "pdb_schedule_free", "pdb_strerror", "pdb_memcpy", "pdb_eval_expf", "pdb_launch_count",
-           "pdb_sgd_epoch_ready_noalloc", "pdb_ssp_epoch"]
+           "pdb_sgd_epoch_ready_noalloc", "pdb_ssp_epoch", "pdb_bsp_plan_build", "pdb_bsp_plan_batches",
+           "pdb_bsp_coef", "pdb_bsp_apply", "pdb_bsp_plan_free"]
 
 
 def load(path: str | None = None):
@@ -142,6 +143,13 @@ def load(path: str | None = None):
         lib.pdb_sgd_epoch_ready_noalloc.argtypes = [ctypes.POINTER(pdb_csr), P, P, P, I32, ctypes.c_float, I32, P]
         lib.pdb_ssp_epoch.argtypes = [ctypes.POINTER(pdb_csr), P, P, P, P, I32, ctypes.c_float, I32, I64, P,
                                       ctypes.POINTER(pdb_opts), P]
+        lib.pdb_bsp_plan_build.argtypes = [P, I64, PP, P]
+        lib.pdb_bsp_plan_batches.argtypes = [P]
+        lib.pdb_bsp_plan_batches.restype = I64
+        lib.pdb_bsp_coef.argtypes = [P, ctypes.POINTER(pdb_csr), P, P, I32, ctypes.c_float, I64, I64, P, P]
+        lib.pdb_bsp_apply.argtypes = [P, P, I64, P, P]
+        lib.pdb_bsp_plan_free.argtypes = [P]
+        lib.pdb_bsp_plan_free.restype = None
         lib.pdb_launch_count.argtypes = []
         lib.pdb_launch_count.restype = I64
         _lib = lib
@@ -291,6 +299,112 @@ def pdb_bsp_epoch(X: Csr, y, c: Conflicts, w, loss: int, eta: float, batch: int,
     margins at the batch-start weights, ordered per-feature sums."""
     _check(load().pdb_bsp_epoch(ctypes.byref(X.struct), _ptr(y), c.handle, _ptr(w), int(loss), float(eta),
                                 int(batch), int(n_epochs), _opts(opts), _stream(stream)), "pdb_bsp_epoch")
+
+
+class BspPlan:
+    """Owns a pdb_bsp_plan handle (keeps its conflicts alive)."""
+
+    def __init__(self, handle, conflicts, batch):
+        self.handle, self.conflicts, self.batch = handle, conflicts, int(batch)
+        self.n_batches = int(load().pdb_bsp_plan_batches(handle))
+
+    def __del__(self):
+        if getattr(self, "handle", None) and _lib is not None:
+            _lib.pdb_bsp_plan_free(self.handle)
+            self.handle = None
+
+
+def pdb_bsp_plan_build(c: Conflicts, batch: int, stream=None) -> BspPlan:
+    """The (batch, feature, example) order of c's pairs for the data-parallel
+    BSP split of Algorithm 2a (synchronizes)."""
+    h = ctypes.c_void_p()
+    _check(load().pdb_bsp_plan_build(c.handle, int(batch), ctypes.byref(h), _stream(stream)), "pdb_bsp_plan_build")
+    return BspPlan(h, c, min(int(batch), max(1, c.n_rows)) if c.n_rows > 0 else int(batch))
+
+
+def pdb_bsp_coef(plan: BspPlan, X: Csr, y, w, loss: int, eta: float, row_begin: int, row_end: int, coef,
+                 stream=None):
+    """coef[i - row_begin] = eta * dloss/dm of rows [row_begin, row_end) at w
+    (the rows lie inside one batch)."""
+    _check(load().pdb_bsp_coef(plan.handle, ctypes.byref(X.struct), _ptr(y), _ptr(w), int(loss), float(eta),
+                               int(row_begin), int(row_end), _ptr(coef), _stream(stream)), "pdb_bsp_coef")
+
+
+def pdb_bsp_apply(plan: BspPlan, w, batch_index: int, coef, stream=None):
+    """The write half of batch `batch_index` from all of its coefficients."""
+    _check(load().pdb_bsp_apply(plan.handle, _ptr(w), int(batch_index), _ptr(coef), _stream(stream)),
+           "pdb_bsp_apply")
+
+
+def rank_rows(r0: int, r1: int, rank: int, world: int) -> tuple[int, int]:
+    """The contiguous share of rows [r0, r1) that rank `rank` of `world` computes
+    (the first (r1 - r0) % world ranks take one row more)."""
+    n = r1 - r0
+    q, extra = divmod(n, world)
+    lo = r0 + rank * q + min(rank, extra)
+    return lo, lo + q + (1 if rank < extra else 0)
+
+
+def bsp_epoch_data_parallel(X: Csr, y, c: Conflicts, w, loss: int, eta: float, batch: int, n_epochs: int,
+                            group=None, plan: BspPlan | None = None, ops=None, stream=None):
+    """Algorithm 2a over the ranks of a torch.distributed group, each holding
+    the whole data and a replica of w: per batch every rank computes the
+    coefficients of its share of the rows (pdb_bsp_coef), the shares are
+    all-gathered in rank order (= row order), and every rank applies the
+    batch (pdb_bsp_apply).  Without an initialized process group it runs on
+    one rank.  The result equals pdb_bsp_epoch's bit for bit.
+
+    `ops` replaces the three library calls (coef, apply, all_gather) with
+    callables of the same meaning; the CPU tests use it to check the
+    partitioning without a GPU."""
+    import torch
+    import torch.distributed as dist
+    world = dist.get_world_size(group) if dist.is_available() and dist.is_initialized() else 1
+    rank = dist.get_rank(group) if world > 1 else 0
+    if ops is None:
+        plan = plan or pdb_bsp_plan_build(c, batch, stream)
+        n_batches, B = plan.n_batches, plan.batch
+
+        def coef_fn(r0, r1, out):
+            pdb_bsp_coef(plan, X, y, w, loss, eta, r0, r1, out, stream)
+
+        def apply_fn(b, coef):
+            pdb_bsp_apply(plan, w, b, coef, stream)
+
+        def gather_fn(parts, mine):
+            if world == 1:
+                return
+            if dist.get_backend(group) == "nccl":
+                dist.all_gather(parts, mine, group=group)
+            else:                              # gloo: host tensors
+                host = [torch.empty(p.numel(), dtype=p.dtype) for p in parts]
+                dist.all_gather(host, mine.cpu(), group=group)
+                for p, h in zip(parts, host):
+                    p.copy_(h)
+        device = w.device
+    else:
+        coef_fn, apply_fn, gather_fn = ops["coef"], ops["apply"], ops["gather"]
+        n_batches, B = ops["n_batches"], ops["batch"]
+        device = ops.get("device", "cpu")
+    n_rows = X.struct.n_rows if hasattr(X, "struct") else ops["n_rows"]
+    coef = torch.empty(max(B, 1), dtype=torch.float32, device=device)
+    for _ in range(n_epochs):
+        for b in range(n_batches):
+            r0, r1 = b * B, min(n_rows, (b + 1) * B)
+            bounds = [rank_rows(r0, r1, r, world) for r in range(world)]
+            # one slice per rank, padded to the longest so that every all_gather part has one size
+            width = max(hi - lo for lo, hi in bounds)
+            if world == 1:
+                coef_fn(r0, r1, coef[: r1 - r0])
+                apply_fn(b, coef[: r1 - r0])
+                continue
+            parts = [torch.zeros(width, dtype=torch.float32, device=device) for _ in range(world)]
+            lo, hi = bounds[rank]
+            coef_fn(lo, hi, parts[rank][: hi - lo])
+            gather_fn(parts, parts[rank])
+            for r, (l2, h2) in enumerate(bounds):
+                coef[l2 - r0: h2 - r0].copy_(parts[r][: h2 - l2])
+            apply_fn(b, coef[: r1 - r0])
 
 
 def pdb_sgd_epoch_ready_noalloc(X: Csr, y, gate_ptr: int, w, loss: int, eta: float, n_epochs: int,

@@ -13,6 +13,7 @@
 #include <cuda_runtime.h>
 
 #include <algorithm>
+#include <new>
 #include <mutex>
 
 #include "common.cuh"
@@ -485,6 +486,81 @@ __global__ void k_bsp_gather(const int32_t *__restrict__ bpos, const int32_t *__
     }
 }
 
+// ---- Algorithm 2a split over data-parallel ranks (pdb_bsp_plan / coef / apply)
+// c_i = eta * dloss/dm(m_i(w), y_i) for the rows [r0, r1), one warp per example,
+// w the weights of the batch start (the read half of the step)
+__global__ void k_bsp_coef(int64_t r0, int64_t r1, const int64_t *__restrict__ row_ptr,
+                           const int32_t *__restrict__ col, const float *__restrict__ val,
+                           const float *__restrict__ y, const float *w, int loss, float eta, float *__restrict__ coef,
+                           const int *status)
+{
+    if (read_status(status)) return;
+    const int lane = threadIdx.x & 31;
+    const int64_t gw = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    for (int64_t t = r0 + gw; t < r1; t += nw) {
+        const float m = margin((int)t, row_ptr, col, val, w);
+        if (lane == 0) coef[t - r0] = __fmul_rn(eta, dev_grad(loss, m, y[t]));
+    }
+}
+
+// The write half of one batch: each feature's terms c_i * x_ij summed in
+// ascending example order from +0, then w_j = w_j - delta_j.  The batch's
+// pairs [s0, s1) are sorted by (feature, example); coef holds the whole
+// batch's coefficients (rows r0.. in order).  A run of at most BSP_LONG
+// terms is summed by one thread; a longer one by a whole warp, 32 terms per
+// load with the same adds in the same order on every lane.
+__global__ void k_bsp_apply(int64_t s0, int64_t s1, int64_t r0, int64_t rows, const int32_t *__restrict__ bcol,
+                            const int32_t *__restrict__ brow, const float *__restrict__ bval,
+                            const float *__restrict__ coef, float *w, int *status)
+{
+    if (read_status(status)) return;
+    const int lane = threadIdx.x & 31;
+    const int64_t gw = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    bool bad = false;
+    for (int64_t base = s0 + gw * 32; base < s1; base += nw * 32) {
+        const int64_t s = base + lane;
+        const int32_t j = s < s1 ? bcol[s] : -1;
+        const bool start = s < s1 && (s == s0 || bcol[s - 1] != j);
+        const bool is_long = start && s + BSP_LONG < s1 && bcol[s + BSP_LONG] == j;
+        if (start && !is_long) {
+            float delta = 0.0f;
+            for (int64_t q = s; q < s1 && bcol[q] == j; ++q) {
+                const int64_t i = brow[q] - r0;
+                bad |= i < 0 || i >= rows;
+                if (i >= 0 && i < rows) delta = __fadd_rn(delta, __fmul_rn(coef[i], bval[q]));
+            }
+            w[j] = __fsub_rn(w[j], delta);
+        }
+        for (unsigned lm = __ballot_sync(FULL, is_long); lm; lm &= lm - 1) {
+            const int src = __ffs(lm) - 1;
+            int64_t q = __shfl_sync(FULL, s, src);
+            const int32_t jr = __shfl_sync(FULL, j, src);
+            float delta = 0.0f;
+            for (;;) {
+                const bool in = q + lane < s1 && bcol[q + lane] == jr;
+                float pv = 0.0f;
+                if (in) {
+                    const int64_t i = brow[q + lane] - r0;
+                    bad |= i < 0 || i >= rows;
+                    if (i >= 0 && i < rows) pv = __fmul_rn(coef[i], bval[q + lane]);
+                }
+                const int n = __popc(__ballot_sync(FULL, in));   // the run is a prefix of the 32
+#pragma unroll
+                for (int u = 0; u < 32; ++u) {
+                    const float v = __shfl_sync(FULL, pv, u);
+                    if (u < n) delta = __fadd_rn(delta, v);
+                }
+                if (n < 32) break;
+                q += 32;
+            }
+            if (lane == 0) w[jr] = __fsub_rn(w[jr], delta);
+        }
+    }
+    if (__any_sync(FULL, bad) && lane == 0) set_status(status, PDB_EFAULT);   // cannot happen with a consistent plan
+}
+
 __global__ void k_eval_expf(const float *__restrict__ x, float *__restrict__ out, int64_t n)
 {
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x)
@@ -733,6 +809,119 @@ int pdb_bsp_epoch(const pdb_csr *X, const float *y, const pdb_conflicts *c, floa
     if (rc == PDB_OK && cudaPeekAtLastError() != cudaSuccess) rc = PDB_ECUDA;
     if (rc != PDB_OK) cudaGetLastError();
     return rc;
+}
+
+int pdb_bsp_plan_build(const pdb_conflicts *c, int64_t batch, pdb_bsp_plan **out, void *stream)
+{
+    ApiScope scope("pdb_bsp_plan_build", c);
+    if (!out) return PDB_EINVAL;
+    *out = nullptr;
+    if (!c || batch < 1) return PDB_EINVAL;
+    cudaStream_t s = (cudaStream_t)stream;
+    pdb_conflicts *cm = const_cast<pdb_conflicts *>(c);
+    const int64_t N = c->n_rows, nnz = c->nnz;
+    if (batch > N && N > 0) batch = N;
+    pdb_bsp_plan *p = new (std::nothrow) pdb_bsp_plan();
+    if (!p) return PDB_ENOMEM;
+    p->c = c;
+    p->batch = batch;
+    p->n_batches = N > 0 ? (N + batch - 1) / batch : 0;
+    uint32_t *key = nullptr, *skey = nullptr, *tkey = nullptr;
+    int32_t *bpos = nullptr, *tval = nullptr;
+    int rc = alloc((void **)&p->bptr, sizeof(int64_t) * (p->n_batches + 1), s);
+    if (rc == PDB_OK && nnz > 0) {
+        rc = alloc((void **)&p->bcol, sizeof(int32_t) * nnz, s);
+        rc = rc ? rc : alloc((void **)&p->brow, sizeof(int32_t) * nnz, s);
+        rc = rc ? rc : alloc((void **)&p->bval, sizeof(float) * nnz, s);
+        rc = rc ? rc : alloc((void **)&key, sizeof(uint32_t) * nnz, s);
+        rc = rc ? rc : alloc((void **)&skey, sizeof(uint32_t) * nnz, s);
+        rc = rc ? rc : alloc((void **)&tkey, sizeof(uint32_t) * nnz, s);
+        rc = rc ? rc : alloc((void **)&bpos, sizeof(int32_t) * nnz, s);
+        rc = rc ? rc : alloc((void **)&tval, sizeof(int32_t) * nnz, s);
+        rc = rc ? rc : ensure_row_of(cm, s);
+        if (rc == PDB_OK) {
+            k_bsp_keys<<<grid_1d(nnz), 256, 0, s>>>(c->csc_pos, c->row_of, nnz, batch, key, cm->status);
+            note_launch();
+            // stable by batch: inside a batch the feature-major CSC order survives
+            rc = radix_sort(key, c->csc_pos, skey, bpos, tkey, tval, nnz, bits_for(p->n_batches - 1), cm->status, s);
+        }
+        if (rc == PDB_OK) {
+            k_bsp_gather<<<grid_1d(nnz), 256, 0, s>>>(bpos, c->col, c->val, c->row_of, nnz, p->bcol, p->brow, p->bval,
+                                                      cm->status);
+            note_launch();
+            rc = segment_bounds(skey, nnz, p->n_batches, nullptr, p->bptr, cm->status, s);
+        }
+    } else if (rc == PDB_OK) {
+        cudaMemsetAsync(p->bptr, 0, sizeof(int64_t) * (p->n_batches + 1), s);
+    }
+    for (void *q : {(void *)key, (void *)skey, (void *)tkey, (void *)bpos, (void *)tval}) release(q, s);
+    if (rc == PDB_OK && cudaPeekAtLastError() != cudaSuccess) rc = PDB_ECUDA;
+    // the host keeps the batches' pair bounds (apply needs them to size its launch)
+    if (rc == PDB_OK) {
+        p->h_bptr = new (std::nothrow) int64_t[p->n_batches + 1];
+        if (!p->h_bptr) rc = PDB_ENOMEM;
+        else if (cudaMemcpyAsync(p->h_bptr, p->bptr, sizeof(int64_t) * (p->n_batches + 1), cudaMemcpyDeviceToHost, s) !=
+                     cudaSuccess ||
+                 cudaStreamSynchronize(s) != cudaSuccess)
+            rc = PDB_ECUDA;
+    }
+    if (rc != PDB_OK) {
+        cudaGetLastError();
+        cudaStreamSynchronize(s);
+        pdb_bsp_plan_free(p);
+        return rc;
+    }
+    *out = p;
+    return PDB_OK;
+}
+
+int64_t pdb_bsp_plan_batches(const pdb_bsp_plan *p) { return p ? p->n_batches : -1; }
+
+int pdb_bsp_coef(const pdb_bsp_plan *p, const pdb_csr *X, const float *y, const float *w, pdb_loss loss, float eta,
+                 int64_t row_begin, int64_t row_end, float *coef, void *stream)
+{
+    ApiScope scope("pdb_bsp_coef", p ? p->c : nullptr, nullptr, nullptr, nullptr, false);
+    if (!p) return PDB_EINVAL;
+    int rc = check_run(X, y, p->c, w, loss, 1);
+    if (rc != PDB_OK) return rc;
+    if (row_begin < 0 || row_end < row_begin || row_end > X->n_rows) return PDB_EINVAL;
+    if (row_end > row_begin && !coef) return PDB_EINVAL;
+    // the rows must lie inside one batch: the margins read that batch's start weights
+    if (row_end > row_begin && row_begin / p->batch != (row_end - 1) / p->batch) return PDB_EINVAL;
+    if (row_end == row_begin) return PDB_OK;
+    cudaStream_t s = (cudaStream_t)stream;
+    k_bsp_coef<<<grid_1d((row_end - row_begin) * 32), 256, 0, s>>>(row_begin, row_end, X->row_ptr, X->col, X->val, y,
+                                                                  w, (int)loss, eta, coef, p->c->status);
+    note_launch();
+    return cudaPeekAtLastError() == cudaSuccess ? PDB_OK : PDB_ECUDA;
+}
+
+int pdb_bsp_apply(const pdb_bsp_plan *p, float *w, int64_t batch_index, const float *coef, void *stream)
+{
+    ApiScope scope("pdb_bsp_apply", p ? p->c : nullptr, nullptr, nullptr, nullptr, false);
+    if (!p || batch_index < 0 || batch_index >= p->n_batches) return PDB_EINVAL;
+    if (p->c->n_cols > 0 && !w) return PDB_EINVAL;
+    const int64_t s0 = p->h_bptr[batch_index], s1 = p->h_bptr[batch_index + 1];
+    if (s1 == s0) return PDB_OK;
+    if (!coef) return PDB_EINVAL;
+    const int64_t r0 = batch_index * p->batch, rows = std::min(p->c->n_rows, r0 + p->batch) - r0;
+    cudaStream_t s = (cudaStream_t)stream;
+    const int64_t blocks = std::max<int64_t>(1, std::min<int64_t>((s1 - s0 + 255) / 256, (int64_t)152 * 16));
+    k_bsp_apply<<<(unsigned)blocks, 256, 0, s>>>(s0, s1, r0, rows, p->bcol, p->brow, p->bval, coef, w,
+                                                 const_cast<pdb_conflicts *>(p->c)->status);
+    note_launch();
+    return cudaPeekAtLastError() == cudaSuccess ? PDB_OK : PDB_ECUDA;
+}
+
+void pdb_bsp_plan_free(pdb_bsp_plan *p)
+{
+    if (!p) return;
+    cudaDeviceSynchronize();
+    cudaGetLastError();
+    for (void *q : {(void *)p->bptr, (void *)p->bcol, (void *)p->brow, (void *)p->bval})
+        if (q) cudaFreeAsync(q, 0);
+    delete[] p->h_bptr;
+    delete p;
 }
 
 int pdb_eval_expf(const float *x, float *out, int64_t n, void *stream)
