@@ -234,6 +234,20 @@ def recorded_traffic(kernel: str, workload: str):
     return float(m_b.group(1)) if h.hexdigest() == m_h.group(1) else None
 
 
+def training_loss(p, X, y, w, torch):
+    """Mean loss of the workload over its examples at weights w (a measurement
+    with library sparse ops, outside every timed region)."""
+    vals = X.val if X.val is not None else torch.ones(p.nnz, dtype=torch.float32, device="cuda")
+    A = torch.sparse_csr_tensor(X.row_ptr, X.col.to(torch.int64), vals, size=(p.n_rows, p.n_cols))
+    m = torch.mv(A.to(torch.float64), w.to(torch.float64))
+    yy = y.to(torch.float64)
+    if p.loss == 0:
+        return float(torch.nn.functional.softplus(-yy * m).mean())
+    if p.loss == 1:
+        return float((0.5 * (m - yy) ** 2).mean())
+    return float(torch.clamp(1.0 - yy * m, min=0.0).mean())
+
+
 def workload_config(name, problem, mode):
     import synthdata
     spec = synthdata.WORKLOADS[name]
@@ -376,6 +390,19 @@ def run_ours(args, rank, world, local_rank):
         result["config"]["ssp_gates"] = args.ssp_gates
         if args.delay > 0:
             result["config"]["note"] = "delay > 0: not serially equivalent, result depends on timing"
+        # what the staleness costs: the training loss after the delayed run beside
+        # the exact (serially equivalent) run's, both from w = 0 over the same epochs
+        c, s = step()
+        pdb.check_status(c, stream)
+        delayed = training_loss(p, X, y, w, torch)
+        w.zero_()
+        c2 = pdb.pdb_build_conflicts(X, stream)
+        s2 = pdb.pdb_schedule_build(c2, pdb.PDB_SCHED_AUTO, stream)
+        pdb.pdb_sgd_epoch(X, y, c2, s2, w, p.loss, p.eta, E, stream=stream)
+        pdb.check_status(c2, stream)
+        result["training_loss"] = {"delayed": delayed, "exact": training_loss(p, X, y, w, torch),
+                                   "loss": {0: "logistic", 1: "squared", 2: "hinge"}[p.loss]}
+        del c, s, c2, s2
     if batch:
         roofline["kernel"] = "k_bsp (whole pdb_bsp_epoch call per epoch: batch sort, gather, cooperative kernel)"
         result["metric"] = METRIC.replace("serially-equivalent sparse SGD", f"BSP mini-batch ({batch}) SGD")
@@ -390,61 +417,89 @@ def run_ours(args, rank, world, local_rank):
 
 
 def run_e2e(args, p, mode, pdb, torch, world):
-    """Same metric through the public API from pinned host buffers: H2D of the
-    inputs and D2H of the trained weights inside the timed region."""
-    stream = torch.cuda.current_stream()
+    """Same metric through the public API from pinned host buffers: every
+    step copies its inputs host-to-device and reads the trained weights back,
+    inside the timed region.  The copies of step i+1 run on a copy stream
+    into a second set of device buffers while step i computes, and step i's
+    weights go back to the host on a third stream while step i+1 computes (a
+    double-buffered input pipeline, as a training loop that streams its data
+    would run it)."""
+    main = torch.cuda.current_stream()
     h_row = torch.from_numpy(p.row_ptr).pin_memory()
     h_col = torch.from_numpy(p.col).pin_memory()
     h_val = None if p.val is None else torch.from_numpy(p.val).pin_memory()
     h_y = torch.from_numpy(p.y).pin_memory()
     h_w0 = torch.zeros(p.n_cols, dtype=torch.float32).pin_memory()
-    h_w = torch.empty(p.n_cols, dtype=torch.float32).pin_memory()
-    d_row = torch.empty_like(h_row, device="cuda")
-    d_col = torch.empty_like(h_col, device="cuda")
-    d_val = None if h_val is None else torch.empty_like(h_val, device="cuda")
-    d_y = torch.empty_like(h_y, device="cuda")
-    d_w = torch.empty_like(h_w0, device="cuda")
-    X = pdb.Csr(d_row, d_col, d_val, p.n_cols)
+    h_w = [torch.empty(p.n_cols, dtype=torch.float32).pin_memory() for _ in range(2)]
     h2d = sum(t.numel() * t.element_size() for t in (h_row, h_col, h_val, h_y, h_w0) if t is not None)
-    d2h = h_w.numel() * h_w.element_size()
+    d2h = h_w[0].numel() * h_w[0].element_size()
 
-    side = torch.cuda.Stream()
+    class Buffers:
+        def __init__(self):
+            self.row = torch.empty_like(h_row, device="cuda")
+            self.col = torch.empty_like(h_col, device="cuda")
+            self.val = None if h_val is None else torch.empty_like(h_val, device="cuda")
+            self.y = torch.empty_like(h_y, device="cuda")
+            self.w = torch.empty_like(h_w0, device="cuda")
+            self.X = pdb.Csr(self.row, self.col, self.val, p.n_cols)
+            self.copied = torch.cuda.Event()
+            self.done = torch.cuda.Event()       # compute on these buffers finished
+            self.read = torch.cuda.Event()       # their weights are back on the host
+            self.done.record(main)
+            self.read.record(main)
 
-    def step():
-        # the conflict build needs only row_ptr and col: the values, labels
-        # and initial weights travel on a second stream while it runs
-        d_row.copy_(h_row, non_blocking=True)
-        d_col.copy_(h_col, non_blocking=True)
-        side.wait_stream(stream)
-        with torch.cuda.stream(side):
-            if d_val is not None:
-                d_val.copy_(h_val, non_blocking=True)
-            d_y.copy_(h_y, non_blocking=True)
-            d_w.copy_(h_w0, non_blocking=True)
-        c = pdb.pdb_build_conflicts(X, stream)
-        s = pdb.pdb_schedule_build(c, mode, stream)
-        stream.wait_stream(side)
-        pdb.pdb_sgd_epoch(X, d_y, c, s, d_w, p.loss, p.eta, p.epochs,
-                          opts=dict(ticket_chunk=args.ticket_chunk, blocks_per_sm=args.blocks_per_sm), stream=stream)
-        h_w.copy_(d_w, non_blocking=True)
-        rc = pdb.pdb_status(c, stream)          # synchronizes: the weights are on the host
-        if rc != 0:
-            raise pdb.PdbError(rc, "e2e step")
-        del c, s
+    bufs = [Buffers(), Buffers()]
+    copy_in, copy_out = torch.cuda.Stream(), torch.cuda.Stream()
+
+    def stage(i):
+        b = bufs[i % 2]
+        copy_in.wait_event(b.done)            # step i-2 no longer reads these inputs
+        copy_in.wait_event(b.read)            # and its weights have left the device
+        with torch.cuda.stream(copy_in):
+            for d, h in ((b.row, h_row), (b.col, h_col), (b.val, h_val), (b.y, h_y), (b.w, h_w0)):
+                if d is not None:
+                    d.copy_(h, non_blocking=True)
+            b.copied.record(copy_in)
+
+    def compute(i):
+        b = bufs[i % 2]
+        main.wait_event(b.copied)
+        c = pdb.pdb_build_conflicts(b.X, main)
+        s = pdb.pdb_schedule_build(c, mode, main)
+        pdb.pdb_sgd_epoch(b.X, b.y, c, s, b.w, p.loss, p.eta, p.epochs,
+                          opts=dict(ticket_chunk=args.ticket_chunk, blocks_per_sm=args.blocks_per_sm), stream=main)
+        b.done.record(main)
+        copy_out.wait_event(b.done)
+        with torch.cuda.stream(copy_out):
+            h_w[i % 2].copy_(b.w, non_blocking=True)
+            b.read.record(copy_out)
+        return c, s
+
+    def run(steps):
+        stage(0)
+        for i in range(steps):
+            if i + 1 < steps:
+                stage(i + 1)
+            c, s = compute(i)
+            rc = pdb.pdb_status(c, main)        # synchronizes main: step i's kernels are done
+            if rc != 0:
+                raise pdb.PdbError(rc, "e2e step")
+            del c, s
+        copy_out.synchronize()                  # the last step's weights are on the host
 
     steps = max(2, min(args.steps, 5))
-    step()
+    run(2)
     barrier(world)
     torch.cuda.synchronize()
     t0 = time.perf_counter()
-    for _ in range(steps):
-        step()
+    run(steps)
     torch.cuda.synchronize()
     dt = (time.perf_counter() - t0) / steps
     dt = reduce_max(dt, world)
     units = reduce_sum(p.epochs * p.nnz, world)
     return {"value": units / dt, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
-            "ms_per_step": dt * 1e3, "steps": steps}
+            "ms_per_step": dt * 1e3, "steps": steps,
+            "pipeline": "step i+1's H2D on a copy stream and step i-1's D2H on another, overlapping step i"}
 
 
 # ---------------------------------------------------------------- reference arm: the CPU oracle
