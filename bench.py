@@ -487,8 +487,22 @@ def run_e2e(args, p, mode, pdb, torch, world):
             del c, s
         copy_out.synchronize()                  # the last step's weights are on the host
 
-    steps = max(2, min(args.steps, 5))
+    steps = max(2, min(args.steps, 10))
     run(2)
+    # the host link's bandwidth on this machine, for reading the number (after the
+    # warm-up steps; best of two copies each way)
+    link = {}
+    for name, dst, src in (("h2d_gbs", bufs[0].col, h_col), ("d2h_gbs", h_w[0], bufs[0].w)):
+        best = 0.0
+        for _ in range(2):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(copy_in)
+            with torch.cuda.stream(copy_in):
+                dst.copy_(src, non_blocking=True)
+            e1.record(copy_in)
+            e1.synchronize()
+            best = max(best, src.numel() * src.element_size() / (e0.elapsed_time(e1) / 1e3) / 1e9)
+        link[name] = round(best, 1)
     barrier(world)
     torch.cuda.synchronize()
     t0 = time.perf_counter()
@@ -498,8 +512,8 @@ def run_e2e(args, p, mode, pdb, torch, world):
     dt = reduce_max(dt, world)
     units = reduce_sum(p.epochs * p.nnz, world)
     return {"value": units / dt, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
-            "ms_per_step": dt * 1e3, "steps": steps,
-            "pipeline": "step i+1's H2D on a copy stream and step i-1's D2H on another, overlapping step i"}
+            "ms_per_step": dt * 1e3, "steps": steps, "host_link": link,
+            "pipeline": "step i+1's H2D on a copy stream and step i's D2H on another, overlapping the next step"}
 
 
 # ---------------------------------------------------------------- reference arm: the CPU oracle

@@ -38,10 +38,11 @@ namespace {
 // device info words of a conflicts handle: status, longest chain, longest row,
 // near occurrence pairs, and two descent counts (every position p >= 1 with
 // col[p-1] >= col[p], and those where p starts a row: a row whose ids do not
-// increase strictly is one with more of the first than of the second)
+// increase strictly is one with more of the first than of the second), each
+// spread over DESC_SPREAD words
 enum {
-    INFO_STATUS = 0, INFO_MAX_CHAIN = 1, INFO_MAX_ROW = 2, INFO_DESC_ALL = 3, INFO_NEAR = 4, INFO_DESC_ROWS = 5,
-    INFO_WORDS = 6
+    INFO_STATUS = 0, INFO_MAX_CHAIN = 1, INFO_MAX_ROW = 2, INFO_NEAR = 4, INFO_DESC_ALL = 8,
+    INFO_DESC_ROWS = INFO_DESC_ALL + DESC_SPREAD, INFO_WORDS = INFO_DESC_ROWS + DESC_SPREAD
 };
 
 // row_ptr[0] = 0, row_ptr[N] = nnz, nondecreasing (Definition 1: D is a list
@@ -65,13 +66,21 @@ __global__ void k_validate_rows(const int64_t *__restrict__ row_ptr, const int32
             if (a > 0 && a < e) desc += col[a - 1] >= col[a] ? 1 : 0;
         }
     }
+    __shared__ int s_longest, s_desc;
+    if (threadIdx.x == 0) s_longest = s_desc = 0;
+    __syncthreads();
     for (int off = 16; off >= 1; off >>= 1) {
         longest = max(longest, __shfl_xor_sync(FULL, longest, off));
         desc += __shfl_xor_sync(FULL, desc, off);
     }
     if ((threadIdx.x & 31) == 0) {
-        if (longest > 0) atomicMax(info + INFO_MAX_ROW, longest);
-        if (desc > 0) atomicAdd(info + INFO_DESC_ROWS, desc);
+        if (longest > 0) atomicMax(&s_longest, longest);
+        if (desc > 0) atomicAdd(&s_desc, desc);
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        if (s_longest > 0) atomicMax(info + INFO_MAX_ROW, s_longest);
+        if (s_desc > 0) atomicAdd(info + INFO_DESC_ROWS + blockIdx.x % DESC_SPREAD, s_desc);
     }
 }
 
@@ -114,8 +123,18 @@ __global__ void k_slots(const uint32_t *__restrict__ skey, const int32_t *__rest
                         int64_t near, uint32_t *__restrict__ gate, uint32_t *__restrict__ gsort,
                         uint32_t *__restrict__ gwin, int *info)
 {
+    __shared__ bool s_check;
+    if (threadIdx.x == 0) {
+        long long all = 0, rows = 0;
+        for (int i = 0; i < DESC_SPREAD; ++i) {
+            all += info[INFO_DESC_ALL + i];
+            rows += info[INFO_DESC_ROWS + i];
+        }
+        s_check = all > rows;
+    }
+    __syncthreads();
     if (read_status(info)) return;
-    const bool check_dup = *(volatile int *)(info + INFO_DESC_ALL) > *(volatile int *)(info + INFO_DESC_ROWS);
+    const bool check_dup = s_check;
     int longest = 0, n_near = 0;
     bool dup = false, big = false;
     // four consecutive slots per thread and iteration (16-byte loads and

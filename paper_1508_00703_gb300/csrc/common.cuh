@@ -43,13 +43,16 @@ int chain_run(const pdb_csr *X, const float *y, const uint32_t *link, float *w, 
               int max_row, int *status, uint64_t *trace, cudaStream_t s);
 void note_launch();                                   // count one kernel launch (pdb_launch_count)
 
+// counters that many blocks add to are spread over this many words (summed by the reader)
+constexpr int DESC_SPREAD = 32;
+
 // Stable LSD radix sort of (key, value) pairs, digits of 8 to 10 bits.
 // vals_in == nullptr means value = index.  Sorted pairs land in
 // keys_out/vals_out; keys_tmp/vals_tmp are scratch of n elements each.
 // Kernels return early when *status != 0.  With range != 0 every key must be
-// below it (else PDB_ERANGE in *status); with descents != nullptr the device
-// counter gains the number of i >= 1 with (int32) key[i-1] >= (int32) key[i]
-// (both counted during the first read of the keys).
+// below it (else PDB_ERANGE in *status); with descents != nullptr the
+// DESC_SPREAD device counters there gain, summed, the number of i >= 1 with
+// (int32) key[i-1] >= (int32) key[i] (both during the first read of the keys).
 int radix_sort(const uint32_t *keys_in, const int32_t *vals_in, uint32_t *keys_out, int32_t *vals_out,
                uint32_t *keys_tmp, int32_t *vals_tmp, int64_t n, int key_bits, const int *status,
                cudaStream_t s, uint32_t range = 0, int *descents = nullptr);
@@ -153,15 +156,21 @@ __device__ __forceinline__ bool grid_sync(GridBarrier *bar, int *status, uint64_
 // applied as two exact power-of-two factors so the one rounding happens in
 // the final product, also for subnormal results.  Inputs are clamped to
 // [-104, 89], where the result has already underflowed to 0 / overflowed.
-__device__ __forceinline__ float dev_expf(float x)
+// rint and the conversion of k to an integer both come from one exact
+// addition of 1.5 * 2^23 (|x log2e| < 2^22: the sum's last mantissa bits are
+// k, rounded to nearest even); a NaN input is returned at the end, so the
+// path has no branch.
+__device__ __forceinline__ float dev_expf(float x0)
 {
-    if (x != x) return x;
-    x = x > 89.0f ? 89.0f : x;
+    float x = x0 > 89.0f ? 89.0f : x0;
     x = x < -104.0f ? -104.0f : x;
     const float log2e = 1.44269502162933349609375f;      // nearest float to log2(e)
     const float ln2_head = 0.693145751953125f;           // 45426 * 2^-16
     const float ln2_tail = 1.428606765330187045e-06f;     // ln2 - head, rounded to float
-    float kf = rintf(__fmul_rn(x, log2e));
+    const float shifter = 12582912.0f;                    // 1.5 * 2^23
+    const float u = __fadd_rn(__fmul_rn(x, log2e), shifter);
+    const float kf = __fsub_rn(u, shifter);
+    const int k = __float_as_int(u) - 0x4B400000;
     float r = __fsub_rn(x, __fmul_rn(kf, ln2_head));
     r = __fsub_rn(r, __fmul_rn(kf, ln2_tail));
     float p = 1.0f / 5040.0f;
@@ -172,12 +181,12 @@ __device__ __forceinline__ float dev_expf(float x)
     p = __fmaf_rn(p, r, 0.5f);
     p = __fmaf_rn(p, r, 1.0f);
     p = __fmaf_rn(p, r, 1.0f);
-    int k = (int)kf;
-    int h = k / 2;
-    int k2 = k - h;
-    float s1 = __int_as_float((h + 127) << 23);
-    float s2 = __int_as_float((k2 + 127) << 23);
-    return __fmul_rn(__fmul_rn(p, s1), s2);
+    const int h = k / 2;
+    const int k2 = k - h;
+    const float s1 = __int_as_float((h + 127) << 23);
+    const float s2 = __int_as_float((k2 + 127) << 23);
+    const float e = __fmul_rn(__fmul_rn(p, s1), s2);
+    return x0 != x0 ? x0 : e;
 }
 
 // execution trace (pdb_opts.trace): lane 0 stamps %globaltimer into

@@ -131,8 +131,9 @@ constexpr int RS_CHUNK = 256;                  // tiles per scan chunk
 
 // Per-tile digit counts.  In the first pass of the conflict build the same
 // read of the ids also checks them: each must be below `range` (else
-// PDB_ERANGE; range = 0: no check), and `descents` (when not null) gains the
-// number of positions i >= 1 with (int32) key[i-1] >= (int32) key[i].
+// PDB_ERANGE; range = 0: no check), and the DESC_SPREAD counters at
+// `descents` (when not null) gain, together, the number of positions i >= 1
+// with (int32) key[i-1] >= (int32) key[i].
 template <int D>
 __global__ __launch_bounds__(RS_THREADS) void k_rs_hist(const uint32_t *__restrict__ keys, int64_t n, int shift,
                                                          uint32_t *__restrict__ hist, uint32_t range, int *descents,
@@ -140,8 +141,10 @@ __global__ __launch_bounds__(RS_THREADS) void k_rs_hist(const uint32_t *__restri
 {
     constexpr int RADIX = 1 << D;
     __shared__ uint32_t h[WARPS][RADIX];
+    __shared__ int s_desc;
     if (read_status(status)) return;
     for (int i = threadIdx.x; i < WARPS * RADIX; i += RS_THREADS) (&h[0][0])[i] = 0;
+    if (threadIdx.x == 0) s_desc = 0;
     const int64_t tile0 = (int64_t)blockIdx.x * RS_TILE;
     const int ntile = (int)min64(RS_TILE, n - tile0);
     uint32_t k[RS_IPT];
@@ -176,8 +179,11 @@ __global__ __launch_bounds__(RS_THREADS) void k_rs_hist(const uint32_t *__restri
     }
     if (range || descents) {
         for (int off = 16; off >= 1; off >>= 1) desc += __shfl_xor_sync(FULL, desc, off);
-        if ((threadIdx.x & 31) == 0 && desc) atomicAdd(descents, desc);
+        if ((threadIdx.x & 31) == 0 && desc) atomicAdd(&s_desc, desc);
         if (__any_sync(FULL, bad) && (threadIdx.x & 31) == 0) set_status(status, PDB_ERANGE);
+        __syncthreads();
+        // one add per block, spread over DESC_SPREAD counters (one address would serialize them)
+        if (threadIdx.x == 0 && s_desc && descents) atomicAdd(descents + (blockIdx.x % DESC_SPREAD), s_desc);
     }
 }
 
