@@ -156,12 +156,17 @@ __global__ __launch_bounds__(RS_THREADS) void k_rs_hist(const uint32_t *__restri
     bool bad = false;
     int desc = 0;
     if (range || descents) {
+        // the key before element idx: the previous lane's, and for lane 0 a load
+        // (it sits in another warp, or in the tile before)
+        const int lane = threadIdx.x & 31;
 #pragma unroll
         for (int i = 0; i < RS_IPT; ++i) {
             const int idx = i * RS_THREADS + threadIdx.x;
+            uint32_t before = __shfl_up_sync(FULL, k[i], 1);
+            if (lane == 0 && tile0 + idx > 0 && idx < ntile) before = keys[tile0 + idx - 1];
             if (idx < ntile) {
                 bad |= range && k[i] >= range;
-                if (descents && tile0 + idx > 0) desc += (int32_t)keys[tile0 + idx - 1] >= (int32_t)k[i] ? 1 : 0;
+                if (descents && tile0 + idx > 0) desc += (int32_t)before >= (int32_t)k[i] ? 1 : 0;
             }
         }
     }
