@@ -54,12 +54,17 @@ constexpr int CH_RP = 64;                   // row_ptr ring (power of two, > (CH
 constexpr int CH_THREADS = 256;
 // link word of a position: bit 31 = its weight will be pushed by an earlier
 // example (skip the gather); bit 30 = push the new weight to the next
-// occurrence, which is element (bits 0..15) of the example (bits 16..23)
-// examples later
-constexpr uint32_t LK_RECV = 1u << 31, LK_PUSH = 1u << 30;
+// occurrence, which is element (bits 0..7) of the example (bits 16..23)
+// examples later; bit 29 = the previous occurrence is in the example just
+// before, as its element (bits 8..15)
+constexpr uint32_t LK_RECV = 1u << 31, LK_PUSH = 1u << 30, LK_LATE = 1u << 29;
 static_assert((CH_SLOTS & (CH_SLOTS - 1)) == 0 && (CH_RP & (CH_RP - 1)) == 0, "ring sizes must be powers of two");
 static_assert(CH_SLOTS > (CH_DS + 2) * CH_G && CH_RP > (CH_L + 2) * CH_G + 1, "rings too short");
-static_assert(CH_D < 256 && CH_MAXK <= 65536, "link word fields");
+static_assert(CH_D < 256 && CH_MAXK <= 256, "link word fields");
+// store address word the compute warp reads per element: the shared-memory
+// address of the new weight (below 2^22), bit 22 = the weight arrives from
+// the example just before, as its element (bits 23..30)
+constexpr uint32_t PA_ADDR = (1u << 22) - 1, PA_LATE = 1u << 22;
 static_assert((CH_G & (CH_G - 1)) == 0, "examples per step must be a power of two");
 // a weight is gathered (not pushed) when its last writer r' lies more than
 // CH_D examples back; r' stores it through at step r'/G + 1, the gather for r
@@ -163,7 +168,7 @@ __device__ __forceinline__ bool row_bounds(const ChainSmem &S, int r, int N, boo
     return true;
 }
 
-template <int R>
+template <int R, int LOSS>
 __global__ __launch_bounds__(CH_THREADS, 1) void k_sgd_chain(int32_t n_rows, const int64_t *__restrict__ row_ptr,
                                                              const int32_t *__restrict__ col,
                                                              const float *__restrict__ val,
@@ -243,8 +248,9 @@ __global__ __launch_bounds__(CH_THREADS, 1) void k_sgd_chain(int32_t n_rows, con
                             const uint32_t lk = S.link[slot][off + i];
                             if (!(lk & LK_RECV)) cp4(&S.wp[slot][i], w + S.col[slot][off + i]);
                             const unsigned tslot = ((unsigned)r + ((lk >> 16) & 0xffu)) & (CH_SLOTS - 1);
-                            S.pa[slot][i] = (lk & LK_PUSH) ? wp_base + 4u * (tslot * CH_MAXK + (lk & 0xffffu))
-                                                           : out_base + 4u * ((unsigned)slot * CH_MAXK + i);
+                            const unsigned addr = (lk & LK_PUSH) ? wp_base + 4u * (tslot * CH_MAXK + (lk & 0xffu))
+                                                                 : out_base + 4u * ((unsigned)slot * CH_MAXK + i);
+                            S.pa[slot][i] = addr | ((lk & LK_LATE) ? PA_LATE | (((lk >> 8) & 0xffu) << 23) : 0u);
                         }
                         if (lane == 0) S.kk[slot] = k;
                     }
@@ -254,13 +260,17 @@ __global__ __launch_bounds__(CH_THREADS, 1) void k_sgd_chain(int32_t n_rows, con
                 cp_commit();
                 cp_wait_b();
             } else if (t >= 0 && t < steps) {
-                // compute the G examples of step t in data order; an example's length,
-                // label, values and store addresses are fetched while the one before
-                // finishes, its weights once that one's pushes are stored
+                // compute the G examples of step t in data order.  The first takes every
+                // weight from its slot.  Each later one fetches its length, label, values,
+                // store words and weights while the example before computes its gradient:
+                // a weight that example writes (its previous occurrence is there) is taken
+                // from it once it exists -- by shuffle from the lane that computed it for
+                // rows of up to 64 ids, else from the slot after the pushes are stored --
+                // and every other weight is final when fetched.
                 const int r0 = t * CH_G, r1 = min(N, r0 + CH_G);
                 const unsigned dump = (unsigned)__cvta_generic_to_shared(&S.dump[lane]);
                 int k;
-                float yr, xv[R];
+                float yr, xv[R], wv[R];
                 unsigned pa[R];
                 auto fetch = [&](int r) {
                     const int slot = r & (CH_SLOTS - 1);
@@ -270,32 +280,53 @@ __global__ __launch_bounds__(CH_THREADS, 1) void k_sgd_chain(int32_t n_rows, con
                     for (int q = 0; q < R; ++q) {
                         xv[q] = S.xa[slot][q * 32 + lane];
                         pa[q] = S.pa[slot][q * 32 + lane];
+                        wv[q] = S.wp[slot][q * 32 + lane];      // past k: unused
                     }
                 };
                 fetch(r0);
                 for (int r = r0; r < r1; ++r) {
-                    const int slot = r & (CH_SLOTS - 1);
-                    float wv[R], xc[R];
+                    float wc[R], xc[R], nw[R];
                     unsigned ac[R];
                     float acc = 0.0f;
 #pragma unroll
                     for (int q = 0; q < R; ++q) {
                         const int i = q * 32 + lane;
-                        wv[q] = S.wp[slot][i];                  // past k: unused
-                        const float f = __fmaf_rn(wv[q], xv[q], acc);
-                        acc = i < k ? f : acc;
+                        wc[q] = wv[q];
                         xc[q] = xv[q];
-                        ac[q] = i < k ? pa[q] : dump;
+                        const float f = __fmaf_rn(wc[q], xc[q], acc);
+                        acc = i < k ? f : acc;
+                        ac[q] = i < k ? (pa[q] & PA_ADDR) : dump;
                     }
                     const float yc = yr;
                     trace_mark(trace, (int64_t)ep * N + r, 0);    // every weight is read
                     const float m = combine_smem(acc, S.part);
                     if (r + 1 < r1) fetch(r + 1);
-                    const float c = __fmul_rn(eta, dev_grad(loss, m, yc));
+                    const float c = __fmul_rn(eta, dev_grad(LOSS, m, yc));
                     trace_mark(trace, (int64_t)ep * N + r, 1);   // before any write is visible
 #pragma unroll
-                    for (int q = 0; q < R; ++q) st_shared(ac[q], __fsub_rn(wv[q], __fmul_rn(c, xc[q])));
+                    for (int q = 0; q < R; ++q) {
+                        nw[q] = __fsub_rn(wc[q], __fmul_rn(c, xc[q]));
+                        st_shared(ac[q], nw[q]);
+                    }
                     __syncwarp();
+                    if (r + 1 < r1) {
+                        const int nslot = (r + 1) & (CH_SLOTS - 1);
+#pragma unroll
+                        for (int q = 0; q < R; ++q) {
+                            const unsigned src = (pa[q] >> 23) & 0xffu;   // element of r
+                            if (R <= 2) {
+                                float v = wv[q];
+#pragma unroll
+                                for (int qs = 0; qs < R; ++qs) {
+                                    const float u = __shfl_sync(FULL, nw[qs], (int)(src & 31u));
+                                    if ((pa[q] & PA_LATE) && (int)(src >> 5) == qs) v = u;
+                                }
+                                wv[q] = v;
+                            } else if (pa[q] & PA_LATE) {
+                                wv[q] = S.wp[nslot][q * 32 + lane];   // stored above, before the __syncwarp
+                            }
+                        }
+                    }
                 }
             }
             __syncthreads();
@@ -316,6 +347,7 @@ __global__ void k_chain_link(const int32_t *__restrict__ prev, const int32_t *__
         const int32_t t = row_of[p], q = prev[p], n = next[p];
         uint32_t l = 0;
         if (q >= 0 && t - row_of[q] <= CH_D) l |= LK_RECV;
+        if (q >= 0 && row_of[q] == t - 1) l |= LK_LATE | ((uint32_t)(q - row_ptr[t - 1]) << 8);
         if (n >= 0) {
             const int32_t tn = row_of[n];
             if (tn - t <= CH_D) l |= LK_PUSH | ((uint32_t)(tn - t) << 16) | (uint32_t)(n - row_ptr[tn]);
@@ -340,21 +372,33 @@ int chain_schedule(const int32_t *prev, const int32_t *next, const int32_t *row_
     return cudaPeekAtLastError() == cudaSuccess ? PDB_OK : PDB_ECUDA;
 }
 
+using ChainKernel = void (*)(int32_t, const int64_t *, const int32_t *, const float *, const float *,
+                             const uint32_t *, float *, int, float, int, bool, int *, uint64_t *);
+
+template <int R>
+static ChainKernel chain_kernel(int loss)
+{
+    return loss == PDB_LOSS_LOGISTIC ? k_sgd_chain<R, PDB_LOSS_LOGISTIC>
+           : loss == PDB_LOSS_SQUARED ? k_sgd_chain<R, PDB_LOSS_SQUARED> : k_sgd_chain<R, PDB_LOSS_HINGE>;
+}
+
 int chain_run(const pdb_csr *X, const float *y, const uint32_t *link, float *w, int loss, float eta, int epochs,
               int max_row, int *status, uint64_t *trace, cudaStream_t s)
 {
-    // registers per lane for the longest example: 1, 2, 4 or 8 (32 to 256 ids)
-    auto kern = max_row <= 32 ? k_sgd_chain<1> : max_row <= 64 ? k_sgd_chain<2>
-              : max_row <= 128 ? k_sgd_chain<4> : k_sgd_chain<8>;
-    const int variant = max_row <= 32 ? 0 : max_row <= 64 ? 1 : max_row <= 128 ? 2 : 3;
+    // registers per lane for the longest example: 1, 2, 4 or 8 (32 to 256 ids);
+    // one kernel per loss, so the gradient has no branch
+    const int rw = max_row <= 32 ? 0 : max_row <= 64 ? 1 : max_row <= 128 ? 2 : 3;
+    const ChainKernel kern = rw == 0 ? chain_kernel<1>(loss) : rw == 1 ? chain_kernel<2>(loss)
+                             : rw == 2 ? chain_kernel<4>(loss) : chain_kernel<8>(loss);
+    const int variant = rw * 3 + (loss >= 0 && loss <= 2 ? loss : 2);
     // set once per device and variant (any device past the table: every call)
-    static std::atomic<bool> configured[64][4];
+    static std::atomic<bool> configured[64][12];
     int dev = 0;
     cudaGetDevice(&dev);
     const bool known = dev >= 0 && dev < 64;
     if (!known || !configured[dev][variant].load(std::memory_order_acquire)) {
-        if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sizeof(ChainSmem)) !=
-            cudaSuccess)
+        if (cudaFuncSetAttribute((const void *)kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)sizeof(ChainSmem)) != cudaSuccess)
             return PDB_ECUDA;
         if (known) configured[dev][variant].store(true, std::memory_order_release);
     }

@@ -15,10 +15,15 @@ separated only by the __syncthreads that ends each iteration:
                    its weights from its slot and storing each new weight
                    into the next occurrence's slot when that lies within
                    D = G * DS examples (a push), else into its own output
-                   slot for W.
+                   slot for W.  Every example but the first of a step
+                   fetches its weights while the example before it is still
+                   computing, before that example's stores; a weight whose
+                   previous occurrence is that very example is taken from
+                   it directly (a shuffle, or a reload after its stores).
 
 The model replays that schedule with the link words the engine builds from
-the conflict chains and checks, on problems full of near repeats: every
+the conflict chains (including the mark of a previous occurrence in the
+example just before) and checks, on problems full of near repeats: every
 example reads, for every feature, exactly the weight its previous occurrence
 wrote (in the epoch, or the last one of the epoch before); global w ends each
 epoch holding each feature's last writer; no two warps touch one shared or
@@ -40,14 +45,17 @@ def _links(p, D):
     prev, nxt = ch["prev"], ch["next"]
     row_of = np.repeat(np.arange(p.n_rows), np.diff(p.row_ptr))
     recv = np.zeros(p.nnz, bool)
+    late = np.zeros(p.nnz, bool)
     push = {}
     for q in range(p.nnz):
         t = row_of[q]
         if prev[q] >= 0 and t - row_of[prev[q]] <= D:
             recv[q] = True
+        if prev[q] >= 0 and row_of[prev[q]] == t - 1:
+            late[q] = True
         if nxt[q] >= 0 and row_of[nxt[q]] - t <= D:
             push[q] = (int(row_of[nxt[q]] - t), int(nxt[q] - p.row_ptr[row_of[nxt[q]]]))
-    return recv, push
+    return recv, push, late
 
 
 class _Iteration:
@@ -73,7 +81,7 @@ def _simulate(p, epochs, G, DS, BS, SLOTS, RP, D=None):
     L = DS + BS + 1
     N = p.n_rows
     rp = p.row_ptr
-    recv, push = _links(p, D)
+    recv, push, late = _links(p, D)
     steps = (N + G - 1) // G
     # weights are tracked as the example (epoch, id) that wrote them; None = w0
     w = {}
@@ -81,7 +89,7 @@ def _simulate(p, epochs, G, DS, BS, SLOTS, RP, D=None):
     for ep in range(epochs):
         ring = {}                         # rp ring: index -> example whose bound it holds
         slot_of = lambda r: r & (SLOTS - 1)
-        col, wp, out, pa = {}, {}, {}, {}
+        col, wp, out, pa, xa, kk, ys = {}, {}, {}, {}, {}, {}, {}
 
         def bounds(it, warp, r):
             if r < 0 or r >= N:
@@ -129,7 +137,9 @@ def _simulate(p, epochs, G, DS, BS, SLOTS, RP, D=None):
                         for arr in ("col", "link", "xa"):
                             it.w(warp, (arr, s, i))
                         effects.append(("col", (s, i), int(p.col[b + i])))
+                        effects.append(("xa", (s, i), (r, i)))
                     it.w(warp, ("y", s))
+                    effects.append(("y", s, r))
                 r = (t + BS) * G + g
                 bk = bounds(it, warp, r)
                 if bk is not None:
@@ -150,23 +160,35 @@ def _simulate(p, epochs, G, DS, BS, SLOTS, RP, D=None):
                         else:
                             effects.append(("pa", (s, i), ("out", s, i)))
                     it.w(warp, ("kk", s))
+                    effects.append(("kk", s, r))
             # C: the compute warp, examples of step t in data order (its own
             # accesses are ordered; pushes into a later example of the same
             # step are read after they are stored)
             if 0 <= t < steps:
                 local = {}
-                for r in range(t * G, min(N, t * G + G)):
+                fetched = local                   # the stores visible when an example fetched its weights
+                for g, r in enumerate(range(t * G, min(N, t * G + G))):
                     # the compute warp takes the length from the slot, not the ring
                     b, k = int(rp[r]), int(rp[r + 1] - rp[r])
                     s = slot_of(r)
                     it.r("C", ("kk", s))
                     it.r("C", ("y", s))
+                    # the slot's length, label and values were written for this very example
+                    assert kk.get(s) == r and ys.get(s) == r, ("slot holds another example", r, kk.get(s), ys.get(s))
                     for i in range(k):
                         for arr in ("xa", "pa", "wp"):
                             it.r("C", (arr, s, i))
+                        assert xa.get((s, i)) == (r, i), ("value of another example", r, i, xa.get((s, i)))
+                        assert col[(s, i)] == int(p.col[b + i]), ("id of another example", r, i)
                         j = int(p.col[b + i])
-                        got = local.get(("wp", s, i), wp.get((s, i)))
+                        if g > 0 and late[b + i]:
+                            got = (ep, r - 1)         # from the example just before, once it has computed
+                        else:
+                            got = fetched.get(("wp", s, i), wp.get((s, i)))
                         assert got == expect.get(j), ("wrong weight read", ep, r, j, got, expect.get(j))
+                    fetched = dict(local)             # the next example fetches before this one stores
+                    for i in range(k):
+                        j = int(p.col[b + i])
                         target = pa[(s, i)]
                         it.w("C", target)
                         local[target] = (ep, r)
@@ -181,6 +203,12 @@ def _simulate(p, epochs, G, DS, BS, SLOTS, RP, D=None):
                     ring[key] = v
                 elif kind == "col":
                     col[key] = v
+                elif kind == "xa":
+                    xa[key] = v
+                elif kind == "kk":
+                    kk[key] = v
+                elif kind == "y":
+                    ys[key] = v
                 elif kind == "wp":
                     wp[key] = v
                 elif kind == "pa":
