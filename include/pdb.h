@@ -422,6 +422,16 @@ int64_t pdb_launch_count(void);
  * with n > 0, is PDB_EINVAL. */
 int pdb_eval_expf(const float *x, float *out, int64_t n, void *stream);
 
+/* out[i] = eta-free loss derivative dloss/dm at margin m[i] and label y[i]
+ * (device arrays of n floats), the same function every engine applies
+ * (Section 6.3's SGD step, gradient of Eq. 2 without a regulariser):
+ * logistic -y / (1 + exp(y m)) with the exp above, squared m - y, hinge
+ * (y m < 1 ? -y : 0).  For the logistic loss with y = +1 or -1 and
+ * 1 <= 1 + exp(y m) < 2^126 the quotient is formed as a reciprocal, equal
+ * bit for bit to the IEEE division.  n < 0, an unknown loss, or a NULL array
+ * with n > 0 is PDB_EINVAL. */
+int pdb_eval_grad(const float *m, const float *y, float *out, int64_t n, pdb_loss loss, void *stream);
+
 #ifdef __cplusplus
 }
 #endif

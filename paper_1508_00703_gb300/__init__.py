@@ -109,7 +109,7 @@ class pdb_stats(ctypes.Structure):
 EXPORTS = ["pdb_build_conflicts", "pdb_conflicts_arrays", "pdb_schedule_build", "pdb_schedule_levels",
            "pdb_schedule_ready",
            "pdb_sgd_epoch", "pdb_bsp_epoch", "pdb_status", "pdb_get_stats", "pdb_conflicts_free",
-           "pdb_schedule_free", "pdb_strerror", "pdb_memcpy", "pdb_eval_expf", "pdb_launch_count",
+           "pdb_schedule_free", "pdb_strerror", "pdb_memcpy", "pdb_eval_expf", "pdb_eval_grad", "pdb_launch_count",
            "pdb_sgd_epoch_ready_noalloc", "pdb_ssp_epoch", "pdb_bsp_plan_build", "pdb_bsp_plan_batches",
            "pdb_bsp_coef", "pdb_bsp_apply", "pdb_bsp_plan_free"]
 
@@ -140,6 +140,7 @@ def load(path: str | None = None):
         lib.pdb_strerror.restype = ctypes.c_char_p
         lib.pdb_memcpy.argtypes = [P, P, ctypes.c_size_t, P]
         lib.pdb_eval_expf.argtypes = [P, P, I64, P]
+        lib.pdb_eval_grad.argtypes = [P, P, P, I64, I32, P]
         lib.pdb_sgd_epoch_ready_noalloc.argtypes = [ctypes.POINTER(pdb_csr), P, P, P, I32, ctypes.c_float, I32, P]
         lib.pdb_ssp_epoch.argtypes = [ctypes.POINTER(pdb_csr), P, P, P, P, I32, ctypes.c_float, I32, I64, P,
                                       ctypes.POINTER(pdb_opts), P]
@@ -436,6 +437,12 @@ def pdb_memcpy(dst_ptr: int, src_ptr: int, nbytes: int, stream=None):
     """Stream-ordered copy between device or host pointers (ints)."""
     _check(load().pdb_memcpy(ctypes.c_void_p(dst_ptr), ctypes.c_void_p(src_ptr), int(nbytes), _stream(stream)),
            "pdb_memcpy")
+
+
+def pdb_eval_grad(m, y, out, loss: int, stream=None):
+    """out = the library's device loss derivative at margins m and labels y
+    (float32 device tensors of one length)."""
+    _check(load().pdb_eval_grad(_ptr(m), _ptr(y), _ptr(out), m.numel(), int(loss), _stream(stream)), "pdb_eval_grad")
 
 
 def pdb_eval_expf(x, out, stream=None):

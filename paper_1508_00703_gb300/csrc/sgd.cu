@@ -561,6 +561,13 @@ __global__ void k_bsp_apply(int64_t s0, int64_t s1, int64_t r0, int64_t rows, co
     if (__any_sync(FULL, bad) && lane == 0) set_status(status, PDB_EFAULT);   // cannot happen with a consistent plan
 }
 
+__global__ void k_eval_grad(const float *__restrict__ m, const float *__restrict__ y, float *__restrict__ out,
+                            int64_t n, int loss)
+{
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x)
+        out[i] = dev_grad(loss, m[i], y[i]);
+}
+
 __global__ void k_eval_expf(const float *__restrict__ x, float *__restrict__ out, int64_t n)
 {
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x)
@@ -922,6 +929,16 @@ void pdb_bsp_plan_free(pdb_bsp_plan *p)
         if (q) cudaFreeAsync(q, 0);
     delete[] p->h_bptr;
     delete p;
+}
+
+int pdb_eval_grad(const float *m, const float *y, float *out, int64_t n, pdb_loss loss, void *stream)
+{
+    if (n < 0 || (n > 0 && (!m || !y || !out))) return PDB_EINVAL;
+    if (loss != PDB_LOSS_LOGISTIC && loss != PDB_LOSS_SQUARED && loss != PDB_LOSS_HINGE) return PDB_EINVAL;
+    if (n == 0) return PDB_OK;
+    k_eval_grad<<<grid_1d(n), 256, 0, (cudaStream_t)stream>>>(m, y, out, n, (int)loss);
+    note_launch();
+    return cudaPeekAtLastError() == cudaSuccess ? PDB_OK : PDB_ECUDA;
 }
 
 int pdb_eval_expf(const float *x, float *out, int64_t n, void *stream)

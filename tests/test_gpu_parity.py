@@ -54,6 +54,28 @@ def test_expf_matches_oracle_bitwise_and_fp64():
     assert np.max(np.abs(got[m] - e64) / ulp) <= 2.0
 
 
+@pytest.mark.parametrize("loss", [0, 1, 2])
+def test_loss_derivative_matches_oracle_bitwise(loss):
+    # the device's dloss/dm against the oracle's on margins from deep saturation
+    # to the far side, labels +-1 (the reciprocal path of the logistic loss,
+    # up to 1 + exp(ym) = 2^126 and past it), 0.5, -3 and 0, and special values
+    import oracle
+    rng = np.random.default_rng(11 + loss)
+    m = np.concatenate([np.linspace(-120, 120, 60_001), rng.normal(0, 4, 40_000),
+                        np.linspace(86.0, 89.5, 20_001)]).astype(np.float32)
+    m = np.concatenate([m, np.array([0.0, -0.0, 1.0, -1.0, np.inf, -np.inf, np.nan], np.float32)])
+    ys = [1.0, -1.0, 0.5, -3.0, 0.0]
+    mm = np.tile(m, len(ys))
+    yy = np.repeat(np.array(ys, np.float32), m.size)
+    out = torch.empty(mm.size, dtype=torch.float32, device="cuda")
+    pdb.pdb_eval_grad(torch.from_numpy(mm).cuda(), torch.from_numpy(yy).cuda(), out, loss)
+    got = out.cpu().numpy()
+    ref = np.array([oracle.grad(loss, float(a), float(b)) for a, b in zip(mm, yy)], np.float32)
+    nan = np.isnan(ref)
+    assert np.array_equal(np.isnan(got), nan)
+    assert np.array_equal(got[~nan].view(np.uint32), ref[~nan].view(np.uint32))
+
+
 @pytest.mark.parametrize("name", ALL)
 def test_chains_bit_exact(name):
     p, X, y = _gpu(name)
