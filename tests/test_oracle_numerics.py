@@ -99,13 +99,20 @@ def test_grad_logistic_closed_forms():
         assert oracle.grad(oracle.LOGISTIC, -200.0 * y, y) == -y   # e^{-200} = 0
 
 
-def test_grad_logistic_matches_fp64():
+def test_grad_logistic_is_the_derivative_of_the_logistic_loss():
+    # pinned to the loss itself, not to the oracle's formula: a central
+    # difference of L(m) = log(1 + exp(-y m)) in fp64 (log1p/exp, step h with
+    # truncation error ~ h^2 |L'''| / 6 and rounding ~ 1e-16 / h)
     rng = np.random.default_rng(2)
+    h = 1e-5
     for m in rng.uniform(-20, 20, 2000).astype(np.float32):
         for y in (1.0, -1.0):
-            ref = -y / (1.0 + math.exp(y * float(m)))
+            def loss(t):
+                z = -y * t
+                return z + math.log1p(math.exp(-z)) if z > 0 else math.log1p(math.exp(z))
+            fd = (loss(float(m) + h) - loss(float(m) - h)) / (2 * h)
             got = float(oracle.grad(oracle.LOGISTIC, m, y))
-            assert abs(got - ref) <= 4 * np.spacing(np.float32(abs(ref))), (m, y, got, ref)
+            assert abs(got - fd) <= 1e-9 + 4 * np.spacing(np.float32(abs(fd))), (m, y, got, fd)
 
 
 def test_grad_squared_and_hinge():

@@ -30,7 +30,10 @@ PLANTS = {
         [num.test_expf_within_2ulp_dense_grid, num.test_expf_within_2ulp_random_and_small]),
     "exp-argument-sign": (
         "return -y / (1.0f + orc_expf(y * m));", "return -y / (1.0f + orc_expf(-y * m));",
-        [num.test_grad_logistic_closed_forms, num.test_grad_logistic_matches_fp64]),
+        [num.test_grad_logistic_closed_forms, num.test_grad_logistic_is_the_derivative_of_the_logistic_loss]),
+    "logistic-numerator-sign": (
+        "return -y / (1.0f + orc_expf(y * m));", "return y / (1.0f + orc_expf(y * m));",
+        [num.test_grad_logistic_is_the_derivative_of_the_logistic_loss]),
     "butterfly-stage-missing": (
         "for (int off = 16; off >= 1; off >>= 1) {", "for (int off = 16; off >= 2; off >>= 1) {",
         [num.test_dot_exact_on_small_integers, num.test_dot_uses_32_partial_sums]),
