@@ -475,6 +475,8 @@ def run_e2e(args, p, mode, pdb, torch, world):
             b.read.record(copy_out)
         return c, s
 
+    phases = []
+
     def run(steps):
         stage(0)
         for i in range(steps):
@@ -484,11 +486,13 @@ def run_e2e(args, p, mode, pdb, torch, world):
             rc = pdb.pdb_status(c, main)        # synchronizes main: step i's kernels are done
             if rc != 0:
                 raise pdb.PdbError(rc, "e2e step")
+            phases.append(pdb.pdb_get_stats(c, s))   # the step's device phases (CUDA events)
             del c, s
         copy_out.synchronize()                  # the last step's weights are on the host
 
     steps = max(2, min(args.steps, 10))
     run(2)
+    phases.clear()
     # the host link's bandwidth on this machine, for reading the number (after the
     # warm-up steps; best of two copies each way)
     link = {}
@@ -513,6 +517,8 @@ def run_e2e(args, p, mode, pdb, torch, world):
     units = reduce_sum(p.epochs * p.nnz, world)
     return {"value": units / dt, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
             "ms_per_step": dt * 1e3, "steps": steps, "host_link": link,
+            "device_phases_ms": {"build_conflicts": statistics.median(ph["ms_build"] for ph in phases),
+                                 "sgd_all_epochs": statistics.median(ph["ms_sgd"] for ph in phases)},
             "pipeline": "step i+1's H2D on a copy stream and step i's D2H on another, overlapping the next step"}
 
 

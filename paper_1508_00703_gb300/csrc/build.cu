@@ -171,7 +171,10 @@ __global__ void k_slots(const uint32_t *__restrict__ skey, const int32_t *__rest
             const uint32_t j = kk[e + 1];
             const int32_t p = pp[e + 1];
             const bool last = s == nnz - 1 || kk[e + 2] != j;
-            r = (e > 0 && kk[e] == j) ? r + 1 : s - feat_ptr[j];
+            // rank: 0 where the feature's run starts, one more than the slot before
+            // inside the group, and from the run's first slot (feat_ptr) only for a
+            // run that began before this group
+            r = kk[e] != j ? 0 : e > 0 ? r + 1 : s - feat_ptr[j];
             const bool near_prev = r > 0 && (int64_t)p - pp[e] < near;
             const bool near_next = !last && (int64_t)pp[e + 2] - p < near;
             big |= r > (int64_t)GATE_RANK;
