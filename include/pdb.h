@@ -350,7 +350,7 @@ int pdb_bsp_epoch(const pdb_csr *X, const float *y, const pdb_conflicts *c, floa
  *   the batch's coefficients in row order (device, rows of the batch
  *   floats); w updated in place.  Asynchronous.  An inconsistent plan is
  *   PDB_EFAULT in c's status word.
- * pdb_bsp_plan_free: waits for the device, frees the plan's arrays. */
+ * pdb_bsp_plan_free: waits for the work enqueued on the plan, frees its arrays. */
 int pdb_bsp_plan_build(const pdb_conflicts *c, int64_t batch, pdb_bsp_plan **out, void *stream);
 int64_t pdb_bsp_plan_batches(const pdb_bsp_plan *p);
 int pdb_bsp_coef(const pdb_bsp_plan *p, const pdb_csr *X, const float *y, const float *w, pdb_loss loss, float eta,
@@ -363,11 +363,14 @@ void pdb_bsp_plan_free(pdb_bsp_plan *p);
  * PDB_ETIMEOUT, PDB_EFAULT); PDB_ECUDA if the synchronization itself fails. */
 int pdb_status(const pdb_conflicts *c, void *stream);
 
-/* Sizes and timings; SYNCHRONIZES (device) to read the event timers and L.
- * s may be NULL. */
+/* Sizes and timings; waits (host) for the work enqueued on c and s to read
+ * the event timers and L, not for the device's other streams.  s may be
+ * NULL. */
 int pdb_get_stats(const pdb_conflicts *c, const pdb_schedule *s, pdb_stats *out);
 
-/* Release a handle (waits for the device, then frees its arrays). */
+/* Release a handle: waits for the work enqueued on this handle by earlier
+ * calls (not for the rest of the device, whose other streams keep running),
+ * then returns its arrays to the library's memory pool. */
 void pdb_conflicts_free(pdb_conflicts *c);
 void pdb_schedule_free(pdb_schedule *s);
 

@@ -27,7 +27,9 @@
 #include <cstdio>
 #include <cstdlib>
 #include <cstring>
+#include <mutex>
 #include <new>
+#include <vector>
 
 #include "common.cuh"
 
@@ -449,9 +451,9 @@ int check_csr(const pdb_csr *X)
     return PDB_OK;
 }
 
-// Callers synchronize the device first.  The arrays go back to the
-// stream-ordered pool (kept, not returned to the driver), so freeing costs no
-// device-wide synchronization and the next build reuses the memory.
+// Callers wait for the handle's last use first (its ev_use).  The arrays go
+// back to the stream-ordered pool (kept, not returned to the driver), so the
+// next build reuses the memory.
 void free_ptrs(std::initializer_list<void *> ptrs)
 {
     for (void *p : ptrs)
@@ -563,6 +565,40 @@ int materialize_chains(pdb_conflicts *c, cudaStream_t s)
 // ------------------------------------------------------------------ C ABI
 namespace pdb {
 
+void mark_use(const pdb_conflicts *c, const pdb_schedule *h, cudaStream_t s)
+{
+    if (c && c->ev_use) cudaEventRecord(c->ev_use, s);
+    if (h && h->ev_use) cudaEventRecord(h->ev_use, s);
+}
+
+static std::mutex g_slot_lock;
+static std::vector<int *> g_free_slots;
+
+int *info_slot_take()
+{
+    std::lock_guard<std::mutex> guard(g_slot_lock);
+    if (g_free_slots.empty()) {
+        constexpr int SLOTS = 64;
+        int *slab = nullptr;
+        if (cudaHostAlloc((void **)&slab, sizeof(int) * INFO_WORDS * SLOTS, cudaHostAllocDefault) != cudaSuccess) {
+            cudaGetLastError();
+            return nullptr;
+        }
+        for (int i = SLOTS - 1; i >= 0; --i) g_free_slots.push_back(slab + i * INFO_WORDS);
+    }
+    int *slot = g_free_slots.back();
+    g_free_slots.pop_back();
+    std::memset(slot, 0, sizeof(int) * INFO_WORDS);
+    return slot;
+}
+
+void info_slot_give(int *slot)
+{
+    if (!slot) return;
+    std::lock_guard<std::mutex> guard(g_slot_lock);
+    g_free_slots.push_back(slot);
+}
+
 ApiScope::ApiScope(const char *name_, const pdb_conflicts *c_, const pdb_schedule *h_, pdb_conflicts *const *pc_,
                    pdb_schedule *const *ph_, bool log_)
     : name(name_), c(c_), h(h_), pc(pc_), ph(ph_), log(log_)
@@ -620,11 +656,12 @@ const char *pdb_strerror(int code)
 void pdb_conflicts_free(pdb_conflicts *c)
 {
     if (!c) return;
-    cudaDeviceSynchronize();
+    // the handle's own work only: other streams of the device keep running
+    if (c->ev_use) cudaEventSynchronize(c->ev_use);
     free_ptrs({c->csc_pos, c->feat_ptr, c->gate, c->gate_sorted, c->gate_window != c->gate ? c->gate_window : nullptr,
                c->row_of, c->prev, c->next, c->rank, c->npred, c->info});
-    if (c->h_info) cudaFreeHost(c->h_info);
-    for (cudaEvent_t e : {c->ev0, c->ev1, c->ev_sgd0, c->ev_sgd1, c->ev_bsp0, c->ev_bsp1, c->ev_k0, c->ev_k1})
+    info_slot_give(c->h_info);
+    for (cudaEvent_t e : {c->ev0, c->ev1, c->ev_sgd0, c->ev_sgd1, c->ev_bsp0, c->ev_bsp1, c->ev_k0, c->ev_k1, c->ev_use})
         if (e) cudaEventDestroy(e);
     delete c;
 }
@@ -666,12 +703,15 @@ int pdb_build_conflicts(const pdb_csr *X, pdb_conflicts **out, void *stream)
             pdb_conflicts_free(c);
             return PDB_ECUDA;
         }
-    if (cudaMallocHost((void **)&c->h_info, sizeof(int) * INFO_WORDS) != cudaSuccess) {
-        cudaGetLastError();
+    if (cudaEventCreateWithFlags(&c->ev_use, cudaEventDisableTiming) != cudaSuccess) {
+        pdb_conflicts_free(c);
+        return PDB_ECUDA;
+    }
+    c->h_info = info_slot_take();
+    if (!c->h_info) {
         pdb_conflicts_free(c);
         return PDB_ENOMEM;
     }
-    std::memset(c->h_info, 0, sizeof(int) * INFO_WORDS);
     cudaEventRecord(c->ev0, s);
     rc = alloc((void **)&c->info, sizeof(int) * INFO_WORDS, s);
     rc = rc ? rc : alloc((void **)&c->csc_pos, sizeof(int32_t) * nnz, s);
@@ -717,6 +757,7 @@ int pdb_build_conflicts(const pdb_csr *X, pdb_conflicts **out, void *stream)
     release(tval, s);
     if (rc == PDB_OK) cudaMemcpyAsync(c->h_info, c->info, sizeof(int) * INFO_WORDS, cudaMemcpyDeviceToHost, s);
     cudaEventRecord(c->ev1, s);
+    mark_use(c, nullptr, s);
     c->timed_build = true;
     if (rc == PDB_OK && cudaPeekAtLastError() != cudaSuccess) rc = PDB_ECUDA;
     if (rc != PDB_OK) {
@@ -736,6 +777,7 @@ int pdb_conflicts_arrays(const pdb_conflicts *c, const int32_t **csc_pos, const 
     pdb_conflicts *cm = const_cast<pdb_conflicts *>(c);
     if (prev || next || rank) {
         int rc = materialize_chains(cm, (cudaStream_t)stream);
+        mark_use(c, nullptr, (cudaStream_t)stream);
         if (rc != PDB_OK) return rc;
     }
     if (csc_pos) *csc_pos = c->csc_pos;
@@ -758,11 +800,12 @@ int pdb_status(const pdb_conflicts *c, void *stream)
 void pdb_schedule_free(pdb_schedule *s)
 {
     if (!s) return;
-    cudaDeviceSynchronize();
+    // the schedule's own work only: other streams of the device keep running
+    if (s->ev_use) cudaEventSynchronize(s->ev_use);
     free_ptrs({s->level, s->order, s->indeg, s->queue, s->level_ptr, s->ctl, s->rec, s->link, s->bar, s->ticket,
                s->prog, s->wctl, s->reads, s->writes, s->rbits, s->wbits});
-    if (s->ev0) cudaEventDestroy(s->ev0);
-    if (s->ev1) cudaEventDestroy(s->ev1);
+    for (cudaEvent_t e : {s->ev0, s->ev1, s->ev_use})
+        if (e) cudaEventDestroy(e);
     delete s;
 }
 
@@ -794,7 +837,8 @@ int pdb_schedule_build(const pdb_conflicts *c, pdb_sched_mode mode, pdb_schedule
     if (!h) return PDB_ENOMEM;
     h->c = c;
     h->mode = mode;
-    if (cudaEventCreate(&h->ev0) != cudaSuccess || cudaEventCreate(&h->ev1) != cudaSuccess) {
+    if (cudaEventCreate(&h->ev0) != cudaSuccess || cudaEventCreate(&h->ev1) != cudaSuccess ||
+        cudaEventCreateWithFlags(&h->ev_use, cudaEventDisableTiming) != cudaSuccess) {
         pdb_schedule_free(h);
         return PDB_ECUDA;
     }
@@ -905,6 +949,7 @@ int pdb_schedule_build(const pdb_conflicts *c, pdb_sched_mode mode, pdb_schedule
         release(tval, s);
     }
     cudaEventRecord(h->ev1, s);
+    mark_use(c, h, s);     // the schedule's build also reads and extends c's arrays
     h->timed = true;
     if (rc == PDB_OK && cudaPeekAtLastError() != cudaSuccess) rc = PDB_ECUDA;
     if (rc != PDB_OK) {
@@ -947,7 +992,10 @@ int pdb_get_stats(const pdb_conflicts *c, const pdb_schedule *h, pdb_stats *out)
 {
     if (!c || !out) return PDB_EINVAL;
     std::memset(out, 0, sizeof *out);
-    if (cudaDeviceSynchronize() != cudaSuccess) return PDB_ECUDA;
+    // the work enqueued on these handles (their timers and words are final then)
+    if ((c->ev_use && cudaEventSynchronize(c->ev_use) != cudaSuccess) ||
+        (h && h->ev_use && cudaEventSynchronize(h->ev_use) != cudaSuccess))
+        return PDB_ECUDA;
     out->n_rows = c->n_rows;
     out->n_cols = c->n_cols;
     out->nnz = c->nnz;

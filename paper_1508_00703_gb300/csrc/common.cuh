@@ -299,6 +299,7 @@ struct pdb_conflicts {
                              // [4] near occurrence pairs
     int *h_info;             // pinned host copy of info, filled at the end of the build
     cudaEvent_t ev0, ev1, ev_sgd0, ev_sgd1, ev_bsp0, ev_bsp1, ev_k0, ev_k1;
+    cudaEvent_t ev_use;      // recorded after the last work any call enqueued on the handle
     bool timed_build, timed_sgd, timed_bsp;
     int *status;             // = info (first error recorded by a kernel)
 };
@@ -330,6 +331,7 @@ struct pdb_schedule {
     pdb::GridBarrier *bar;    // barrier for the level-synchronous engine
     unsigned long long *ticket;
     cudaEvent_t ev0, ev1;
+    cudaEvent_t ev_use;      // recorded after the last work any call enqueued on the handle
     bool timed;
 };
 
@@ -342,10 +344,29 @@ struct pdb_bsp_plan {
     int64_t *bptr;            // [n_batches + 1] device
     int64_t *h_bptr;          // [n_batches + 1] host
     int32_t *bcol, *brow;
+    cudaEvent_t ev_use;       // recorded after the last work any call enqueued on the plan
     float *bval;
 };
 
 namespace pdb {
+// Handles record ev_use on the call's stream after every call that enqueues
+// work on them; freeing a handle waits for that event only (not for the whole
+// device, where other streams may be busy), then returns its arrays to the
+// pool.
+void mark_use(const pdb_conflicts *c, const pdb_schedule *h, cudaStream_t s);
+// records ev_use of the handles on the call's stream when the call returns
+// (every return path, after everything the call enqueued)
+struct UseMark {
+    const pdb_conflicts *c;
+    const pdb_schedule *h;
+    cudaStream_t s;
+    ~UseMark() { mark_use(c, h, s); }
+};
+// host-side pinned words for a conflicts handle's info copy, from a slab that
+// is kept for the process (freeing pinned memory would synchronize the device)
+int *info_slot_take();
+void info_slot_give(int *slot);
+
 // Scope of one C-ABI call: an NVTX range named after the call (shown by
 // profilers, a no-op without one), and, when the environment variable
 // PDB_LOG is set to anything but "" or "0", one line of pdb_get_stats on

@@ -606,6 +606,7 @@ int pdb_sgd_epoch(const pdb_csr *X, const float *y, const pdb_conflicts *c, cons
                   pdb_loss loss, float eta, int n_epochs, const pdb_opts *opts, void *stream)
 {
     ApiScope scope("pdb_sgd_epoch", c, h);
+    UseMark use{c, h, (cudaStream_t)stream};
     int rc = check_run(X, y, c, w, loss, n_epochs);
     if (rc != PDB_OK) return rc;
     if (!h || h->c != c) return PDB_EINVAL;
@@ -680,6 +681,7 @@ int pdb_ssp_epoch(const pdb_csr *X, const float *y, const pdb_conflicts *c, cons
                   void *stream)
 {
     ApiScope scope("pdb_ssp_epoch", c, h);
+    UseMark use{c, h, (cudaStream_t)stream};
     int rc = check_run(X, y, c, w, loss, n_epochs);
     if (rc != PDB_OK) return rc;
     if (!h || h->c != c || delay < 0) return PDB_EINVAL;
@@ -735,6 +737,7 @@ int pdb_bsp_epoch(const pdb_csr *X, const float *y, const pdb_conflicts *c, floa
                   int64_t batch, int n_epochs, const pdb_opts *opts, void *stream)
 {
     ApiScope scope("pdb_bsp_epoch", c);
+    UseMark use{c, nullptr, (cudaStream_t)stream};
     int rc = check_run(X, y, c, w, loss, n_epochs);
     if (rc != PDB_OK) return rc;
     if (batch < 1) return PDB_EINVAL;
@@ -832,6 +835,10 @@ int pdb_bsp_plan_build(const pdb_conflicts *c, int64_t batch, pdb_bsp_plan **out
     if (!p) return PDB_ENOMEM;
     p->c = c;
     p->batch = batch;
+    if (cudaEventCreateWithFlags(&p->ev_use, cudaEventDisableTiming) != cudaSuccess) {
+        cudaGetLastError();
+        p->ev_use = nullptr;
+    }
     p->n_batches = N > 0 ? (N + batch - 1) / batch : 0;
     uint32_t *key = nullptr, *skey = nullptr, *tkey = nullptr;
     int32_t *bpos = nullptr, *tval = nullptr;
@@ -888,6 +895,7 @@ int pdb_bsp_coef(const pdb_bsp_plan *p, const pdb_csr *X, const float *y, const 
                  int64_t row_begin, int64_t row_end, float *coef, void *stream)
 {
     ApiScope scope("pdb_bsp_coef", p ? p->c : nullptr, nullptr, nullptr, nullptr, false);
+    UseMark use{p ? p->c : nullptr, nullptr, (cudaStream_t)stream};
     if (!p) return PDB_EINVAL;
     int rc = check_run(X, y, p->c, w, loss, 1);
     if (rc != PDB_OK) return rc;
@@ -906,6 +914,7 @@ int pdb_bsp_coef(const pdb_bsp_plan *p, const pdb_csr *X, const float *y, const 
 int pdb_bsp_apply(const pdb_bsp_plan *p, float *w, int64_t batch_index, const float *coef, void *stream)
 {
     ApiScope scope("pdb_bsp_apply", p ? p->c : nullptr, nullptr, nullptr, nullptr, false);
+    UseMark use{p ? p->c : nullptr, nullptr, (cudaStream_t)stream};
     if (!p || batch_index < 0 || batch_index >= p->n_batches) return PDB_EINVAL;
     if (p->c->n_cols > 0 && !w) return PDB_EINVAL;
     const int64_t s0 = p->h_bptr[batch_index], s1 = p->h_bptr[batch_index + 1];
@@ -917,13 +926,18 @@ int pdb_bsp_apply(const pdb_bsp_plan *p, float *w, int64_t batch_index, const fl
     k_bsp_apply<<<(unsigned)blocks, 256, 0, s>>>(s0, s1, r0, rows, p->bcol, p->brow, p->bval, coef, w,
                                                  const_cast<pdb_conflicts *>(p->c)->status);
     note_launch();
+    if (p->ev_use) cudaEventRecord(p->ev_use, s);
     return cudaPeekAtLastError() == cudaSuccess ? PDB_OK : PDB_ECUDA;
 }
 
 void pdb_bsp_plan_free(pdb_bsp_plan *p)
 {
     if (!p) return;
-    cudaDeviceSynchronize();
+    // the plan's own work only: other streams of the device keep running
+    if (p->ev_use) {
+        cudaEventSynchronize(p->ev_use);
+        cudaEventDestroy(p->ev_use);
+    }
     cudaGetLastError();
     for (void *q : {(void *)p->bptr, (void *)p->bcol, (void *)p->brow, (void *)p->bval})
         if (q) cudaFreeAsync(q, 0);
