@@ -424,7 +424,9 @@ def run_e2e(args, p, mode, pdb, torch, world):
     weights go back to the host on a third stream while step i+1 computes (a
     double-buffered input pipeline, as a training loop that streams its data
     would run it)."""
-    main = torch.cuda.current_stream()
+    # a stream of its own for the compute: the legacy default stream would order
+    # itself against the copy streams
+    main = torch.cuda.Stream()
     h_row = torch.from_numpy(p.row_ptr).pin_memory()
     h_col = torch.from_numpy(p.col).pin_memory()
     h_val = None if p.val is None else torch.from_numpy(p.val).pin_memory()

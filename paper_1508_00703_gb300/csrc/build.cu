@@ -451,13 +451,16 @@ int check_csr(const pdb_csr *X)
     return PDB_OK;
 }
 
-// Callers wait for the handle's last use first (its ev_use).  The arrays go
-// back to the stream-ordered pool (kept, not returned to the driver), so the
-// next build reuses the memory.
+// Callers wait for the handle's last use first (its ev_use), so the arrays
+// are idle: they go back to the stream-ordered pool (kept, not returned to the
+// driver) on the library's own stream, and the next allocation on any stream
+// reuses them without an ordering against the legacy default stream (which
+// would wait for every blocking stream's pending work).
 void free_ptrs(std::initializer_list<void *> ptrs)
 {
+    cudaStream_t s = own_stream();
     for (void *p : ptrs)
-        if (p) cudaFreeAsync(p, 0);
+        if (p) cudaFreeAsync(p, s);
 }
 
 }  // namespace
@@ -571,6 +574,25 @@ void mark_use(const pdb_conflicts *c, const pdb_schedule *h, cudaStream_t s)
     if (h && h->ev_use) cudaEventRecord(h->ev_use, s);
 }
 
+// Small device-to-host reads of handle words.  A plain cudaMemcpy runs on the
+// legacy default stream, which waits for every blocking stream of the device
+// (another caller's copies, say); these reads go on the caller's stream, or,
+// where the call has none, on the library's own stream (own_stream).
+static int read_words(void *dst, const void *src, size_t bytes, cudaStream_t s)
+{
+    if (cudaMemcpyAsync(dst, src, bytes, cudaMemcpyDeviceToHost, s) != cudaSuccess ||
+        cudaStreamSynchronize(s) != cudaSuccess) {
+        cudaGetLastError();
+        return PDB_ECUDA;
+    }
+    return PDB_OK;
+}
+
+static int read_words(void *dst, const void *src, size_t bytes)
+{
+    return read_words(dst, src, bytes, own_stream());
+}
+
 static std::mutex g_slot_lock;
 static std::vector<int *> g_free_slots;
 
@@ -620,7 +642,7 @@ ApiScope::~ApiScope()
         return;
     }
     int status = 0;
-    cudaMemcpy(&status, cc->status, sizeof status, cudaMemcpyDeviceToHost);
+    read_words(&status, cc->status, sizeof status);
     std::fprintf(stderr,
                  "pdb %s: n_rows=%lld n_cols=%lld nnz=%lld max_chain=%lld sched_mode=%lld n_levels=%lld "
                  "max_level_width=%lld ms_build=%.3f ms_schedule=%.3f ms_sgd=%.3f ms_sgd_kernels=%.3f ms_bsp=%.3f "
@@ -791,9 +813,8 @@ int pdb_conflicts_arrays(const pdb_conflicts *c, const int32_t **csc_pos, const 
 int pdb_status(const pdb_conflicts *c, void *stream)
 {
     if (!c) return PDB_EINVAL;
-    if (cudaStreamSynchronize((cudaStream_t)stream) != cudaSuccess) return PDB_ECUDA;
     int st = 0;
-    if (cudaMemcpy(&st, c->status, sizeof(int), cudaMemcpyDeviceToHost) != cudaSuccess) return PDB_ECUDA;
+    if (read_words(&st, c->status, sizeof(int), (cudaStream_t)stream) != PDB_OK) return PDB_ECUDA;   // after the stream's work
     return st;
 }
 
@@ -971,9 +992,8 @@ int pdb_schedule_levels(const pdb_schedule *h, const int32_t **level, const int3
     if (order) *order = h->order;
     if (level_ptr) *level_ptr = h->level_ptr;
     if (n_levels) {
-        if (cudaStreamSynchronize((cudaStream_t)stream) != cudaSuccess) return PDB_ECUDA;
         LevelCtl ctl;
-        if (cudaMemcpy(&ctl, h->ctl, sizeof ctl, cudaMemcpyDeviceToHost) != cudaSuccess) return PDB_ECUDA;
+        if (read_words(&ctl, h->ctl, sizeof ctl, (cudaStream_t)stream) != PDB_OK) return PDB_ECUDA;
         *n_levels = h->c->n_rows > 0 ? ctl.n_levels : 0;
     }
     return PDB_OK;
@@ -1002,7 +1022,7 @@ int pdb_get_stats(const pdb_conflicts *c, const pdb_schedule *h, pdb_stats *out)
     out->n_levels = -1;
     out->max_level_width = -1;
     int info[INFO_WORDS] = {};
-    if (cudaMemcpy(info, c->info, sizeof info, cudaMemcpyDeviceToHost) != cudaSuccess) return PDB_ECUDA;
+    if (read_words(info, c->info, sizeof info) != PDB_OK) return PDB_ECUDA;
     out->max_chain = info[INFO_MAX_CHAIN];
     float ms = 0;
     if (c->timed_build && cudaEventElapsedTime(&ms, c->ev0, c->ev1) == cudaSuccess) out->ms_build = ms;
@@ -1015,7 +1035,7 @@ int pdb_get_stats(const pdb_conflicts *c, const pdb_schedule *h, pdb_stats *out)
         if (h->timed && cudaEventElapsedTime(&ms, h->ev0, h->ev1) == cudaSuccess) out->ms_schedule = ms;
         if (h->mode == PDB_SCHED_LEVELS) {
             LevelCtl ctl;
-            if (cudaMemcpy(&ctl, h->ctl, sizeof ctl, cudaMemcpyDeviceToHost) != cudaSuccess) return PDB_ECUDA;
+            if (read_words(&ctl, h->ctl, sizeof ctl) != PDB_OK) return PDB_ECUDA;
             out->n_levels = c->n_rows > 0 ? ctl.n_levels : 0;
             out->max_level_width = ctl.max_width;
         }

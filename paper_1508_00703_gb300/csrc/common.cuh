@@ -26,6 +26,7 @@ int persistent_grid(const void *kernel, const pdb_opts *opts);
 uint64_t timeout_ns(const pdb_opts *opts);
 int alloc(void **p, size_t bytes, cudaStream_t s);   // stream-ordered, 256-byte aligned
 void release(void *p, cudaStream_t s);
+cudaStream_t own_stream();                           // the library's non-blocking stream (current device)
 int bits_for(int64_t max_key);                        // bits to hold values 0..max_key (>= 1)
 int grid_1d(int64_t n);                               // blocks of 256 threads for a grid-stride loop
 

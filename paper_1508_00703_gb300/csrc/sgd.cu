@@ -940,7 +940,7 @@ void pdb_bsp_plan_free(pdb_bsp_plan *p)
     }
     cudaGetLastError();
     for (void *q : {(void *)p->bptr, (void *)p->bcol, (void *)p->brow, (void *)p->bval})
-        if (q) cudaFreeAsync(q, 0);
+        if (q) cudaFreeAsync(q, own_stream());
     delete[] p->h_bptr;
     delete p;
 }

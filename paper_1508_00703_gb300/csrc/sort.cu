@@ -74,6 +74,23 @@ static cudaMemPool_t library_pool(int device)
     return g_pool[device];
 }
 
+// The library's own non-blocking stream per device, for work that belongs to
+// no caller stream: small reads of handle words and the frees of idle arrays.
+static std::mutex g_own_lock;
+static cudaStream_t g_own_stream[64];
+
+cudaStream_t own_stream()
+{
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
+    std::lock_guard<std::mutex> guard(g_own_lock);
+    if (!g_own_stream[dev] && cudaStreamCreateWithFlags(&g_own_stream[dev], cudaStreamNonBlocking) != cudaSuccess) {
+        cudaGetLastError();
+        return nullptr;
+    }
+    return g_own_stream[dev];
+}
+
 int alloc(void **p, size_t bytes, cudaStream_t s)
 {
     *p = nullptr;
