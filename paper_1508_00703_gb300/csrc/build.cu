@@ -895,7 +895,8 @@ int pdb_schedule_build(const pdb_conflicts *c, pdb_sched_mode mode, pdb_schedule
             rc = rc ? rc : materialize_chains(cm, s);
             rc = rc ? rc : alloc((void **)&h->link, sizeof(uint32_t) * nnz, s);
             rc = rc ? rc : ensure_row_of(cm, s);
-            rc = rc ? rc : chain_schedule(c->prev, c->next, c->row_of, c->row_ptr, nnz, h->link, c->status, s);
+            rc = rc ? rc : chain_schedule(c->prev, c->next, c->row_of, c->row_ptr, nnz, c->h_info[INFO_MAX_ROW], h->link,
+                                          c->status, s);
         }
     } else {
         // Theorem 3's levels by dataflow (default) or by the Kahn frontier sweep

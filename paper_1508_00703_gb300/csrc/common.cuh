@@ -39,7 +39,7 @@ int block_ready_run(const pdb_csr *X, const float *y, const uint32_t *gate, floa
 int resident_run(const pdb_csr *X, const float *y, float *w, int loss, float eta, int epochs, int max_row,
                  int *status, uint64_t *trace, cudaStream_t s);
 int chain_schedule(const int32_t *prev, const int32_t *next, const int32_t *row_of, const int64_t *row_ptr,
-                   int64_t nnz, uint32_t *link, const int *status, cudaStream_t s);
+                   int64_t nnz, int64_t max_row, uint32_t *link, const int *status, cudaStream_t s);
 int chain_run(const pdb_csr *X, const float *y, const uint32_t *link, float *w, int loss, float eta, int epochs,
               int max_row, int *status, uint64_t *trace, cudaStream_t s);
 void note_launch();                                   // count one kernel launch (pdb_launch_count)
@@ -160,11 +160,11 @@ __device__ __forceinline__ bool grid_sync(GridBarrier *bar, int *status, uint64_
 // rint and the conversion of k to an integer both come from one exact
 // addition of 1.5 * 2^23 (|x log2e| < 2^22: the sum's last mantissa bits are
 // k, rounded to nearest even); a NaN input is returned at the end, so the
-// path has no branch.
+// path has no branch (the clamp, a min and a max, maps NaN to -104 on the
+// way).  k*head is exact, so x - k*head is one fused multiply-add.
 __device__ __forceinline__ float dev_expf(float x0)
 {
-    float x = x0 > 89.0f ? 89.0f : x0;
-    x = x < -104.0f ? -104.0f : x;
+    const float x = fminf(fmaxf(x0, -104.0f), 89.0f);
     const float log2e = 1.44269502162933349609375f;      // nearest float to log2(e)
     const float ln2_head = 0.693145751953125f;           // 45426 * 2^-16
     const float ln2_tail = 1.428606765330187045e-06f;     // ln2 - head, rounded to float
@@ -172,7 +172,7 @@ __device__ __forceinline__ float dev_expf(float x0)
     const float u = __fadd_rn(__fmul_rn(x, log2e), shifter);
     const float kf = __fsub_rn(u, shifter);
     const int k = __float_as_int(u) - 0x4B400000;
-    float r = __fsub_rn(x, __fmul_rn(kf, ln2_head));
+    float r = __fmaf_rn(-kf, ln2_head, x);
     r = __fsub_rn(r, __fmul_rn(kf, ln2_tail));
     float p = 1.0f / 5040.0f;
     p = __fmaf_rn(p, r, 1.0f / 720.0f);
@@ -221,19 +221,34 @@ __device__ __forceinline__ float recip_ge1(float d)
 
 // derivative of the example's loss with respect to its margin m; for the
 // logistic loss with y = +1 or -1, -y/d = -y * (1/d) exactly (rounding to
-// nearest is symmetric), so the reciprocal above gives the IEEE quotient's bits
+// nearest is symmetric), so the reciprocal above gives the IEEE quotient's
+// bits.  The reciprocal is formed unconditionally and the division taken only
+// outside its range, so the common path has no branch.
 __device__ __forceinline__ float dev_grad(int loss, float m, float y)
 {
     if (loss == PDB_LOSS_LOGISTIC) {
         const float d = __fadd_rn(1.0f, dev_expf(__fmul_rn(y, m)));
-        if ((y == 1.0f || y == -1.0f) && d < 0x1p126f) {
-            const float q = recip_ge1(d);
-            return y > 0.0f ? -q : q;
-        }
-        return __fdiv_rn(-y, d);
+        const float q = recip_ge1(d);
+        float g = y > 0.0f ? -q : q;
+        if (!((y == 1.0f || y == -1.0f) && d < 0x1p126f)) g = __fdiv_rn(-y, d);
+        return g;
     }
     if (loss == PDB_LOSS_SQUARED) return __fsub_rn(m, y);
     return __fmul_rn(y, m) < 1.0f ? -y : 0.0f;
+}
+
+// the step size times the derivative, eta * dev_grad(loss, m, y), with the
+// same bits: on the reciprocal path eta * (-y q) = (-y eta) * q exactly, so
+// the sign goes on eta, which is known before m
+__device__ __forceinline__ float dev_step(int loss, float m, float y, float eta)
+{
+    if (loss == PDB_LOSS_LOGISTIC) {
+        const float d = __fadd_rn(1.0f, dev_expf(__fmul_rn(y, m)));
+        float c = __fmul_rn(y > 0.0f ? -eta : eta, recip_ge1(d));
+        if (!((y == 1.0f || y == -1.0f) && d < 0x1p126f)) c = __fmul_rn(eta, __fdiv_rn(-y, d));
+        return c;
+    }
+    return __fmul_rn(eta, dev_grad(loss, m, y));
 }
 
 // combine the 32 lane partial sums pairwise: xor 16, 8, 4, 2, 1 (every lane
