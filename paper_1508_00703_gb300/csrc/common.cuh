@@ -186,7 +186,10 @@ __device__ __forceinline__ float dev_expf(float x0)
     const int k2 = k - h;
     const float s1 = __int_as_float((h + 127) << 23);
     const float s2 = __int_as_float((k2 + 127) << 23);
-    const float e = __fmul_rn(__fmul_rn(p, s1), s2);
+    // with 0.7 < p < 1.5 and -125 <= k <= 127, p * 2^k is normal, so one exact
+    // scaling by 2^k equals the two-factor form (which the rest of the range needs)
+    const float sk = __int_as_float((k + 127) << 23);
+    const float e = k >= -125 && k <= 127 ? __fmul_rn(p, sk) : __fmul_rn(__fmul_rn(p, s1), s2);
     return x0 != x0 ? x0 : e;
 }
 
