@@ -27,6 +27,14 @@ import sys
 import tempfile
 import time
 
+# The end-to-end measurement runs four streams at once (compute, host-to-device
+# copies, device-to-host copies, the library's own stream for frees).  With the
+# default 8 hardware work queues per device some of them share a queue, and
+# work on one then waits behind a long copy on another; 32 queues keep them
+# apart.  Read when the CUDA context is created, so it is set before anything
+# imports torch.
+os.environ.setdefault("CUDA_DEVICE_MAX_CONNECTIONS", "32")
+
 ROOT = os.path.dirname(os.path.abspath(__file__))
 if ROOT not in sys.path:
     sys.path.insert(0, ROOT)

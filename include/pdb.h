@@ -41,6 +41,11 @@
  *     reuse (its release threshold is raised) until the process exits; the
  *     device's default pool and every other process-wide CUDA setting are left
  *     as they are.
+ *   - Host memory: a pinned, device-mapped slab of small words, one per
+ *     process (grown in slabs of 64 slots), holds each conflicts handle's info
+ *     words and stages pdb_status' read.  The library's kernels store those
+ *     words into it directly: a device-to-host copy of a few bytes would queue
+ *     behind the caller's large copies on the copy engine.
  *   - Diagnostics: every call opens an NVTX range named after it (seen by
  *     profilers); with the environment variable PDB_LOG set to anything but
  *     "" or "0" each call (but pdb_sgd_epoch_ready_noalloc) prints one line

@@ -574,18 +574,42 @@ void mark_use(const pdb_conflicts *c, const pdb_schedule *h, cudaStream_t s)
     if (h && h->ev_use) cudaEventRecord(h->ev_use, s);
 }
 
-// Small device-to-host reads of handle words.  A plain cudaMemcpy runs on the
-// legacy default stream, which waits for every blocking stream of the device
-// (another caller's copies, say); these reads go on the caller's stream, or,
-// where the call has none, on the library's own stream (own_stream).
-static int read_words(void *dst, const void *src, size_t bytes, cudaStream_t s)
+// Small device-to-host reads of handle words go on the caller's stream, or,
+// where the call has none, on the library's own stream (own_stream): a plain
+// cudaMemcpy runs on the legacy default stream, which waits for every
+// blocking stream of the device.  They are made by a one-block kernel that
+// stores the words into mapped pinned host memory, not by a copy: a
+// device-to-host copy of a few bytes queues behind whatever large copy the
+// caller has in flight on the same copy engine (a training loop's weights
+// going back to the host, say), and the read would wait for it.
+__global__ void k_copy_words(const uint32_t *__restrict__ src, uint32_t *__restrict__ dst, int n)
 {
-    if (cudaMemcpyAsync(dst, src, bytes, cudaMemcpyDeviceToHost, s) != cudaSuccess ||
-        cudaStreamSynchronize(s) != cudaSuccess) {
+    for (int i = threadIdx.x; i < n; i += blockDim.x) dst[i] = src[i];
+}
+
+static int copy_words_to_host(int *pinned, const void *src, size_t bytes, cudaStream_t s)
+{
+    int *dev = nullptr;
+    if (bytes % 4 != 0 || cudaHostGetDevicePointer((void **)&dev, pinned, 0) != cudaSuccess) {
         cudaGetLastError();
         return PDB_ECUDA;
     }
-    return PDB_OK;
+    k_copy_words<<<1, 128, 0, s>>>((const uint32_t *)src, (uint32_t *)dev, (int)(bytes / 4));
+    note_launch();
+    return cudaPeekAtLastError() == cudaSuccess ? PDB_OK : PDB_ECUDA;
+}
+
+static int read_words(void *dst, const void *src, size_t bytes, cudaStream_t s)
+{
+    if (bytes > sizeof(int) * INFO_WORDS) return PDB_EINVAL;
+    int *stage = info_slot_take();          // a pinned, mapped slot of the info slab
+    if (!stage) return PDB_ENOMEM;
+    int rc = copy_words_to_host(stage, src, bytes, s);
+    if (rc == PDB_OK && cudaStreamSynchronize(s) != cudaSuccess) rc = PDB_ECUDA;
+    if (rc == PDB_OK) std::memcpy(dst, stage, bytes);
+    cudaGetLastError();
+    info_slot_give(stage);
+    return rc;
 }
 
 static int read_words(void *dst, const void *src, size_t bytes)
@@ -602,7 +626,8 @@ int *info_slot_take()
     if (g_free_slots.empty()) {
         constexpr int SLOTS = 64;
         int *slab = nullptr;
-        if (cudaHostAlloc((void **)&slab, sizeof(int) * INFO_WORDS * SLOTS, cudaHostAllocDefault) != cudaSuccess) {
+        if (cudaHostAlloc((void **)&slab, sizeof(int) * INFO_WORDS * SLOTS, cudaHostAllocMapped | cudaHostAllocPortable) !=
+            cudaSuccess) {
             cudaGetLastError();
             return nullptr;
         }
@@ -777,7 +802,7 @@ int pdb_build_conflicts(const pdb_csr *X, pdb_conflicts **out, void *stream)
     release(skey, s);
     release(tkey, s);
     release(tval, s);
-    if (rc == PDB_OK) cudaMemcpyAsync(c->h_info, c->info, sizeof(int) * INFO_WORDS, cudaMemcpyDeviceToHost, s);
+    if (rc == PDB_OK) rc = copy_words_to_host(c->h_info, c->info, sizeof(int) * INFO_WORDS, s);
     cudaEventRecord(c->ev1, s);
     mark_use(c, nullptr, s);
     c->timed_build = true;
@@ -1022,9 +1047,10 @@ int pdb_get_stats(const pdb_conflicts *c, const pdb_schedule *h, pdb_stats *out)
     out->nnz = c->nnz;
     out->n_levels = -1;
     out->max_level_width = -1;
-    int info[INFO_WORDS] = {};
-    if (read_words(info, c->info, sizeof info) != PDB_OK) return PDB_ECUDA;
-    out->max_chain = info[INFO_MAX_CHAIN];
+    // the longest chain is final when the build ends, which copied its info
+    // words to the handle's pinned slot (complete once ev_use is): no device
+    // read, so nothing here waits for other streams' copies
+    out->max_chain = c->h_info[INFO_MAX_CHAIN];
     float ms = 0;
     if (c->timed_build && cudaEventElapsedTime(&ms, c->ev0, c->ev1) == cudaSuccess) out->ms_build = ms;
     if (c->timed_sgd && cudaEventElapsedTime(&ms, c->ev_sgd0, c->ev_sgd1) == cudaSuccess) out->ms_sgd = ms;
