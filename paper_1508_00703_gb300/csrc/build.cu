@@ -587,6 +587,22 @@ __global__ void k_copy_words(const uint32_t *__restrict__ src, uint32_t *__restr
     for (int i = threadIdx.x; i < n; i += blockDim.x) dst[i] = src[i];
 }
 
+__global__ void k_fill_words(uint32_t *__restrict__ p, uint32_t v, int64_t n)
+{
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x)
+        p[i] = v;
+}
+
+int fill_words(void *p, uint32_t v, size_t bytes, cudaStream_t s)
+{
+    if (bytes % 4 != 0) return PDB_EINVAL;
+    const int64_t n = (int64_t)(bytes / 4);
+    if (n == 0) return PDB_OK;
+    k_fill_words<<<grid_1d(n), 256, 0, s>>>((uint32_t *)p, v, n);
+    note_launch();
+    return cudaPeekAtLastError() == cudaSuccess ? PDB_OK : PDB_ECUDA;
+}
+
 static int copy_words_to_host(int *pinned, const void *src, size_t bytes, cudaStream_t s)
 {
     int *dev = nullptr;
@@ -773,7 +789,7 @@ int pdb_build_conflicts(const pdb_csr *X, pdb_conflicts **out, void *stream)
     } else {
         rc = rc ? rc : alloc((void **)&c->gate_sorted, sizeof(uint32_t) * nnz, s);
         rc = rc ? rc : alloc((void **)&c->gate_window, sizeof(uint32_t) * nnz, s);
-        if (rc == PDB_OK) cudaMemsetAsync(c->gate_window, 0, sizeof(uint32_t) * nnz, s);
+        if (rc == PDB_OK) rc = fill_words(c->gate_window, 0u, sizeof(uint32_t) * nnz, s);
     }
     rc = rc ? rc : alloc((void **)&c->feat_ptr, sizeof(int64_t) * (F + 1), s);
     uint32_t *skey = nullptr, *tkey = nullptr;
@@ -783,13 +799,13 @@ int pdb_build_conflicts(const pdb_csr *X, pdb_conflicts **out, void *stream)
     rc = rc ? rc : alloc((void **)&tval, sizeof(int32_t) * nnz, s);
     c->status = c->info;
     if (rc == PDB_OK) {
-        cudaMemsetAsync(c->info, 0, sizeof(int) * INFO_WORDS, s);
+        rc = fill_words(c->info, 0u, sizeof(int) * INFO_WORDS, s);
         k_validate_rows<<<grid_1d(N + 1), 256, 0, s>>>(X->row_ptr, X->col, N, nnz, c->info);
         note_launch();
         // (feature, position) pairs sorted by feature, stable: positions stay in data order.
         // The sort's first read of the ids also checks that they lie in [0, n_cols)
         // (PDB_ERANGE) and counts the descents.
-        rc = radix_sort((const uint32_t *)X->col, nullptr, skey, c->csc_pos, tkey, tval, nnz,
+        rc = rc ? rc : radix_sort((const uint32_t *)X->col, nullptr, skey, c->csc_pos, tkey, tval, nnz,
                         bits_for(F > 0 ? F - 1 : 0), c->info, s, (uint32_t)F, c->info + INFO_DESC_ALL);
     }
     if (rc == PDB_OK) rc = segment_bounds(skey, nnz, F, nullptr, c->feat_ptr, c->info, s);
@@ -893,8 +909,8 @@ int pdb_schedule_build(const pdb_conflicts *c, pdb_sched_mode mode, pdb_schedule
     int rc = alloc((void **)&h->bar, sizeof(GridBarrier), s);
     rc = rc ? rc : alloc((void **)&h->ticket, sizeof(unsigned long long), s);
     if (rc == PDB_OK) {
-        cudaMemsetAsync(h->bar, 0, sizeof(GridBarrier), s);
-        cudaMemsetAsync(h->ticket, 0, sizeof(unsigned long long), s);
+        rc = fill_words(h->bar, 0u, sizeof(GridBarrier), s);
+        rc = rc ? rc : fill_words(h->ticket, 0u, sizeof(unsigned long long), s);
     }
     if (mode == PDB_SCHED_READY) {
         // one (weight, version) record per feature; filled from w by pdb_sgd_epoch;
@@ -908,9 +924,9 @@ int pdb_schedule_build(const pdb_conflicts *c, pdb_sched_mode mode, pdb_schedule
         // epoch)
         h->prog_cap = (std::max<int64_t>(N, 1) + 3) & ~(int64_t)3;   // the sweeper reads four flags at a time
         rc = rc ? rc : alloc((void **)&h->rec, sizeof(unsigned long long) * std::max<int64_t>(F, 1), s);
-        if (rc == PDB_OK) cudaMemsetAsync(h->rec, 0, sizeof(unsigned long long) * std::max<int64_t>(F, 1), s);
+        if (rc == PDB_OK) rc = fill_words(h->rec, 0u, sizeof(unsigned long long) * std::max<int64_t>(F, 1), s);
         rc = rc ? rc : alloc((void **)&h->prog, sizeof(unsigned) * h->prog_cap, s);
-        if (rc == PDB_OK) cudaMemsetAsync(h->prog, 0, sizeof(unsigned) * h->prog_cap, s);
+        if (rc == PDB_OK) rc = fill_words(h->prog, 0u, sizeof(unsigned) * h->prog_cap, s);
         rc = rc ? rc : alloc((void **)&h->wctl, sizeof(WindowCtl), s);
     } else if (mode == PDB_SCHED_CHAIN) {
         // rows longer than the forwarding engine takes: weights resident in

@@ -383,6 +383,9 @@ struct UseMark {
 };
 // host-side pinned words for a conflicts handle's info copy, from a slab that
 // is kept for the process (freeing pinned memory would synchronize the device)
+// fill bytes / 4 words at p with v on s by a kernel (a memset may run on a
+// copy engine and queue behind the caller's copies); bytes a multiple of 4
+int fill_words(void *p, uint32_t v, size_t bytes, cudaStream_t s);
 int *info_slot_take();
 void info_slot_give(int *slot);
 

@@ -413,8 +413,9 @@ int window_run(const pdb_csr *X, const float *y, const uint32_t *gate, float *w,
         const unsigned count = (*epoch_count)++;
         const unsigned stamp = (1u + count % 7u) << 29;
         const unsigned tag = count % 0xffffffffu + 1u;
-        if (tag == 1u && count != 0) cudaMemsetAsync(done, 0, sizeof(unsigned) * (size_t)done_cap, s);
-        cudaMemsetAsync(ctl, 0, sizeof(WindowCtl), s);
+        if (tag == 1u && count != 0 && fill_words(done, 0u, sizeof(unsigned) * (size_t)done_cap, s) != PDB_OK)
+            return PDB_ECUDA;
+        if (fill_words(ctl, 0u, sizeof(WindowCtl), s) != PDB_OK) return PDB_ECUDA;
         kern<<<grid, THREADS, 0, s>>>(n, X->row_ptr, X->col, X->val, y, gate, w, rec, stamp, done, tag, ctl, near,
                                       loss, eta, chunk, status, timeout, opts ? opts->trace : nullptr,
                                       (int64_t)ep * X->n_rows);
