@@ -968,13 +968,13 @@ int pdb_schedule_build(const pdb_conflicts *c, pdb_sched_mode mode, pdb_schedule
         rc = rc ? rc : alloc((void **)&tkey, sizeof(uint32_t) * N, s);
         rc = rc ? rc : alloc((void **)&tval, sizeof(int32_t) * N, s);
         if (rc == PDB_OK) {
-            cudaMemsetAsync(h->ctl, 0, sizeof(LevelCtl), s);
+            rc = rc ? rc : fill_words(h->ctl, 0u, sizeof(LevelCtl), s);
             if (N > 0) {
                 int32_t n32 = (int32_t)N;
                 uint64_t tmo = timeout_ns(nullptr);
                 if (flow) {
-                    cudaMemsetAsync(h->level, 0xff, sizeof(int32_t) * N, s);
-                    cudaMemsetAsync(h->ticket, 0, sizeof(unsigned long long), s);
+                    rc = fill_words(h->level, 0xffffffffu, sizeof(int32_t) * N, s);
+                    rc = rc ? rc : fill_words(h->ticket, 0u, sizeof(unsigned long long), s);
                     const int grid = persistent_grid((const void *)k_levels_flow, nullptr);
                     k_levels_flow<<<grid, THREADS, 0, s>>>(n32, c->row_ptr, c->prev, c->row_of, h->level, h->ticket, 4,
                                                            c->status, tmo);
@@ -1003,7 +1003,7 @@ int pdb_schedule_build(const pdb_conflicts *c, pdb_sched_mode mode, pdb_schedule
                     note_launch();
                 }
             } else {
-                cudaMemsetAsync(h->level_ptr, 0, sizeof(int64_t), s);
+                rc = rc ? rc : fill_words(h->level_ptr, 0u, sizeof(int64_t), s);
             }
         }
         release(key, s);

@@ -659,8 +659,8 @@ int pdb_sgd_epoch(const pdb_csr *X, const float *y, const pdb_conflicts *c, cons
             const int chunk = (opts && opts->ticket_chunk > 0) ? opts->ticket_chunk : 2;
             k_pack<<<grid_1d(F), 256, 0, s>>>(w, F, h->rec, cm->status);
             note_launch();
+            if (fill_words(h->ticket, 0u, sizeof(unsigned long long), s) != PDB_OK) return PDB_ECUDA;
             cudaEventRecord(cm->ev_k0, s);
-            cudaMemsetAsync(h->ticket, 0, sizeof(unsigned long long), s);
             kern<<<grid, THREADS, 0, s>>>(n32, X->row_ptr, X->col, X->val, y, c->gate, h->rec, lossi, eta, n_epochs,
                                           h->ticket, chunk, cm->status, tmo, trace);
             note_launch();
@@ -777,8 +777,8 @@ int pdb_bsp_epoch(const pdb_csr *X, const float *y, const pdb_conflicts *c, floa
         rc = rc ? rc : alloc((void **)&bptr, sizeof(int64_t) * (n_batches + 1), s);
         rc = rc ? rc : alloc((void **)&bar, sizeof(GridBarrier), s);
         if (rc == PDB_OK) {
-            cudaMemsetAsync(bar, 0, sizeof(GridBarrier), s);
-            if (nnz > 0) rc = ensure_row_of(cm, s);
+            rc = fill_words(bar, 0u, sizeof(GridBarrier), s);
+            if (rc == PDB_OK && nnz > 0) rc = ensure_row_of(cm, s);
             if (rc == PDB_OK && nnz > 0) {
                 k_bsp_keys<<<grid_1d(nnz), 256, 0, s>>>(c->csc_pos, c->row_of, nnz, batch, key, cm->status); note_launch();
                 // stable by batch: inside a batch the feature-major CSC order survives
@@ -866,7 +866,7 @@ int pdb_bsp_plan_build(const pdb_conflicts *c, int64_t batch, pdb_bsp_plan **out
             rc = segment_bounds(skey, nnz, p->n_batches, nullptr, p->bptr, cm->status, s);
         }
     } else if (rc == PDB_OK) {
-        cudaMemsetAsync(p->bptr, 0, sizeof(int64_t) * (p->n_batches + 1), s);
+        rc = fill_words(p->bptr, 0u, sizeof(int64_t) * (p->n_batches + 1), s);
     }
     for (void *q : {(void *)key, (void *)skey, (void *)tkey, (void *)bpos, (void *)tval}) release(q, s);
     if (rc == PDB_OK && cudaPeekAtLastError() != cudaSuccess) rc = PDB_ECUDA;
@@ -1055,7 +1055,7 @@ extern "C" int pdb_sgd_epoch_ready_noalloc(const pdb_csr *X, const float *y, con
     int *status = (int *)(scratch + NOALLOC_MAX_COLS + 1);
     cudaStream_t s = (cudaStream_t)stream;
     // the previous call left its status and ticket behind: start from zero
-    if (cudaMemsetAsync(status, 0, sizeof(int), s) != cudaSuccess) return PDB_ECUDA;
+    if (fill_words(status, 0u, sizeof(int), s) != PDB_OK) return PDB_ECUDA;
     if (X->n_rows > 0 && n_epochs > 0) {
         const int64_t F = X->n_cols;
         const int32_t n32 = (int32_t)X->n_rows;
@@ -1065,7 +1065,7 @@ extern "C" int pdb_sgd_epoch_ready_noalloc(const pdb_csr *X, const float *y, con
             k_pack<<<grid_1d(F), 256, 0, s>>>(w, F, rec, status);
             note_launch();
         }
-        cudaMemsetAsync(ticket, 0, sizeof(unsigned long long), s);
+        if (fill_words(ticket, 0u, sizeof(unsigned long long), s) != PDB_OK) return PDB_ECUDA;
         k_sgd_ready<8><<<grid, THREADS, 0, s>>>(n32, X->row_ptr, X->col, X->val, y, gate, rec, (int)loss, eta,
                                                 n_epochs, ticket, 2, status, tmo, nullptr);
         note_launch();

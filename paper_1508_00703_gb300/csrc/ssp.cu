@@ -304,13 +304,14 @@ int ssp_run(const pdb_csr *X, const float *y, const uint32_t *gate, float *w, un
                        : (width == 2 ? k_sgd_ssp<2, false> : width == 4 ? k_sgd_ssp<4, false> : k_sgd_ssp<8, false>);
     const int grid = persistent_grid((const void *)kern, opts);
     for (int ep = 0; ep < n_epochs; ++ep) {
-        cudaMemsetAsync(writes, 0, sizeof(unsigned) * (size_t)F, s);
-        cudaMemsetAsync(reads, 0, sizeof(unsigned) * (size_t)F, s);
+        int rc = fill_words(writes, 0u, sizeof(unsigned) * (size_t)F, s);
+        rc = rc ? rc : fill_words(reads, 0u, sizeof(unsigned) * (size_t)F, s);
         if (prefix) {
-            cudaMemsetAsync(rbits, 0, sizeof(unsigned) * (size_t)n_words, s);
-            cudaMemsetAsync(wbits, 0, sizeof(unsigned) * (size_t)n_words, s);
+            rc = rc ? rc : fill_words(rbits, 0u, sizeof(unsigned) * (size_t)n_words, s);
+            rc = rc ? rc : fill_words(wbits, 0u, sizeof(unsigned) * (size_t)n_words, s);
         }
-        cudaMemsetAsync(ticket, 0, sizeof(unsigned long long), s);
+        rc = rc ? rc : fill_words(ticket, 0u, sizeof(unsigned long long), s);
+        if (rc != PDB_OK) return rc;
         kern<<<grid, THREADS, 0, s>>>(n, X->row_ptr, X->col, X->val, y, gate, w, writes, reads, delay,
                                       coef ? coef + (int64_t)ep * n : nullptr, loss, eta, ticket, chunk, status,
                                       timeout, opts ? opts->trace : nullptr, (int64_t)ep * n, feat_ptr, rbits, wbits);
