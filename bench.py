@@ -427,11 +427,12 @@ def run_ours(args, rank, world, local_rank):
 def run_e2e(args, p, mode, pdb, torch, world):
     """Same metric through the public API from pinned host buffers: every
     step copies its inputs host-to-device and reads the trained weights back,
-    inside the timed region.  The copies of step i+1 run on a copy stream
-    into a second set of device buffers while step i computes, and step i's
-    weights go back to the host on a third stream while step i+1 computes (a
-    double-buffered input pipeline, as a training loop that streams its data
-    would run it)."""
+    inside the timed region.  The inputs of steps i+1 and i+2 copy on a copy
+    stream into two more sets of device buffers while step i computes, and
+    step i's weights go back to the host on a third stream while step i+1
+    computes (an input pipeline two steps deep, as a training loop that
+    streams its data would run it: one copy slowed by the host link then
+    delays no step by itself)."""
     # a stream of its own for the compute: the legacy default stream would order
     # itself against the copy streams
     main = torch.cuda.Stream()
@@ -440,7 +441,8 @@ def run_e2e(args, p, mode, pdb, torch, world):
     h_val = None if p.val is None else torch.from_numpy(p.val).pin_memory()
     h_y = torch.from_numpy(p.y).pin_memory()
     h_w0 = torch.zeros(p.n_cols, dtype=torch.float32).pin_memory()
-    h_w = [torch.empty(p.n_cols, dtype=torch.float32).pin_memory() for _ in range(2)]
+    DEPTH = 3                                   # sets of device buffers: step i and the inputs of i+1, i+2
+    h_w = [torch.empty(p.n_cols, dtype=torch.float32).pin_memory() for _ in range(DEPTH)]
     h2d = sum(t.numel() * t.element_size() for t in (h_row, h_col, h_val, h_y, h_w0) if t is not None)
     d2h = h_w[0].numel() * h_w[0].element_size()
 
@@ -458,12 +460,12 @@ def run_e2e(args, p, mode, pdb, torch, world):
             self.done.record(main)
             self.read.record(main)
 
-    bufs = [Buffers(), Buffers()]
+    bufs = [Buffers() for _ in range(DEPTH)]
     copy_in, copy_out = torch.cuda.Stream(), torch.cuda.Stream()
 
     def stage(i):
-        b = bufs[i % 2]
-        copy_in.wait_event(b.done)            # step i-2 no longer reads these inputs
+        b = bufs[i % DEPTH]
+        copy_in.wait_event(b.done)            # step i-DEPTH no longer reads these inputs
         copy_in.wait_event(b.read)            # and its weights have left the device
         with torch.cuda.stream(copy_in):
             for d, h in ((b.row, h_row), (b.col, h_col), (b.val, h_val), (b.y, h_y), (b.w, h_w0)):
@@ -472,7 +474,7 @@ def run_e2e(args, p, mode, pdb, torch, world):
             b.copied.record(copy_in)
 
     def compute(i):
-        b = bufs[i % 2]
+        b = bufs[i % DEPTH]
         main.wait_event(b.copied)
         c = pdb.pdb_build_conflicts(b.X, main)
         s = pdb.pdb_schedule_build(c, mode, main)
@@ -481,17 +483,18 @@ def run_e2e(args, p, mode, pdb, torch, world):
         b.done.record(main)
         copy_out.wait_event(b.done)
         with torch.cuda.stream(copy_out):
-            h_w[i % 2].copy_(b.w, non_blocking=True)
+            h_w[i % DEPTH].copy_(b.w, non_blocking=True)
             b.read.record(copy_out)
         return c, s
 
     phases = []
 
     def run(steps):
-        stage(0)
+        for i in range(min(DEPTH - 1, steps)):
+            stage(i)
         for i in range(steps):
-            if i + 1 < steps:
-                stage(i + 1)
+            if i + DEPTH - 1 < steps:
+                stage(i + DEPTH - 1)
             c, s = compute(i)
             rc = pdb.pdb_status(c, main)        # synchronizes main: step i's kernels are done
             if rc != 0:
@@ -529,7 +532,7 @@ def run_e2e(args, p, mode, pdb, torch, world):
             "ms_per_step": dt * 1e3, "steps": steps, "host_link": link,
             "device_phases_ms": {"build_conflicts": statistics.median(ph["ms_build"] for ph in phases),
                                  "sgd_all_epochs": statistics.median(ph["ms_sgd"] for ph in phases)},
-            "pipeline": "step i+1's H2D on a copy stream and step i's D2H on another, overlapping the next step"}
+            "pipeline": "steps i+1 and i+2's H2D on a copy stream and step i's D2H on another, overlapping the next step"}
 
 
 # ---------------------------------------------------------------- reference arm: the CPU oracle
