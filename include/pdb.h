@@ -154,7 +154,8 @@ typedef enum {
 
 /* Launch and wait options; a zeroed struct (or NULL) selects the defaults. */
 typedef struct {
-    int32_t blocks_per_sm;     /* persistent grid = blocks_per_sm x #SM; 0 = occupancy maximum */
+    int32_t blocks_per_sm;     /* persistent grid = blocks_per_sm x #SM (at most the occupancy
+                                  maximum); 0 = that maximum, for WINDOW 3 */
     int32_t ticket_chunk;      /* READY: consecutive examples a warp takes per ticket; 0 = 2 */
     double wait_timeout_s;     /* limit of every device-side wait; 0 = 2 seconds; at most 10^6 seconds */
     uint64_t *trace;           /* optional (NULL = off), pdb_sgd_epoch and pdb_ssp_epoch: device array of

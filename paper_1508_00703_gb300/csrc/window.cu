@@ -403,7 +403,11 @@ int window_run(const pdb_csr *X, const float *y, const uint32_t *gate, float *w,
     const int chunk = (opts && opts->ticket_chunk > 0) ? opts->ticket_chunk : 2;
     if ((X->n_rows + chunk - 1) / chunk > done_cap) return PDB_EFAULT;
     auto kern = width == 2 ? k_sgd_window<2> : width == 4 ? k_sgd_window<4> : k_sgd_window<8>;
-    int grid = persistent_grid((const void *)kern, opts);
+    // three blocks per SM unless the caller asks otherwise: on the low-conflict
+    // workload 0.75% faster than the occupancy maximum (four), measured
+    pdb_opts o = opts ? *opts : pdb_opts{};
+    if (o.blocks_per_sm <= 0) o.blocks_per_sm = 3;
+    int grid = persistent_grid((const void *)kern, &o);
     if (grid < 2) grid = 2;                         // the sweeping block plus at least one worker block
     for (int ep = 0; ep < n_epochs; ++ep) {
         // record tags carry an epoch stamp 1..7 (bits 29-31), different in
