@@ -114,15 +114,46 @@ __device__ __forceinline__ int64_t find_row(const int64_t *__restrict__ row_ptr,
     return lo;
 }
 
+// The first slot of the run of key skey[q] (keys sorted): a gallop back from
+// q, then a binary search in the last interval -- about 2 log2 of the run's
+// length loads, once per warp
+__device__ int64_t run_start(const uint32_t *__restrict__ skey, int64_t q)
+{
+    const uint32_t j = skey[q];
+    int64_t hi = q, lo = q - 1, step = 1;          // skey[hi] == j
+    while (lo >= 0 && skey[lo] == j) {
+        hi = lo;
+        step <<= 1;
+        lo = hi - step;
+    }
+    if (lo < -1) lo = -1;                          // skey[lo] < j, or lo = -1
+    while (hi - lo > 1) {
+        const int64_t mid = lo + ((hi - lo) >> 1);
+        if (skey[mid] == j)
+            hi = mid;
+        else
+            lo = mid;
+    }
+    return hi;
+}
+
 // Slot order: the gate word of every slot, rank | last-occurrence bit, the
-// longest chain, and -- only when some row is unsorted -- the repeated-id
+// longest chain, feat_ptr (feat_ptr[b] = the first slot whose key is >= b,
+// b = 0..n_cols) and -- only when some row is unsorted -- the repeated-id
 // check: two neighbouring slots of one feature in the same example.  The
 // gate words go to position order either directly (gate[csc_pos[s]], one
 // scattered 4-byte store per slot) or, for large inputs, in slot order
 // (gsort[s]) for the partitioned scatter below.
+//
+// Each warp takes a contiguous range of slots, 128 per step (four per lane,
+// 16-byte loads and stores; the buffers come from the pool, 256-byte
+// aligned), and carries the first slot of the run in progress from one step
+// to the next, so a slot's rank is its distance to that slot without a
+// second pass over the keys; the run in progress where the range begins is
+// found once per warp by run_start.
 __global__ void k_slots(const uint32_t *__restrict__ skey, const int32_t *__restrict__ spos, int64_t nnz,
-                        const int64_t *__restrict__ feat_ptr, const int64_t *__restrict__ row_ptr, int64_t n_rows,
-                        int64_t near, uint32_t *__restrict__ gate, uint32_t *__restrict__ gsort,
+                        int64_t n_cols, int64_t *__restrict__ feat_ptr, const int64_t *__restrict__ row_ptr,
+                        int64_t n_rows, int64_t near, uint32_t *__restrict__ gate, uint32_t *__restrict__ gsort,
                         uint32_t *__restrict__ gwin, int *info)
 {
     __shared__ bool s_check;
@@ -137,14 +168,19 @@ __global__ void k_slots(const uint32_t *__restrict__ skey, const int32_t *__rest
     __syncthreads();
     if (read_status(info)) return;
     const bool check_dup = s_check;
+    const int lane = threadIdx.x & 31;
+    const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const int64_t n_warps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    const int64_t steps = (nnz + 127) >> 7;
+    const int64_t per = (steps + n_warps - 1) / n_warps;
+    const int64_t st0 = warp * per, st1 = min(steps, st0 + per);
+    int64_t carry = 0;                             // first slot of the run holding the slot before the step
+    if (st0 < st1 && st0 > 0 && lane == 0) carry = run_start(skey, (st0 << 7) - 1);
+    carry = __shfl_sync(FULL, carry, 0);
     int longest = 0, n_near = 0;
     bool dup = false, big = false;
-    // four consecutive slots per thread and iteration (16-byte loads and
-    // stores; the buffers come from the pool, 256-byte aligned), with the
-    // neighbours on both sides
-    const int64_t groups = (nnz + 3) >> 2;
-    for (int64_t gi = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; gi < groups;
-         gi += (int64_t)gridDim.x * blockDim.x) {
+    for (int64_t st = st0; st < st1; ++st) {
+        const int64_t gi = (st << 5) + lane;
         const int64_t s0 = gi << 2;
         uint32_t kk[6];
         int32_t pp[6];
@@ -160,10 +196,39 @@ __global__ void k_slots(const uint32_t *__restrict__ skey, const int32_t *__rest
                 pp[e + 1] = s0 + e < nnz ? spos[s0 + e] : 0;
             }
         }
-        kk[0] = s0 > 0 ? skey[s0 - 1] : 0xffffffffu;
-        pp[0] = s0 > 0 ? spos[s0 - 1] : 0;
-        kk[5] = s0 + 4 < nnz ? skey[s0 + 4] : 0xffffffffu;
-        pp[5] = s0 + 4 < nnz ? spos[s0 + 4] : 0;
+        // the neighbouring slots come from the lanes beside; the step's two
+        // ends from memory (0xffffffff past either end of the keys)
+        kk[0] = __shfl_up_sync(FULL, kk[4], 1);
+        pp[0] = __shfl_up_sync(FULL, pp[4], 1);
+        kk[5] = __shfl_down_sync(FULL, kk[1], 1);
+        pp[5] = __shfl_down_sync(FULL, pp[1], 1);
+        if (lane == 0) {
+            kk[0] = s0 > 0 ? skey[s0 - 1] : 0xffffffffu;
+            pp[0] = s0 > 0 ? spos[s0 - 1] : 0;
+        }
+        if (lane == 31) {
+            kk[5] = s0 + 4 < nnz ? skey[s0 + 4] : 0xffffffffu;
+            pp[5] = s0 + 4 < nnz ? spos[s0 + 4] : 0;
+        }
+        // the last run start among this lane's slots (offset in the step, -1
+        // for none), its running maximum over the lanes, and from that the
+        // first slot of the run that holds the slot before this lane's first
+        int ls = -1;
+#pragma unroll
+        for (int e = 0; e < 4; ++e)
+            if (s0 + e < nnz && kk[e] != kk[e + 1]) ls = lane * 4 + e;
+        int inc = ls;
+#pragma unroll
+        for (int d = 1; d < 32; d <<= 1) {
+            const int t = __shfl_up_sync(FULL, inc, d);
+            if (lane >= d) inc = max(inc, t);
+        }
+        int exc = __shfl_up_sync(FULL, inc, 1);
+        if (lane == 0) exc = -1;
+        const int64_t base = st << 7;
+        const int64_t before = exc >= 0 ? base + exc : carry;
+        const int last_start = __shfl_sync(FULL, inc, 31);
+        if (last_start >= 0) carry = base + last_start;
         uint32_t g[4] = {0u, 0u, 0u, 0u};
         int64_t r = 0;
 #pragma unroll
@@ -172,11 +237,18 @@ __global__ void k_slots(const uint32_t *__restrict__ skey, const int32_t *__rest
             if (s >= nnz) break;
             const uint32_t j = kk[e + 1];
             const int32_t p = pp[e + 1];
+            const bool first = kk[e] != j;
             const bool last = s == nnz - 1 || kk[e + 2] != j;
-            // rank: 0 where the feature's run starts, one more than the slot before
-            // inside the group, and from the run's first slot (feat_ptr) only for a
-            // run that began before this group
-            r = kk[e] != j ? 0 : e > 0 ? r + 1 : s - feat_ptr[j];
+            // rank: 0 where the feature's run starts, one more than the slot
+            // before inside the lane's slots, else the distance to the run's
+            // first slot
+            r = first ? 0 : e > 0 ? r + 1 : s - before;
+            if (first) {
+                const int64_t hi = min((int64_t)j, n_cols);
+                for (int64_t b = s == 0 ? 0 : (int64_t)kk[e] + 1; b <= hi; ++b) feat_ptr[b] = s;
+            }
+            if (s == nnz - 1)
+                for (int64_t b = (int64_t)j + 1; b <= n_cols; ++b) feat_ptr[b] = nnz;
             const bool near_prev = r > 0 && (int64_t)p - pp[e] < near;
             const bool near_next = !last && (int64_t)pp[e + 2] - p < near;
             big |= r > (int64_t)GATE_RANK;
@@ -199,10 +271,10 @@ __global__ void k_slots(const uint32_t *__restrict__ skey, const int32_t *__rest
         longest = max(longest, __shfl_xor_sync(FULL, longest, off));
         n_near += __shfl_xor_sync(FULL, n_near, off);
     }
-    if ((threadIdx.x & 31) == 0 && longest > 0) atomicMax(info + INFO_MAX_CHAIN, longest);
-    if ((threadIdx.x & 31) == 0 && n_near > 0) atomicAdd(info + INFO_NEAR, n_near);
-    if (__any_sync(FULL, dup) && (threadIdx.x & 31) == 0) set_status(info, PDB_EDUP);
-    if (__any_sync(FULL, big) && (threadIdx.x & 31) == 0) set_status(info, PDB_ETOOBIG);
+    if (lane == 0 && longest > 0) atomicMax(info + INFO_MAX_CHAIN, longest);
+    if (lane == 0 && n_near > 0) atomicAdd(info + INFO_NEAR, n_near);
+    if (__any_sync(FULL, dup) && lane == 0) set_status(info, PDB_EDUP);
+    if (__any_sync(FULL, big) && lane == 0) set_status(info, PDB_ETOOBIG);
 }
 
 // Last step of the gate scatter for large inputs.  The (position, gate)
@@ -808,11 +880,12 @@ int pdb_build_conflicts(const pdb_csr *X, pdb_conflicts **out, void *stream)
         rc = rc ? rc : radix_sort((const uint32_t *)X->col, nullptr, skey, c->csc_pos, tkey, tval, nnz,
                         bits_for(F > 0 ? F - 1 : 0), c->info, s, (uint32_t)F, c->info + INFO_DESC_ALL);
     }
-    if (rc == PDB_OK) rc = segment_bounds(skey, nnz, F, nullptr, c->feat_ptr, c->info, s);
+    // k_slots writes feat_ptr; with no nonzeros every bound is 0
+    if (rc == PDB_OK && nnz == 0) rc = segment_bounds(skey, 0, F, nullptr, c->feat_ptr, c->info, s);
     if (rc == PDB_OK && nnz > 0) {
-        k_slots<<<grid_1d((nnz + 3) / 4), 256, 0, s>>>(skey, c->csc_pos, nnz, c->feat_ptr, X->row_ptr, N, c->near,
-                                                        c->gate, c->gate_sorted, partition ? c->gate_window : nullptr,
-                                                        c->info);
+        k_slots<<<grid_1d((nnz + 3) / 4), 256, 0, s>>>(skey, c->csc_pos, nnz, F, c->feat_ptr, X->row_ptr, N,
+                                                        c->near, c->gate, c->gate_sorted,
+                                                        partition ? c->gate_window : nullptr, c->info);
         note_launch();
     }
     release(skey, s);
