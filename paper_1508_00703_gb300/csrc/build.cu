@@ -137,6 +137,27 @@ __device__ int64_t run_start(const uint32_t *__restrict__ skey, int64_t q)
     return hi;
 }
 
+// slots 4 gi .. 4 gi + 3 of the sorted keys and positions (0xffffffff and 0
+// past the end); 16-byte loads where the group is whole
+__device__ __forceinline__ void load_group(const uint32_t *__restrict__ skey, const int32_t *__restrict__ spos,
+                                           int64_t nnz, int64_t gi, uint4 &k4, int4 &p4)
+{
+    const int64_t s0 = gi << 2;
+    if (s0 + 4 <= nnz) {
+        k4 = __ldcs(reinterpret_cast<const uint4 *>(skey) + gi);
+        p4 = __ldcs(reinterpret_cast<const int4 *>(spos) + gi);
+    } else {
+        k4.x = s0 < nnz ? skey[s0] : 0xffffffffu;
+        k4.y = s0 + 1 < nnz ? skey[s0 + 1] : 0xffffffffu;
+        k4.z = s0 + 2 < nnz ? skey[s0 + 2] : 0xffffffffu;
+        k4.w = s0 + 3 < nnz ? skey[s0 + 3] : 0xffffffffu;
+        p4.x = s0 < nnz ? spos[s0] : 0;
+        p4.y = s0 + 1 < nnz ? spos[s0 + 1] : 0;
+        p4.z = s0 + 2 < nnz ? spos[s0 + 2] : 0;
+        p4.w = s0 + 3 < nnz ? spos[s0 + 3] : 0;
+    }
+}
+
 // Slot order: the gate word of every slot, rank | last-occurrence bit, the
 // longest chain, feat_ptr (feat_ptr[b] = the first slot whose key is >= b,
 // b = 0..n_cols) and -- only when some row is unsorted -- the repeated-id
@@ -177,6 +198,25 @@ __global__ void k_slots(const uint32_t *__restrict__ skey, const int32_t *__rest
     int64_t carry = 0;                             // first slot of the run holding the slot before the step
     if (st0 < st1 && st0 > 0 && lane == 0) carry = run_start(skey, (st0 << 7) - 1);
     carry = __shfl_sync(FULL, carry, 0);
+    // each step's keys and positions are loaded one step ahead, with the slot
+    // after the step (lane 31); the slot before it is the last one of the step
+    // before (lane 0), loaded only for the first step
+    uint4 nk = make_uint4(0xffffffffu, 0xffffffffu, 0xffffffffu, 0xffffffffu);
+    int4 np = make_int4(0, 0, 0, 0);
+    uint32_t nke = 0xffffffffu, lk = 0xffffffffu;
+    int32_t npe = 0, lp = 0;
+    if (st0 < st1) {
+        load_group(skey, spos, nnz, (st0 << 5) + lane, nk, np);
+        const int64_t e = (st0 + 1) << 7;
+        if (lane == 31 && e < nnz) {
+            nke = skey[e];
+            npe = spos[e];
+        }
+        if (lane == 0 && st0 > 0) {
+            lk = skey[(st0 << 7) - 1];
+            lp = spos[(st0 << 7) - 1];
+        }
+    }
     int longest = 0, n_near = 0;
     bool dup = false, big = false;
     for (int64_t st = st0; st < st1; ++st) {
@@ -184,32 +224,36 @@ __global__ void k_slots(const uint32_t *__restrict__ skey, const int32_t *__rest
         const int64_t s0 = gi << 2;
         uint32_t kk[6];
         int32_t pp[6];
-        if (s0 + 4 <= nnz) {
-            const uint4 k4 = __ldcs(reinterpret_cast<const uint4 *>(skey) + gi);
-            const int4 p4 = __ldcs(reinterpret_cast<const int4 *>(spos) + gi);
-            kk[1] = k4.x; kk[2] = k4.y; kk[3] = k4.z; kk[4] = k4.w;
-            pp[1] = p4.x; pp[2] = p4.y; pp[3] = p4.z; pp[4] = p4.w;
-        } else {
-#pragma unroll
-            for (int e = 0; e < 4; ++e) {
-                kk[e + 1] = s0 + e < nnz ? skey[s0 + e] : 0xffffffffu;
-                pp[e + 1] = s0 + e < nnz ? spos[s0 + e] : 0;
+        kk[1] = nk.x; kk[2] = nk.y; kk[3] = nk.z; kk[4] = nk.w;
+        pp[1] = np.x; pp[2] = np.y; pp[3] = np.z; pp[4] = np.w;
+        const uint32_t ke = nke;
+        const int32_t pe = npe;
+        if (st + 1 < st1) {
+            load_group(skey, spos, nnz, gi + 32, nk, np);
+            const int64_t e = (st + 2) << 7;
+            nke = 0xffffffffu;
+            npe = 0;
+            if (lane == 31 && e < nnz) {
+                nke = skey[e];
+                npe = spos[e];
             }
         }
-        // the neighbouring slots come from the lanes beside; the step's two
-        // ends from memory (0xffffffff past either end of the keys)
+        // the neighbouring slots come from the lanes beside, the step's two
+        // ends from the loads above (0xffffffff past either end of the keys)
         kk[0] = __shfl_up_sync(FULL, kk[4], 1);
         pp[0] = __shfl_up_sync(FULL, pp[4], 1);
         kk[5] = __shfl_down_sync(FULL, kk[1], 1);
         pp[5] = __shfl_down_sync(FULL, pp[1], 1);
         if (lane == 0) {
-            kk[0] = s0 > 0 ? skey[s0 - 1] : 0xffffffffu;
-            pp[0] = s0 > 0 ? spos[s0 - 1] : 0;
+            kk[0] = lk;
+            pp[0] = lp;
         }
         if (lane == 31) {
-            kk[5] = s0 + 4 < nnz ? skey[s0 + 4] : 0xffffffffu;
-            pp[5] = s0 + 4 < nnz ? spos[s0 + 4] : 0;
+            kk[5] = ke;
+            pp[5] = pe;
         }
+        lk = __shfl_sync(FULL, kk[4], 31);
+        lp = __shfl_sync(FULL, pp[4], 31);
         // the last run start among this lane's slots (offset in the step, -1
         // for none), its running maximum over the lanes, and from that the
         // first slot of the run that holds the slot before this lane's first

@@ -136,8 +136,8 @@ int bits_for(int64_t max_key)
 //   2. k_rs_chunk_sum / k_rs_chunk_scan / k_rs_chunk_down: the counts in
 //      digit-major order become the global output offset of each (tile,
 //      digit), computed hierarchically over chunks of 256 tiles;
-//   3. k_rs_scatter: each tile ranks its pairs stably (warp match on the
-//      digit, per-warp running counts, prefix over warps and digits), stages
+//   3. k_rs_scatter: each tile ranks its pairs stably (one ballot per
+//      digit bit, per-warp running counts, prefix over warps and digits), stages
 //      them in shared memory in output order, and writes every digit's run
 //      with consecutive threads.
 // Digits are D = 8..10 bits, equal for all passes (27-bit ids: 3 passes of 9).
@@ -157,10 +157,13 @@ __global__ __launch_bounds__(RS_THREADS) void k_rs_hist(const uint32_t *__restri
                                                          int *status)
 {
     constexpr int RADIX = 1 << D;
-    __shared__ uint32_t h[WARPS][RADIX];
+    // one count per digit for the block: shared-memory atomics on one address
+    // from different warps do not wait on each other, so per-warp copies would
+    // only add their clearing and summing
+    __shared__ uint32_t h[RADIX];
     __shared__ int s_desc;
     if (read_status(status)) return;
-    for (int i = threadIdx.x; i < WARPS * RADIX; i += RS_THREADS) (&h[0][0])[i] = 0;
+    for (int i = threadIdx.x; i < RADIX; i += RS_THREADS) h[i] = 0;
     if (threadIdx.x == 0) s_desc = 0;
     const int64_t tile0 = (int64_t)blockIdx.x * RS_TILE;
     const int ntile = (int)min64(RS_TILE, n - tile0);
@@ -188,17 +191,11 @@ __global__ __launch_bounds__(RS_THREADS) void k_rs_hist(const uint32_t *__restri
         }
     }
     __syncthreads();
-    const int warp = threadIdx.x >> 5;
 #pragma unroll
     for (int i = 0; i < RS_IPT; ++i)
-        if (i * RS_THREADS + (int)threadIdx.x < ntile) atomicAdd(&h[warp][(k[i] >> shift) & (RADIX - 1)], 1u);
+        if (i * RS_THREADS + (int)threadIdx.x < ntile) atomicAdd(&h[(k[i] >> shift) & (RADIX - 1)], 1u);
     __syncthreads();
-    for (int d = threadIdx.x; d < RADIX; d += RS_THREADS) {
-        uint32_t sum = 0;
-#pragma unroll
-        for (int w = 0; w < WARPS; ++w) sum += h[w][d];
-        hist[(int64_t)blockIdx.x * RADIX + d] = sum;
-    }
+    for (int d = threadIdx.x; d < RADIX; d += RS_THREADS) hist[(int64_t)blockIdx.x * RADIX + d] = h[d];
     if (range || descents) {
         for (int off = 16; off >= 1; off >>= 1) desc += __shfl_xor_sync(FULL, desc, off);
         if ((threadIdx.x & 31) == 0 && desc) atomicAdd(&s_desc, desc);
