@@ -403,8 +403,8 @@ const char *pdb_strerror(int code);
  *               caller-owned here).
  * Same arithmetic and result as pdb_sgd_epoch.  Set-up: the first call on
  * each device (and again after that device's context is reset) looks up
- * the array's device address with cudaGetSymbolAddress; make that first
- * call before any stream capture.  All calls on a device share the array,
+ * the array's device address with cudaGetSymbolAddress.  The call cannot be
+ * recorded into a CUDA graph (it synchronizes).  All calls on a device share the array,
  * which keeps the last call's contents (each call clears what must start at
  * zero): calls whose GPU work overlaps race, so order them on one stream.
  * SYNCHRONIZES `stream` (the status word is copied to the host) and returns
