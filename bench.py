@@ -220,9 +220,12 @@ def cpu_baseline(problem, target_s: float):
     return {"value": nnz / dt, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample}
 
 
-def recorded_traffic(kernel: str, workload: str):
+def recorded_traffic(kernel: str, workload: str, nnz: int):
     """DRAM bytes per launch from the committed ncu summary of this kernel and
-    workload, if the kernel sources still hash as they did when it was taken."""
+    workload, if the kernel sources still hash as they did when it was taken;
+    the record is for a launch over `traffic_nnz` nonzeros and scales to this
+    run's nonzeros in proportion (the summary shows the bytes per nonzero
+    holding across sizes)."""
     import hashlib
     import re
     path = os.path.join(ROOT, "profiles", f"{kernel}_{workload}.md")
@@ -231,15 +234,18 @@ def recorded_traffic(kernel: str, workload: str):
     except OSError:
         return None
     m_b = re.search(r"traffic_bytes_per_launch:\s*([0-9.eE+]+)", text)
+    m_n = re.search(r"traffic_nnz:\s*([0-9]+)", text)
     m_h = re.search(r"source_sha256:\s*([0-9a-f]{64})", text)
-    if not (m_b and m_h):
+    if not (m_b and m_n and m_h):
         return None
     h = hashlib.sha256()
     sources = {"k_sgd_window": "window.cu", "k_sgd_chain": "chain.cu"}.get(kernel, "sgd.cu")
     for f in (sources, "common.cuh"):
         with open(os.path.join(ROOT, "paper_1508_00703_gb300", "csrc", f), "rb") as fh:
             h.update(fh.read())
-    return float(m_b.group(1)) if h.hexdigest() == m_h.group(1) else None
+    if h.hexdigest() != m_h.group(1):
+        return None
+    return float(m_b.group(1)) * nnz / int(m_n.group(1))
 
 
 def training_loss(p, X, y, w, torch):
@@ -358,7 +364,7 @@ def run_ours(args, rank, world, local_rank):
              pdb.PDB_SCHED_CHAIN: "k_sgd_chain", pdb.PDB_SCHED_WINDOW: "k_sgd_window"}[resolved]
     roofline = {"kernel": kname,
                 "bound": "hbm", "achieved": round(sgd_gbs, 1), "peak": peak, "unit": "GB/s",
-                "frac": round(sgd_gbs / peak, 4), "traffic": recorded_traffic(kname, args.workload),
+                "frac": round(sgd_gbs / peak, 4), "traffic": recorded_traffic(kname, args.workload, p.nnz),
                 "peak_source": peak_kind,
                 "algorithmic_bytes_per_launch": sgd_bytes_per_launch, "launch_ms": round(sgd_launch_ms, 4),
                 "frac_of_8TBs": round(sgd_gbs / 8000.0, 4)}

@@ -88,7 +88,7 @@ def test_clock_summary_reads_samples_and_throttle_reasons(tmp_path):
 
 def test_recorded_traffic_only_while_the_sources_match(tmp_path, monkeypatch):
     # the committed ncu traffic is reported only while the kernel's sources
-    # hash as they did when it was captured
+    # hash as they did when it was captured, scaled to the run's nonzeros
     sys.path.insert(0, ROOT)
     import hashlib
     import bench
@@ -99,9 +99,10 @@ def test_recorded_traffic_only_while_the_sources_match(tmp_path, monkeypatch):
     (tmp_path / "profiles").mkdir()
     h = hashlib.sha256(b"kernel A\n" + b"helpers\n").hexdigest()
     (tmp_path / "profiles" / "k_sgd_window_low-conflict.md").write_text(
-        f"traffic_bytes_per_launch: 123456\nsource_sha256: {h}\n")
+        f"traffic_bytes_per_launch: 123456\ntraffic_nnz: 1000\nsource_sha256: {h}\n")
     monkeypatch.setattr(bench, "ROOT", str(tmp_path))
-    assert bench.recorded_traffic("k_sgd_window", "low-conflict") == 123456.0
+    assert bench.recorded_traffic("k_sgd_window", "low-conflict", 1000) == 123456.0
+    assert bench.recorded_traffic("k_sgd_window", "low-conflict", 100) == 12345.6
     (csrc / "window.cu").write_text("kernel B\n")
-    assert bench.recorded_traffic("k_sgd_window", "low-conflict") is None
-    assert bench.recorded_traffic("k_sgd_window", "zipf-1m") is None
+    assert bench.recorded_traffic("k_sgd_window", "low-conflict", 1000) is None
+    assert bench.recorded_traffic("k_sgd_window", "zipf-1m", 1000) is None
