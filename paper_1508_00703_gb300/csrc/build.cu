@@ -172,12 +172,15 @@ __device__ __forceinline__ void load_group(const uint32_t *__restrict__ skey, co
 // to the next, so a slot's rank is its distance to that slot without a
 // second pass over the keys; the run in progress where the range begins is
 // found once per warp by run_start.
-__global__ void k_slots(const uint32_t *__restrict__ skey, const int32_t *__restrict__ spos, int64_t nnz,
+constexpr int SLOTS_THREADS = 256;
+
+__global__ __launch_bounds__(SLOTS_THREADS) void k_slots(const uint32_t *__restrict__ skey, const int32_t *__restrict__ spos, int64_t nnz,
                         int64_t n_cols, int64_t *__restrict__ feat_ptr, const int64_t *__restrict__ row_ptr,
                         int64_t n_rows, int64_t near, uint32_t *__restrict__ gate, uint32_t *__restrict__ gsort,
                         uint32_t *__restrict__ gwin, int *info)
 {
     __shared__ bool s_check;
+    __shared__ __align__(16) uint32_t s_keys[SLOTS_THREADS / 32][128];   // each warp's step of keys
     if (threadIdx.x == 0) {
         long long all = 0, rows = 0;
         for (int i = 0; i < DESC_SPREAD; ++i) {
@@ -190,6 +193,7 @@ __global__ void k_slots(const uint32_t *__restrict__ skey, const int32_t *__rest
     if (read_status(info)) return;
     const bool check_dup = s_check;
     const int lane = threadIdx.x & 31;
+    uint32_t *sk = s_keys[threadIdx.x >> 5];
     const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
     const int64_t n_warps = ((int64_t)gridDim.x * blockDim.x) >> 5;
     const int64_t steps = (nnz + 127) >> 7;
@@ -287,12 +291,6 @@ __global__ void k_slots(const uint32_t *__restrict__ skey, const int32_t *__rest
             // before inside the lane's slots, else the distance to the run's
             // first slot
             r = first ? 0 : e > 0 ? r + 1 : s - before;
-            if (first) {
-                const int64_t hi = min((int64_t)j, n_cols);
-                for (int64_t b = s == 0 ? 0 : (int64_t)kk[e] + 1; b <= hi; ++b) feat_ptr[b] = s;
-            }
-            if (s == nnz - 1)
-                for (int64_t b = (int64_t)j + 1; b <= n_cols; ++b) feat_ptr[b] = nnz;
             const bool near_prev = r > 0 && (int64_t)p - pp[e] < near;
             const bool near_next = !last && (int64_t)pp[e + 2] - p < near;
             big |= r > (int64_t)GATE_RANK;
@@ -310,6 +308,30 @@ __global__ void k_slots(const uint32_t *__restrict__ skey, const int32_t *__rest
             else
                 for (int e = 0; e < 4 && s0 + e < nnz; ++e) gsort[s0 + e] = g[e];
         }
+        // feat_ptr[b] for the features b after the key before the step up to
+        // the step's last key: the first slot of the step whose key is >= b
+        // (a binary search in the step's keys), consecutive b on consecutive
+        // lanes so that the stores coalesce; after the last slot of all, n
+        *reinterpret_cast<uint4 *>(sk + lane * 4) = make_uint4(kk[1], kk[2], kk[3], kk[4]);
+        __syncwarp();
+        const int nv = (int)min((int64_t)128, nnz - base);
+        const uint32_t kb = __shfl_sync(FULL, kk[0], 0);
+        const int64_t khi = (int64_t)sk[nv - 1];
+        const int64_t bhi = min(khi, n_cols);
+        for (int64_t b = (base == 0 ? 0 : (int64_t)kb + 1) + lane; b <= bhi; b += 32) {
+            int lo = 0, hi = nv;
+            while (lo < hi) {
+                const int mid = (lo + hi) >> 1;
+                if ((int64_t)sk[mid] < b)
+                    lo = mid + 1;
+                else
+                    hi = mid;
+            }
+            feat_ptr[b] = base + lo;
+        }
+        if (base + nv == nnz)
+            for (int64_t b = khi + 1 + lane; b <= n_cols; b += 32) feat_ptr[b] = nnz;
+        __syncwarp();                              // sk is rewritten by the next step
     }
     for (int off = 16; off >= 1; off >>= 1) {
         longest = max(longest, __shfl_xor_sync(FULL, longest, off));
@@ -927,7 +949,7 @@ int pdb_build_conflicts(const pdb_csr *X, pdb_conflicts **out, void *stream)
     // k_slots writes feat_ptr; with no nonzeros every bound is 0
     if (rc == PDB_OK && nnz == 0) rc = segment_bounds(skey, 0, F, nullptr, c->feat_ptr, c->info, s);
     if (rc == PDB_OK && nnz > 0) {
-        k_slots<<<grid_1d((nnz + 3) / 4), 256, 0, s>>>(skey, c->csc_pos, nnz, F, c->feat_ptr, X->row_ptr, N,
+        k_slots<<<grid_1d((nnz + 3) / 4), SLOTS_THREADS, 0, s>>>(skey, c->csc_pos, nnz, F, c->feat_ptr, X->row_ptr, N,
                                                         c->near, c->gate, c->gate_sorted,
                                                         partition ? c->gate_window : nullptr, c->info);
         note_launch();
