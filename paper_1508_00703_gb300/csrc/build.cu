@@ -171,13 +171,18 @@ __device__ __forceinline__ void load_group(const uint32_t *__restrict__ skey, co
 // aligned), and carries the first slot of the run in progress from one step
 // to the next, so a slot's rank is its distance to that slot without a
 // second pass over the keys; the run in progress where the range begins is
-// found once per warp by run_start.
+// found once per warp by run_start.  feat_ptr is written per step, for the
+// features from the key before the step to the step's last key, with
+// consecutive features on consecutive lanes (stores that coalesce).
 constexpr int SLOTS_THREADS = 256;
 
-__global__ __launch_bounds__(SLOTS_THREADS) void k_slots(const uint32_t *__restrict__ skey, const int32_t *__restrict__ spos, int64_t nnz,
-                        int64_t n_cols, int64_t *__restrict__ feat_ptr, const int64_t *__restrict__ row_ptr,
-                        int64_t n_rows, int64_t near, uint32_t *__restrict__ gate, uint32_t *__restrict__ gsort,
-                        uint32_t *__restrict__ gwin, int *info)
+__global__ __launch_bounds__(SLOTS_THREADS) void k_slots(const uint32_t *__restrict__ skey,
+                                                         const int32_t *__restrict__ spos, int64_t nnz, int64_t n_cols,
+                                                         int64_t *__restrict__ feat_ptr,
+                                                         const int64_t *__restrict__ row_ptr, int64_t n_rows,
+                                                         int64_t near, uint32_t *__restrict__ gate,
+                                                         uint32_t *__restrict__ gsort, uint32_t *__restrict__ gwin,
+                                                         int *info)
 {
     __shared__ bool s_check;
     __shared__ __align__(16) uint32_t s_keys[SLOTS_THREADS / 32][128];   // each warp's step of keys
